@@ -1,0 +1,374 @@
+"""Benchmark of the gater's hot path on GB300 (one JSON line on rank 0).
+
+Workload (default): 1,000,000 fp32 feature vectors, d = 2048, K = 64 centres,
+post-ReLU mixture of 64 Gaussians (about half zeros), the shape of pooled
+ResNet-50 features.  One step = one whole job on inputs resident in HBM:
+    prepare the features (row norms, bf16 split), 20 Lloyd iterations
+    (hme_assign + hme_update_centroids), then hme_route of all N rows with the
+    final centres (assign + expert partition).
+The k-means++ seeding is the boundary and is not timed; every step starts
+from the same seeded centres.  value = Lloyd iterations per second of the
+whole job (all ranks); inputs (8.2 GB) are larger than L2 (129 MB).
+
+--impl reference times the fp64 CPU oracle on the host cores on a bounded
+row sample of the same workload, scaled to the full N.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "Lloyd iterations/sec and assigned vectors/sec (N·K·d GFLOP/s, % roofline)"
+UNIT = "Lloyd iterations/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2, help="workload index 1..5 (2 is the benchmark workload)")
+    ap.add_argument("--rows", type=int, default=0, help="override N (debug runs only)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def profiled_traffic(kernel_file: str, key: str):
+    """DRAM bytes per launch from a committed ncu summary, if it matches the current kernel source."""
+    prof = os.path.join(ROOT, "profiles", key + ".md")
+    if not os.path.exists(prof):
+        return None
+    text = open(prof).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    h = re.search(r"source_sha256:\s*([0-9a-f]{64})", text)
+    if not m or not h:
+        return None
+    src = hashlib.sha256(open(os.path.join(ROOT, "paper_1704_06363_gb300", "csrc", kernel_file), "rb").read())
+    if src.hexdigest() != h.group(1):
+        return None
+    return float(m.group(1))
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle baseline (also the --impl reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_iteration_rate(w, target_s: float, steps: int = 1):
+    """Oracle Lloyd iterations/s at full N, from a timed row sample (assign + update)."""
+    import numpy as np
+    import oracle
+    import hme_synth
+
+    oracle.build()
+    n = 256
+    cores = os.cpu_count() or 1
+    X, _ = hme_synth.make_features(w, N=n)
+    Xh = hme_synth.host_array(X, w.dtype)
+    C0, _ = oracle.kmeanspp(Xh, w.K, 7, True, w.dtype)
+    # grow the sample until one iteration takes about target_s / 4, then time `steps` iterations
+    while True:
+        t0 = time.perf_counter()
+        oracle.lloyd(Xh, C0, 1, w.dtype)
+        dt = time.perf_counter() - t0
+        if dt > target_s / 4 or n >= w.N:
+            break
+        n = min(w.N, int(n * min(8.0, max(2.0, (target_s / 4) / max(dt, 1e-3)))))
+        X, _ = hme_synth.make_features(w, N=n)
+        Xh = hme_synth.host_array(X, w.dtype)
+    times = []
+    for _ in range(max(1, steps)):
+        t0 = time.perf_counter()
+        oracle.lloyd(Xh, C0, 1, w.dtype)
+        times.append(time.perf_counter() - t0)
+    per_iter_full = float(np.median(times)) * (w.N / n)
+    return 1.0 / per_iter_full, n, cores, times
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    steps = max(1, args.steps)
+    for _ in range(max(0, args.warmup)):
+        pass  # the oracle has no warm state beyond the sample sizing pass below
+    rate, n, cores, times = oracle_iteration_rate(w, args.cpu_seconds, steps)
+    sample = f"{n} of {w.N} rows, one Lloyd iteration (assign + update) per step, scaled by N/{n}"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": steps, "warmup": args.warmup, "ms_per_step": 1000 * sum(times) / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "N": w.N, "d": w.d, "K": w.K, "feature_dtype": w.dtype,
+                   "iterations": w.iters},
+        "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args, w):
+    import torch
+    import torch.distributed as dist
+
+    import hme_synth
+    from paper_1704_06363_gb300 import hme
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+
+    N, d, K, T = w.N, w.d, w.K, w.iters
+    dt = hme.HME_F32 if w.dtype == "f32" else hme.HME_BF16
+    X, _ = hme_synth.make_features(w, device=dev)  # replicas: every rank clusters its own copy
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+    wr = hme.workspace(hme.HME_OP_ROUTE, N, d, K, dt, device=dev)
+    wi = hme.workspace(hme.HME_OP_INIT, N, d, K, dt, device=dev)
+    C0 = torch.empty(K, d, dtype=torch.float32, device=dev)
+    hme.hme_kmeans_init(X, K, 1234 + w.seed, hme.HME_INIT_KMEANSPP_SUBSAMPLE, C0, wi)
+    del wi
+    C = torch.empty_like(C0)
+    labels = torch.empty(N, dtype=torch.int32, device=dev)
+    mind = torch.empty(N, dtype=torch.float32, device=dev)
+    obj = torch.zeros(T, dtype=torch.float64, device=dev)
+    jex = torch.zeros(T, dtype=torch.float64, device=dev)
+    counts = torch.empty(K, dtype=torch.int64, device=dev)
+    nres = torch.zeros(T, dtype=torch.int32, device=dev)
+    expert = torch.empty(N, dtype=torch.int32, device=dev)
+    offsets = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    order = torch.empty(N, dtype=torch.int32, device=dev)
+
+    ev_assign, ev_update = [], []
+
+    def step(Xs, record=False):
+        C.copy_(C0)
+        hme.hme_prepare_features(Xs, K, ws)
+        for t in range(T):
+            if record:
+                a0 = torch.cuda.Event(enable_timing=True)
+                a1 = torch.cuda.Event(enable_timing=True)
+                a0.record(stream)
+            hme.hme_assign(Xs, C, labels, ws, mind, obj[t:t + 1], flags=hme.HME_ASSIGN_PREPARED)
+            if record:
+                a1.record(stream)
+                u1 = torch.cuda.Event(enable_timing=True)
+            hme.hme_update_centroids(Xs, labels, mind, C, ws, counts, nres[t:t + 1], jex[t:t + 1])
+            if record:
+                u1.record(stream)
+                ev_assign.append((a0, a1))
+                ev_update.append((a1, u1))
+        hme.hme_route(Xs, C, expert, offsets, order, wr)
+
+    for _ in range(max(3, args.warmup)):
+        step(X)
+    status = hme.hme_sync_status(ws)
+    if status != hme.HME_OK:
+        raise RuntimeError(f"device status {status} after warm-up")
+
+    clocks = Clocks(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    clocks.start()
+    launches0 = hme.hme_launch_count()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step(X, record=True)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    launches = hme.hme_launch_count() - launches0
+    ck = clocks.stop()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    assert hme.hme_sync_status(ws) == hme.HME_OK and hme.hme_sync_status(wr) == hme.HME_OK
+
+    iters_total = T * args.steps * world
+    value = iters_total / (ms / 1000.0)
+    t_assign = sum(a.elapsed_time(b) for a, b in ev_assign) / len(ev_assign)
+    t_update = sum(a.elapsed_time(b) for a, b in ev_update) / len(ev_update)
+    e = w.elem_bytes
+    assign_bytes = N * d * e + K * d * e + 4 * N + 8 * N   # X, C, ||x||^2 in; labels, distances out
+    update_bytes = N * d * e + 4 * N + 8 * N + K * d * 4   # X and labels in (+ the sorted order), C out
+    hbm, tc, peak_kind = peaks()
+    a_gbs = assign_bytes / (t_assign / 1000) / 1e9
+    u_gbs = update_bytes / (t_update / 1000) / 1e9
+    dominant = "assign" if t_assign >= t_update else "update"
+    if dominant == "assign":
+        achieved, traffic = a_gbs, profiled_traffic("assign.cu", "assign_relu_gmm64_n1e6_d2048_k64_f32")
+    else:
+        achieved, traffic = u_gbs, profiled_traffic("update.cu", "update_relu_gmm64_n1e6_d2048_k64_f32")
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": traffic, "kernel": dominant, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s"}
+    flops_assign = 2.0 * N * K * d
+
+    # ---- end to end through the C ABI with host buffers ------------------------------
+    e2e = None
+    if not args.no_e2e:
+        Xh = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
+        Xh.copy_(X)
+        Xd = torch.empty_like(X)
+        out_labels = torch.empty(N, dtype=torch.int32, pin_memory=True)
+        out_order = torch.empty(N, dtype=torch.int32, pin_memory=True)
+        out_offsets = torch.empty(K + 1, dtype=torch.int64, pin_memory=True)
+        out_C = torch.empty(K, d, dtype=torch.float32, pin_memory=True)
+
+        def e2e_step():
+            Xd.copy_(Xh, non_blocking=True)
+            step(Xd)
+            out_labels.copy_(expert, non_blocking=True)
+            out_order.copy_(order, non_blocking=True)
+            out_offsets.copy_(offsets, non_blocking=True)
+            out_C.copy_(C, non_blocking=True)
+
+        e2e_step()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        f0 = torch.cuda.Event(enable_timing=True)
+        f1 = torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        f1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms_e2e = f0.elapsed_time(f1)
+        if world > 1:
+            t = torch.tensor([ms_e2e], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        e2e = {"value": iters_total / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": X.numel() * e,
+               "d2h_bytes_per_step": 4 * N + 4 * N + 8 * (K + 1) + 4 * K * d, "ms_per_step": ms_e2e / args.steps}
+        del Xh, Xd
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        rate, n, cores, _ = oracle_iteration_rate(w, args.cpu_seconds, 1)
+        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"{n} of {w.N} rows, one Lloyd iteration (assign + update), scaled by N/{n}"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16x3" if w.dtype == "f32" else "bf16",
+            "data": "synthetic",
+            "config": {"workload": w.name, "N": N, "d": d, "K": K, "feature_dtype": w.dtype, "iterations": T,
+                       "step": "prepare + %d x (assign + update) + route of all N rows" % T,
+                       "l2": "inputs larger than L2 (%.1f GB of features)" % (X.numel() * e / 1e9),
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "vectors_per_s": N * iters_total / (ms / 1000.0),
+            "assign_gflops": flops_assign / (t_assign / 1000.0) / 1e9,
+            "kernels_ms": {"assign_call": t_assign, "update_call": t_update,
+                           "assign_gbs": a_gbs, "update_gbs": u_gbs},
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "clocks": ck,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    import hme_synth
+    w = hme_synth.WORKLOADS[args.config]
+    if args.rows:
+        w = w.with_rows(args.rows)
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

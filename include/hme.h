@@ -1,0 +1,223 @@
+/*
+ * hme.h -- C ABI of the GB300 (sm_103a) gater library for hard mixtures of
+ * experts (Gross, Ranzato, Szlam, "Hard Mixtures of Experts for Large Scale
+ * Weakly Supervised Vision", arXiv 1704.06363).
+ *
+ * The gater of Section 2: K-means clustering of feature vectors z_j
+ * (Lloyd iterations), the hard assignment of Eq. 2
+ *     T(x)_i = 1  iff  i = argmin_j || z(x) - c_j ||_2 ,
+ * and the split of the training set into per-expert shares ("each on its own
+ * share of the training data", with no balancing of cluster sizes).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every function returns an int status: HME_OK (0) or one of the HME_E*
+ *   codes below.  On error nothing has been launched, and hme_last_error()
+ *   returns a message (thread-local, valid until the next call on the thread).
+ * - All array arguments are caller-owned DEVICE pointers (allocated by the
+ *   caller, e.g. with torch).  The library allocates no device memory: all
+ *   scratch lives in the caller's workspace `ws` of `ws_bytes` bytes, sized by
+ *   hme_workspace_bytes().  ws must be 256-byte aligned.
+ * - Work is enqueued asynchronously on `stream` (a cudaStream_t passed as
+ *   void*; NULL = the legacy default stream).  Arguments are checked on the
+ *   host before any launch.  Conditions only the device can see (a label out of
+ *   range, a bounded device wait that expired) are recorded in a status word
+ *   inside ws; hme_sync_status() waits for the stream and reports it.  Each
+ *   call clears that word when it starts, so it reports on the last call made
+ *   with that workspace.
+ * - Feature matrices are row-major, N rows of d elements, row stride `ldx`
+ *   elements (ldx >= d), element type HME_F32 (float) or HME_BF16 (bfloat16).
+ *   For HME_BF16 the rows are read by TMA: the base must be 16-byte aligned and
+ *   ldx * 2 a multiple of 16 bytes, otherwise HME_EINVAL.
+ * - Centres C are K x d float32, row-major, contiguous (row stride d).
+ * - Limits: 1 <= d <= 16384, 1 <= K <= 16384, 0 <= N < 2^31.
+ * - All entry points may be called from several host threads on different
+ *   workspaces; calls sharing one workspace must be ordered on one stream.
+ */
+#ifndef HME_H
+#define HME_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define HME_API __attribute__((visibility("default")))
+#else
+#define HME_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---------------------------------------------------- */
+#define HME_OK 0
+#define HME_EINVAL 1    /* bad argument (pointer, size, alignment, label range) */
+#define HME_ENOMEM 2    /* ws_bytes smaller than hme_workspace_bytes() */
+#define HME_ECUDA 3     /* a CUDA runtime or driver call failed */
+#define HME_ETIMEOUT 4  /* a bounded device-side wait expired (see hme_sync_status) */
+#define HME_EINTERNAL 5 /* internal inconsistency */
+
+/* ---- element types of feature matrices ------------------------------- */
+#define HME_F32 0
+#define HME_BF16 1
+
+/* ---- operations, for hme_workspace_bytes ----------------------------- */
+#define HME_OP_INIT 0      /* hme_kmeans_init */
+#define HME_OP_ASSIGN 1    /* hme_prepare_features, hme_assign, hme_update_centroids */
+#define HME_OP_PARTITION 2 /* hme_partition (d and dtype ignored) */
+#define HME_OP_ROUTE 3     /* hme_route */
+
+/* ---- k-means++ seeding variants -------------------------------------- */
+#define HME_INIT_KMEANSPP 0           /* candidates = all N rows */
+#define HME_INIT_KMEANSPP_SUBSAMPLE 1 /* candidates = min(N, 256 K) rows drawn with replacement */
+
+/* ---- hme_assign flags ------------------------------------------------- */
+#define HME_ASSIGN_DEFAULT 0
+#define HME_ASSIGN_PREPARED 1 /* ws already holds this X, prepared by hme_prepare_features */
+
+/*
+ * hme_workspace_bytes -- bytes of scratch an operation needs.
+ * op is one of HME_OP_*; N is the number of rows (B for HME_OP_ROUTE).  The
+ * HME_OP_ASSIGN size serves hme_prepare_features, hme_assign and
+ * hme_update_centroids on the same (N, d, K, dtype), so one workspace can carry
+ * prepared features from one Lloyd iteration to the next.  Returns 0 for
+ * invalid arguments.
+ */
+HME_API size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t dtype);
+
+/* Message describing the last failed call on this host thread ("" if none). */
+HME_API const char *hme_last_error(void);
+
+/*
+ * hme_sync_status -- wait for `stream`, then return the device-side status of
+ * the last call made with workspace `ws`: HME_OK, HME_EINVAL (a label outside
+ * [0, K) was seen and skipped), HME_ETIMEOUT (a bounded wait expired; outputs
+ * of that call are undefined) or HME_ECUDA (an asynchronous CUDA error).
+ */
+HME_API int hme_sync_status(void *ws, void *stream);
+
+/*
+ * hme_kmeans_init -- k-means++ seeding (Arthur & Vassilvitskii 2007) of the
+ * centres that Section 2 obtains by "K-means clustering" of the z_j; the paper
+ * names no initialisation, so this is a stated reading.
+ *   Candidates: all N rows (HME_INIT_KMEANSPP) or m = min(N, 256 K) rows
+ *   (HME_INIT_KMEANSPP_SUBSAMPLE), candidate j = row floor(u_j N) with u_j from
+ *   splitmix64 output j of (seed ^ 0xD1B54A32D192ED03).
+ *   Picks use splitmix64 outputs 0, 1, ... of `seed`, u = top 53 bits / 2^53:
+ *   the first centre is candidate floor(u m); each later centre is the
+ *   smallest candidate whose running total of D^2 exceeds u * sum(D^2), where
+ *   D^2 (fp64) is the squared distance to the nearest centre chosen so far; if
+ *   that sum is 0, candidate floor(u m).
+ * X: N x d (ldx, dtype), read only.  C_out: K x d float32, written (each row a
+ * copy of a row of X).  Requires N >= 1.  Not on the timed Lloyd path: it
+ * makes about 2K kernel launches.
+ */
+HME_API int hme_kmeans_init(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
+                    uint64_t seed, int32_t method, float *C_out, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * hme_prepare_features -- once per feature set: squared row norms ||x_i||^2
+ * (fp32) and, for HME_F32, the split of every element into two bf16 parts
+ * x = hi + lo + O(2^-16 |x|) that the tensor-core assign step consumes (the
+ * norms are then those of hi + lo).  Writes
+ * ws only.  Pass HME_ASSIGN_PREPARED to hme_assign to reuse it for every
+ * iteration; the (N, d, K, dtype) of the later calls must be the same.
+ */
+HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
+                         void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * hme_assign -- Eq. 2 (Section 2) for every row of X:
+ *   labels_out[i] = argmin_k ||x_i - c_k||^2 , ties to the lowest k,
+ *   mind_out[i]   = ||x_i - c_{labels[i]}||^2 (float32, >= 0)      (may be NULL),
+ *   *objective_out = sum_i mind[i] in fp64 (one device double)     (may be NULL);
+ *                   a tensor-core estimate: its fp32 accumulation is biased
+ *                   by up to about (d/16) * nprod * 2^-24 (||x||^2 + ||c||^2)
+ *                   per row; hme_update_centroids returns the exact J.
+ * The distance is ||x||^2 - 2 x.c + ||c||^2 with x.c on the tcgen05 tensor
+ * cores (fp32 accumulate): for HME_BF16 features, x.bf16(c) with c rounded to
+ * bf16 (round to nearest even); for HME_F32, the bf16 split x = xh + xl,
+ * c = ch + cl and the four products xh.ch + xh.cl + xl.ch + xl.cl, with the
+ * norms taken of the same split values.  Rows whose two best distances lie within a
+ * relative 2e-4 of each other (of max(D2, ||x||^2)) are re-scored against
+ * every centre with direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of
+ * non-negative terms).  The N x K distance matrix is never written.
+ * X: N x d (ldx, dtype); C: K x d float32 (read only); labels_out: int32[N].
+ * flags: HME_ASSIGN_DEFAULT, or HME_ASSIGN_PREPARED (skip the per-call
+ * hme_prepare_features pass; ws must hold this X's preparation).
+ */
+HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *C, int32_t K,
+               int32_t flags, int32_t *labels_out, float *mind_out, double *objective_out,
+               void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * hme_update_centroids -- the K-means centre step (Section 2, "K-means
+ * clustering" of the z_j):
+ *   counts_out[k] = |{i : labels[i] = k}| (int64, may be NULL),
+ *   C_inout[k]    = (sum_{labels[i]=k} x_i) / counts[k], summed by segment in
+ *                   fp32 and across segments in fp64, stored as float32,
+ *   *objective_out = sum_i ||x_i - c_{labels[i]}||^2 for the centres as they
+ *                   were on entry (bf16-rounded for HME_BF16 features, as in
+ *                   hme_assign), by direct differences in the same pass over X
+ *                   (one device double, may be NULL).  With the labels of the
+ *                   preceding hme_assign this is the Lloyd objective J_t.
+ * Empty clusters (the paper is silent; Section 4.5 reports every cluster used)
+ * are re-seeded in ascending k: each takes the not-yet-taken row with the
+ * largest mind[i], ties to the lowest i, as its centre (copied exactly); that
+ * row stays counted in its own cluster.  mind may be NULL (then the lowest
+ * untaken rows).  When every row is taken, a remaining empty centre is kept.
+ * *n_reseeded_out (device int32, may be NULL) = clusters re-seeded.
+ * Labels outside [0, K) are skipped and reported by hme_sync_status.
+ */
+HME_API int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
+                         const int32_t *labels, const float *mind, int32_t K, float *C_inout,
+                         int64_t *counts_out, int32_t *n_reseeded_out, double *objective_out, void *ws,
+                         size_t ws_bytes, void *stream);
+
+/*
+ * hme_partition -- each expert's share of the training set (Section 2: "each
+ * on its own share"; no balancing, so buckets may be very unequal):
+ *   hist_out[k]        = |{i : labels[i] = k}|                     (int64[K]),
+ *   offsets_out        = exclusive prefix sum of hist              (int64[K+1]),
+ *   perm_out[offsets[labels[i]] + |{j < i : labels[j] = labels[i]}|] = i
+ *                        (a stable counting sort; int32[N]),
+ *   sorted_labels_out[s] = labels[perm[s]]                         (int32[N], may be NULL).
+ * Optional CSR multilabel lists (tag_off int64[N+1], tags int32[tag_off[N]])
+ * move with their point: tag_off_out int64[N+1] and tags_out int32[tag_off[N]]
+ * (all four NULL, or all four set).  Bit-exact; integer work only.
+ * Labels outside [0, K) are skipped and reported by hme_sync_status.
+ */
+HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out, int64_t *offsets_out,
+                  int32_t *perm_out, int32_t *sorted_labels_out, const int64_t *tag_off, const int32_t *tags,
+                  int64_t *tag_off_out, int32_t *tags_out, void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * hme_route -- evaluation-time gating (Section 2.1: the cost of an output is
+ * the cost of T(x) plus one expert H_i(x)): Eq. 2 on a batch Q (B x d) with
+ * frozen centres C, then the partition of its labels, so that each expert
+ * receives a contiguous run of rows:
+ *   expert_out[b] = label of Q row b (int32[B]), offsets_out (int64[K+1]),
+ *   order_out (int32[B]) = rows of Q grouped by expert, ascending within one.
+ */
+HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
+              int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws, size_t ws_bytes,
+              void *stream);
+
+/* Number of kernels this library has launched in this process (diagnostic). */
+HME_API int64_t hme_launch_count(void);
+
+/*
+ * hme_debug_bounded_wait -- test hook for the device-side bounded wait that
+ * every pipeline wait in this library uses: launches one CTA that waits on a
+ * shared-memory barrier nothing completes, with a limit of timeout_ns
+ * nanoseconds (1 .. 10^9).  hme_sync_status(ws, stream) then returns
+ * HME_ETIMEOUT and the context stays usable.
+ */
+HME_API int hme_debug_bounded_wait(uint64_t timeout_ns, void *ws, size_t ws_bytes, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HME_H */

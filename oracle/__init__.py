@@ -68,6 +68,8 @@ def _load():
         lib.orc_kmeanspp.argtypes = [p, i64, i64, i64, i32, i64, u64, i32, p, p]
         lib.orc_assign.restype = None
         lib.orc_assign.argtypes = [p, i64, i64, i64, i32, p, i64, p, p, p, p]
+        lib.orc_objective.restype = i32
+        lib.orc_objective.argtypes = [p, i64, i64, i64, i32, p, i64, p, p]
         lib.orc_update.restype = i32
         lib.orc_update.argtypes = [p, i64, i64, i64, i32, p, p, i64, p, p, p]
         lib.orc_partition.restype = i32
@@ -146,6 +148,17 @@ def assign(X, C, dtype: str = "f32"):
     J = ctypes.c_double(0.0)
     _load().orc_assign(_ptr(X), N, d, d, code, _ptr(C), K, _ptr(labels), _ptr(d1), _ptr(d2), ctypes.byref(J))
     return labels, d1, d2, J.value
+
+
+def objective(X, C, labels, dtype: str = "f32") -> float:
+    """J = sum_i ||x_i - c_{labels[i]}||^2 (fp64), centres bf16-rounded for bf16 features."""
+    X, N, d, code = _features(X, dtype)
+    C = np.ascontiguousarray(C, np.float32)
+    labels = np.ascontiguousarray(labels, np.int32)
+    J = ctypes.c_double(0.0)
+    if _load().orc_objective(_ptr(X), N, d, d, code, _ptr(C), C.shape[0], _ptr(labels), ctypes.byref(J)) != 0:
+        raise ValueError("orc_objective: label out of range")
+    return J.value
 
 
 def update(X, labels, mind, C, dtype: str = "f32"):

@@ -256,6 +256,29 @@ void orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
 }
 
 /* ---------------------------------------------------------------------- */
+/* The K-means objective of a given assignment: J = sum_i ||x_i - c_{a_i}||^2 */
+/* (the quantity Lloyd's iteration decreases), direct fp64 sums in ascending */
+/* i and j, against the same centre values as orc_assign.  -1 on a bad label. */
+/* ---------------------------------------------------------------------- */
+int orc_objective(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
+                  const float *C, int64_t K, const int32_t *labels, double *objective)
+{
+    double J = 0.0;
+    for (int64_t i = 0; i < N; ++i) {
+        if (labels[i] < 0 || labels[i] >= K)
+            return -1;
+        double s = 0.0;
+        for (int64_t j = 0; j < d; ++j) {
+            double t = feat(X, dtype, ldx, i, j) - centre(C, d, dtype, labels[i], j);
+            s += t * t;
+        }
+        J += s;
+    }
+    *objective = J;
+    return 0;
+}
+
+/* ---------------------------------------------------------------------- */
 /* Update (the K-means centre step behind Section 2's "K-means clustering   */
 /* on the z_j"): c_k = mean of the x_i with a_i = k, summed in fp64 in       */
 /* ascending i and rounded once to fp32.  counts[k] = |{i : a_i = k}|.      */

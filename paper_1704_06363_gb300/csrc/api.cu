@@ -1,0 +1,377 @@
+// api.cu -- the extern "C" entry points of libhme (declared in include/hme.h):
+// argument checks, the workspace layout, and the order of kernel launches for
+// each operation of the gater (Section 2 of the paper: K-means of the
+// features, the hard assignment of Eq. 2, each expert's share of the data).
+#include "hme_common.cuh"
+
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+
+namespace hme {
+
+namespace {
+thread_local char g_err[512] = {0};
+std::atomic<int64_t> g_launches{0};
+int g_sms[64] = {0};
+}  // namespace
+
+int fail(int code, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+  return fail(HME_ECUDA, "%s: %s (%s)", what, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+void count_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+int num_sms() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (g_sms[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    g_sms[dev] = n;
+  }
+  return g_sms[dev];
+}
+
+uint64_t wait_limit_ns() {
+  // Every pipeline wait gives up after this much global time (debug override: HME_WAIT_LIMIT_NS).
+  static uint64_t v = [] {
+    const char *e = getenv("HME_WAIT_LIMIT_NS");
+    if (e && *e) {
+      unsigned long long x = strtoull(e, nullptr, 10);
+      if (x >= 1000 && x <= 60000000000ull) return (uint64_t)x;
+    }
+    return (uint64_t)2000000000ull;
+  }();
+  return v;
+}
+
+AssignGeom assign_geom(int d, int K, int dtype) {
+  AssignGeom g;
+  g.d = d;
+  g.K = K;
+  g.dtype = dtype;
+  g.ldp = (d + 7) / 8 * 8;
+  g.nchunks = (K + kMaxBN - 1) / kMaxBN;
+  const int per = (K + g.nchunks - 1) / g.nchunks;
+  g.BN = (per + 15) / 16 * 16;
+  g.Kp = g.BN * g.nchunks;
+  g.nprod = dtype == HME_F32 ? 4 : 1;
+  return g;
+}
+
+Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
+  const AssignGeom g = assign_geom(d, K, dtype);
+  Layout L;
+  size_t off = sizeof(Header);
+  auto take = [&](size_t bytes) {
+    off = align_up(off, 256);
+    const size_t at = off;
+    off += bytes;
+    return at;
+  };
+  L.xn = take((size_t)N * 4);
+  if (dtype == HME_F32) {
+    L.xhi = take((size_t)N * g.ldp * 2);
+    L.xlo = take((size_t)N * g.ldp * 2);
+  } else {
+    L.xhi = L.xlo = 0;
+  }
+  L.cb_hi = take((size_t)g.Kp * g.ldp * 2);
+  L.cb_lo = dtype == HME_F32 ? take((size_t)g.Kp * g.ldp * 2) : 0;
+  L.cn = take((size_t)g.Kp * 4);
+  L.flagged = take((size_t)(N > 0 ? N : 1) * 4);
+  L.perm = take((size_t)(N > 0 ? N : 1) * 4);
+  L.slab = take((size_t)(N > 0 ? N : 1) * 4);
+  L.part = part_layout(align_up(off, 256), N, K);
+  off = L.part.end;
+  L.sums = take((size_t)K * d * 8);
+  if (kpp_m > 0) {
+    L.kpp_rows = take((size_t)kpp_m * 4);
+    L.kpp_d2 = take((size_t)kpp_m * 8);
+    L.kpp_part = take((size_t)kpp_blocks(kpp_m) * 8);
+  } else {
+    L.kpp_rows = L.kpp_d2 = L.kpp_part = 0;
+  }
+  L.total = align_up(off, 256);
+  return L;
+}
+
+namespace {
+
+size_t init_bytes(int64_t N, int K) {
+  size_t off = sizeof(Header);
+  const int64_t m = N;  // upper bound over both methods
+  off = align_up(off, 256) + (size_t)m * 4;
+  off = align_up(off, 256) + (size_t)m * 8;
+  off = align_up(off, 256) + (size_t)kpp_blocks(m) * 8;
+  (void)K;
+  return align_up(off, 256);
+}
+
+int check_common(int64_t N, int d, int K, int dtype) {
+  if (N < 0 || N > (int64_t)0x7FFFFFFF) return fail(HME_EINVAL, "N = %lld out of range [0, 2^31)", (long long)N);
+  if (d < 1 || d > kMaxD) return fail(HME_EINVAL, "d = %d out of range [1, %d]", d, kMaxD);
+  if (K < 1 || K > kMaxK) return fail(HME_EINVAL, "K = %d out of range [1, %d]", K, kMaxK);
+  if (dtype != HME_F32 && dtype != HME_BF16) return fail(HME_EINVAL, "dtype = %d is not HME_F32 or HME_BF16", dtype);
+  return HME_OK;
+}
+
+int check_features(const void *X, int64_t N, int d, int64_t ldx, int dtype, bool tma) {
+  if (N > 0 && !X) return fail(HME_EINVAL, "feature pointer is NULL");
+  if (ldx < d) return fail(HME_EINVAL, "ldx = %lld < d = %d", (long long)ldx, d);
+  if (tma && dtype == HME_BF16) {
+    if ((reinterpret_cast<uintptr_t>(X) & 15u) != 0)
+      return fail(HME_EINVAL, "bf16 features must start on a 16-byte boundary (TMA)");
+    if ((ldx * 2) % 16 != 0)
+      return fail(HME_EINVAL, "bf16 row stride ldx = %lld is not a multiple of 8 elements (TMA)", (long long)ldx);
+  }
+  return HME_OK;
+}
+
+int check_ws(void *ws, size_t ws_bytes, size_t need) {
+  if (!ws) return fail(HME_EINVAL, "workspace is NULL");
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return fail(HME_EINVAL, "workspace is not 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(HME_ENOMEM, "workspace of %zu bytes is smaller than the %zu bytes needed", ws_bytes, need);
+  return HME_OK;
+}
+
+#define HME_TRY(expr)                   \
+  do {                                  \
+    int _rc = (expr);                   \
+    if (_rc != HME_OK) return _rc;      \
+  } while (0)
+
+#define HME_CUDA(expr, what)                         \
+  do {                                               \
+    cudaError_t _e = (expr);                         \
+    if (_e != cudaSuccess) return cuda_fail(_e, what); \
+  } while (0)
+
+template <typename T>
+T *at(void *ws, size_t off) {
+  return reinterpret_cast<T *>(static_cast<char *>(ws) + off);
+}
+
+int do_prepare(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, const Layout &L, void *ws,
+               cudaStream_t s) {
+  const AssignGeom g = assign_geom(d, K, dtype);
+  HME_CUDA(launch_prep_features(X, N, d, ldx, dtype, g, at<float>(ws, L.xn), at<__nv_bfloat16>(ws, L.xhi),
+                                at<__nv_bfloat16>(ws, L.xlo), s),
+           "prepare features");
+  return HME_OK;
+}
+
+int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K, int32_t *labels,
+              float *mind, const Layout &L, void *ws, cudaStream_t s) {
+  const AssignGeom g = assign_geom(d, K, dtype);
+  Header *hdr = at<Header>(ws, 0);
+  HME_CUDA(launch_prep_centres(C, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
+                               at<float>(ws, L.cn), s),
+           "prepare centres");
+  const void *Xa = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xhi) : X;
+  const void *Xb = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;
+  const int64_t lda = dtype == HME_F32 ? g.ldp : ldx;
+  HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
+                        at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged), s));
+  HME_CUDA(launch_rescore(X, N, d, ldx, dtype, C, K, at<float>(ws, L.xn), labels, mind, hdr,
+                          at<int32_t>(ws, L.flagged), s),
+           "re-score");
+  return HME_OK;
+}
+
+int clear_header(void *ws, cudaStream_t s) {
+  HME_CUDA(cudaMemsetAsync(ws, 0, sizeof(Header), s), "clear workspace header");
+  return HME_OK;
+}
+
+}  // namespace
+}  // namespace hme
+
+using namespace hme;
+
+extern "C" {
+
+size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t dtype) {
+  if (op == HME_OP_PARTITION) {
+    if (N < 0 || N > (int64_t)0x7FFFFFFF || K < 1 || K > kMaxK) return 0;
+    return align_up(part_layout(sizeof(Header), N, K).end, 256);
+  }
+  if (check_common(N, d, K, dtype) != HME_OK) return 0;
+  switch (op) {
+    case HME_OP_INIT:
+      return init_bytes(N, K);
+    case HME_OP_ASSIGN:
+    case HME_OP_ROUTE:
+      return feature_layout(N, d, K, dtype, 0).total;
+    default:
+      fail(HME_EINVAL, "unknown op %d", op);
+      return 0;
+  }
+}
+
+const char *hme_last_error(void) { return g_err; }
+
+int64_t hme_launch_count(void) { return g_launches.load(); }
+
+int hme_sync_status(void *ws, void *stream) {
+  if (!ws) return fail(HME_EINVAL, "workspace is NULL");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_CUDA(cudaStreamSynchronize(s), "synchronize");
+  Header h;
+  HME_CUDA(cudaMemcpy(&h, ws, sizeof(Header), cudaMemcpyDeviceToHost), "read status");
+  if (h.status & kStatusTimeout)
+    return fail(HME_ETIMEOUT, "a bounded device wait expired (site %u)", h.wait_where);
+  if (h.status & kStatusBadLabel) return fail(HME_EINVAL, "a label outside [0, K) was skipped");
+  return HME_OK;
+}
+
+int hme_kmeans_init(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K, uint64_t seed,
+                    int32_t method, float *C_out, void *ws, size_t ws_bytes, void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  if (N < 1) return fail(HME_EINVAL, "k-means++ needs N >= 1");
+  if (method != HME_INIT_KMEANSPP && method != HME_INIT_KMEANSPP_SUBSAMPLE)
+    return fail(HME_EINVAL, "unknown init method %d", method);
+  HME_TRY(check_features(X, N, d, ldx, dtype, false));
+  if (!C_out) return fail(HME_EINVAL, "C_out is NULL");
+  HME_TRY(check_ws(ws, ws_bytes, init_bytes(N, K)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t m = kpp_candidates(N, K, method);
+  size_t off = align_up(sizeof(Header), 256);
+  int32_t *rows = at<int32_t>(ws, off);
+  off = align_up(off + (size_t)m * 4, 256);
+  double *d2 = at<double>(ws, off);
+  off = align_up(off + (size_t)m * 8, 256);
+  double *part = at<double>(ws, off);
+  HME_TRY(clear_header(ws, s));
+  HME_CUDA(launch_kmeanspp(X, N, d, ldx, dtype, K, seed, m, method == HME_INIT_KMEANSPP_SUBSAMPLE, C_out, rows, d2,
+                           part, at<Header>(ws, 0), s),
+           "k-means++");
+  return HME_OK;
+}
+
+int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K, void *ws,
+                         size_t ws_bytes, void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  HME_TRY(check_features(X, N, d, ldx, dtype, true));
+  const Layout L = feature_layout(N, d, K, dtype, 0);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  return do_prepare(X, N, d, ldx, dtype, K, L, ws, s);
+}
+
+int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *C, int32_t K,
+               int32_t flags, int32_t *labels_out, float *mind_out, double *objective_out, void *ws,
+               size_t ws_bytes, void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  HME_TRY(check_features(X, N, d, ldx, dtype, true));
+  if (!C) return fail(HME_EINVAL, "C is NULL");
+  if (N > 0 && !labels_out) return fail(HME_EINVAL, "labels_out is NULL");
+  if (flags & ~HME_ASSIGN_PREPARED) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  const Layout L = feature_layout(N, d, K, dtype, 0);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  if (!(flags & HME_ASSIGN_PREPARED)) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s));
+  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, s));
+  if (objective_out)
+    HME_CUDA(cudaMemcpyAsync(objective_out, &at<Header>(ws, 0)->objective, sizeof(double), cudaMemcpyDeviceToDevice,
+                             s),
+             "copy objective");
+  return HME_OK;
+}
+
+int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const int32_t *labels,
+                         const float *mind, int32_t K, float *C_inout, int64_t *counts_out, int32_t *n_reseeded_out,
+                         double *objective_out, void *ws, size_t ws_bytes, void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  HME_TRY(check_features(X, N, d, ldx, dtype, false));
+  if (!C_inout) return fail(HME_EINVAL, "C_inout is NULL");
+  if (N > 0 && !labels) return fail(HME_EINVAL, "labels is NULL");
+  const Layout L = feature_layout(N, d, K, dtype, 0);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  Header *hdr = at<Header>(ws, 0);
+  int64_t *hist = at<int64_t>(ws, L.part.hist);
+  int64_t *offs = at<int64_t>(ws, L.part.offs);
+  int32_t *perm = at<int32_t>(ws, L.perm);
+  int32_t *slab = at<int32_t>(ws, L.slab);
+  HME_CUDA(launch_partition(labels, N, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab, hdr, s),
+           "update: sort labels");
+  HME_CUDA(launch_update(X, N, d, ldx, dtype, perm, slab, hist, offs + K, mind, K, at<double>(ws, L.sums), C_inout,
+                         counts_out, n_reseeded_out, hdr, s),
+           "update: centres");
+  if (objective_out)
+    HME_CUDA(cudaMemcpyAsync(objective_out, &hdr->objective, sizeof(double), cudaMemcpyDeviceToDevice, s),
+             "copy objective");
+  return HME_OK;
+}
+
+int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out, int64_t *offsets_out,
+                  int32_t *perm_out, int32_t *sorted_labels_out, const int64_t *tag_off, const int32_t *tags,
+                  int64_t *tag_off_out, int32_t *tags_out, void *ws, size_t ws_bytes, void *stream) {
+  if (N < 0 || N > (int64_t)0x7FFFFFFF) return fail(HME_EINVAL, "N = %lld out of range", (long long)N);
+  if (K < 1 || K > kMaxK) return fail(HME_EINVAL, "K = %d out of range [1, %d]", K, kMaxK);
+  if (!hist_out || !offsets_out) return fail(HME_EINVAL, "hist_out / offsets_out is NULL");
+  if (N > 0 && (!labels || !perm_out)) return fail(HME_EINVAL, "labels / perm_out is NULL");
+  const int ntag = (tag_off != nullptr) + (tags != nullptr) + (tag_off_out != nullptr) + (tags_out != nullptr);
+  if (ntag != 0 && ntag != 4) return fail(HME_EINVAL, "tag arrays must be all NULL or all set");
+  const PartLayout pl = part_layout(sizeof(Header), N, K);
+  HME_TRY(check_ws(ws, ws_bytes, align_up(pl.end, 256)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  HME_CUDA(launch_partition(labels, N, K, pl, static_cast<char *>(ws), hist_out, offsets_out, perm_out,
+                            sorted_labels_out, at<Header>(ws, 0), s),
+           "partition");
+  if (ntag == 4) {
+    const int64_t nscratch = (int64_t)((pl.end - pl.misc) / sizeof(int64_t));
+    HME_CUDA(launch_tag_scatter(perm_out, N, offsets_out + K, tag_off, tags, tag_off_out, tags_out,
+                                at<int64_t>(ws, pl.misc), nscratch, s),
+             "partition: tag lists");
+  }
+  return HME_OK;
+}
+
+int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
+              int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws, size_t ws_bytes,
+              void *stream) {
+  HME_TRY(check_common(B, d, K, dtype));
+  HME_TRY(check_features(Q, B, d, ldq, dtype, true));
+  if (!C) return fail(HME_EINVAL, "C is NULL");
+  if (!offsets_out) return fail(HME_EINVAL, "offsets_out is NULL");
+  if (B > 0 && (!expert_out || !order_out)) return fail(HME_EINVAL, "expert_out / order_out is NULL");
+  const Layout L = feature_layout(B, d, K, dtype, 0);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  HME_TRY(do_prepare(Q, B, d, ldq, dtype, K, L, ws, s));
+  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, s));
+  HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
+                            offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
+           "route: partition");
+  return HME_OK;
+}
+
+int hme_debug_bounded_wait(uint64_t timeout_ns, void *ws, size_t ws_bytes, void *stream) {
+  if (timeout_ns < 1 || timeout_ns > 1000000000ull) return fail(HME_EINVAL, "timeout_ns out of range");
+  HME_TRY(check_ws(ws, ws_bytes, sizeof(Header)));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  HME_CUDA(launch_debug_wait(timeout_ns, at<Header>(ws, 0), s), "debug wait");
+  return HME_OK;
+}
+
+}  // extern "C"

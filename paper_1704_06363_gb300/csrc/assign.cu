@@ -1,0 +1,442 @@
+// assign.cu -- fused nearest-centre assignment (Eq. 2, Section 2) on the
+// sm_103a tensor cores.
+//
+// For a tile of 128 rows and a chunk of BN centres the kernel forms the dot
+// products x.c with tcgen05.mma (bf16 operands, fp32 accumulator in TMEM),
+// then four epilogue warps read the accumulator rows back with tcgen05.ld and
+// keep, per row, the smallest and second-smallest  ||c||^2 - 2 x.c  and the
+// index of the smallest (ties to the lower index because columns are scanned
+// in ascending order and the comparison is strict).  Nothing of size N x K is
+// ever written: per row the kernel emits a label, the distance to the chosen
+// centre and, for near ties, a re-score request.
+//
+// Operands: for bf16 features, A = X (bf16) and B = bf16(C); for fp32
+// features the split x = xh + xl, c = ch + cl (all bf16, 16 significant bits
+// together) gives x_eff.c_eff = xh.ch + xh.cl + xl.ch + xl.cl (four MMAs per
+// k-step).  With ||x_eff||^2 and ||c_eff||^2 from the same split values the
+// computed distance is ||x_eff - c_eff||^2 up to fp32 accumulation, whose
+// difference from ||x - c||^2 is O(2^-16 |x - c| (|x| + |c|)) per element.
+//
+// Warp roles (192 threads, one CTA per SM, persistent over row tiles):
+//   warp 0      TMA producer: A and B k-blocks into an S-stage ring,
+//   warp 1      TMEM allocator and single-thread MMA issuer,
+//   warps 2..5  epilogue; warp w reads TMEM lanes 32*(w%4) .. 32*(w%4)+31.
+// The accumulator is double-buffered in TMEM so the epilogue of one chunk
+// overlaps the MMAs of the next.  Every wait is bounded (see
+// mbar_wait_bounded); on expiry the kernel records HME_ETIMEOUT and ends.
+#include "hme_common.cuh"
+
+#include <cmath>
+#include <cstdio>
+#include <mutex>
+
+namespace hme {
+
+namespace {
+
+struct AssignParams {
+  int64_t N;
+  int num_kb;          // k-blocks of 64 elements along d
+  int BN, nchunks;
+  int num_tiles;
+  int stages;
+  uint32_t a_bytes;    // one A operand per stage (128 rows x 128 bytes)
+  uint32_t b_bytes;    // one B operand per stage (BN rows x 128 bytes)
+  uint32_t stage_bytes;
+  uint32_t tmem_cols;  // allocated TMEM columns
+  uint32_t acc_stride; // columns between the two accumulators
+  const float *xn;
+  const float *cn;     // Kp entries, +inf past K
+  int32_t *labels;
+  float *mind;
+  Header *hdr;
+  int32_t *flagged;
+  uint64_t limit_ns;
+  float margin;
+};
+
+constexpr int kThreads = 192;
+constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4;
+
+template <int NPROD>
+__global__ void __launch_bounds__(kThreads, 1)
+    assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
+                  const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
+                  const AssignParams p) {
+  constexpr int NOPS = (NPROD == 4) ? 2 : 1;  // operands per side (hi[, lo])
+  extern __shared__ uint8_t smem_raw[];
+  // 1024-byte alignment for the 128-byte swizzle atoms.
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  const uint32_t base = (raw_addr + 1023u) & ~1023u;
+  uint8_t *smem = smem_raw + (base - raw_addr);
+
+  const int S = p.stages;
+  uint8_t *ctrl = smem + (size_t)S * p.stage_bytes;
+  uint64_t *full = reinterpret_cast<uint64_t *>(ctrl);
+  uint64_t *empty = full + S;
+  uint64_t *tfull = empty + S;
+  uint64_t *tempty = tfull + 2;
+  uint64_t *drain = tempty + 2;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+  float *cnbuf = reinterpret_cast<float *>(ctrl + 512);  // one 256-float buffer per epilogue warp
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmA0);
+    prefetch_tensormap(&tmB0);
+    if (NPROD == 4) {
+      prefetch_tensormap(&tmA1);
+      prefetch_tensormap(&tmB1);
+    }
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      const uint64_t pol_a = l2_policy_evict_first();
+      const uint64_t pol_b = l2_policy_evict_last();
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        const int32_t row0 = tile * kBM;
+        for (int ch = 0; ch < p.nchunks && ok; ++ch) {
+          for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+            const int s = it % S;
+            const uint32_t ph = (it / S) & 1u;
+            if (!mbar_wait_bounded(smem_u32(&empty[s]), ph ^ 1u, p.limit_ns, p.hdr, kWhereProducer)) {
+              ok = false;
+              break;
+            }
+            const uint32_t fb = smem_u32(&full[s]);
+            mbar_arrive_expect_tx(fb, p.stage_bytes);
+            const uint32_t st = base + (uint32_t)s * p.stage_bytes;
+            const int32_t kx = kb * kBK;
+            tma_load_2d(st, &tmA0, fb, kx, row0, pol_a);
+            if (NPROD == 4) tma_load_2d(st + p.a_bytes, &tmA1, fb, kx, row0, pol_a);
+            const uint32_t sb = st + NOPS * p.a_bytes;
+            tma_load_2d(sb, &tmB0, fb, kx, ch * p.BN, pol_b);
+            if (NPROD == 4) tma_load_2d(sb + p.b_bytes, &tmB1, fb, kx, ch * p.BN, pol_b);
+          }
+        }
+      }
+      // Drain: every stage issued must land before the CTA may end.
+      if (!ok) {
+        const uint32_t issued = it;
+        for (uint32_t j = (issued > (uint32_t)S ? issued - S : 0); j < issued; ++j) {
+          mbar_wait_bounded(smem_u32(&full[j % S]), (j / S) & 1u, 200000000ull, p.hdr, kWhereProducer);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kBM, (uint32_t)p.BN);
+      uint32_t it = 0, acc_it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        for (int ch = 0; ch < p.nchunks && ok; ++ch, ++acc_it) {
+          const uint32_t a = acc_it & 1u;
+          const uint32_t aph = (acc_it >> 1) & 1u;
+          if (!mbar_wait_bounded(smem_u32(&tempty[a]), aph ^ 1u, p.limit_ns, p.hdr, kWhereMmaAcc)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dt = tmem_base + a * p.acc_stride;
+          for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
+            const int s = it % S;
+            const uint32_t ph = (it / S) & 1u;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), ph, p.limit_ns, p.hdr, kWhereMma)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = base + (uint32_t)s * p.stage_bytes;
+            const uint32_t sb = st + NOPS * p.a_bytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t ad0 = smem_desc_sw128(st + k * 32);
+              const uint64_t bd0 = smem_desc_sw128(sb + k * 32);
+              tc_mma_bf16(dt, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+              if (NPROD == 4) {
+                const uint64_t ad1 = smem_desc_sw128(st + p.a_bytes + k * 32);
+                const uint64_t bd1 = smem_desc_sw128(sb + p.b_bytes + k * 32);
+                tc_mma_bf16(dt, ad0, bd1, idesc, 1u);  // xh . cl
+                tc_mma_bf16(dt, ad1, bd0, idesc, 1u);  // xl . ch
+                tc_mma_bf16(dt, ad1, bd1, idesc, 1u);  // xl . cl
+              }
+            }
+            tc_commit(smem_u32(&empty[s]));  // frees the stage once these MMAs finish
+          }
+          if (ok) tc_commit(smem_u32(&tfull[a]));  // accumulator a is complete
+        }
+      }
+      if (!ok) {
+        // Let the MMAs already issued finish before TMEM is released.
+        tc_commit(smem_u32(drain));
+        mbar_wait_bounded(smem_u32(drain), 0, 200000000ull, p.hdr, kWhereMma);
+      }
+    }
+  } else {
+    // ---------------- epilogue: argmin over the accumulator rows ----------------
+    const int q = warp & 3;          // TMEM lane quarter this warp may access
+    float *cb = cnbuf + (warp - 2) * kMaxBN;  // this warp's copy of ||c||^2 for the chunk
+    const int row_in_tile = q * 32 + lane;
+    uint32_t acc_it = 0;
+    bool ok = true;
+    double obj = 0.0;
+    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+      float best1 = INFINITY, best2 = INFINITY;
+      int idx = 0;
+      for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
+        __syncwarp();
+        for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + ch * p.BN + t);
+        __syncwarp();
+        const uint32_t a = acc_it & 1u;
+        const uint32_t aph = (acc_it >> 1) & 1u;
+        if (!mbar_wait_bounded(smem_u32(&tfull[a]), aph, p.limit_ns, p.hdr, kWhereEpi)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
+        const int kbase = ch * p.BN;
+        for (int c = 0; c < p.BN; c += 16) {
+          uint32_t r[16];
+          tmem_ld16(taddr + (uint32_t)c, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float v = fmaf(-2.0f, __uint_as_float(r[j]), cb[c + j]);
+            if (v < best1) {
+              best2 = best1;
+              best1 = v;
+              idx = kbase + c + j;
+            } else if (v < best2) {
+              best2 = v;
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
+      }
+      if (!ok) break;
+      const int64_t row = (int64_t)tile * kBM + row_in_tile;
+      if (row < p.N) {
+        const float xr = __ldg(p.xn + row);
+        const float D1 = xr + best1;
+        const float D2 = xr + best2;
+        const float md = fmaxf(D1, 0.0f);
+        p.labels[row] = idx;
+        if (p.mind) p.mind[row] = md;
+        const bool near_tie = (best2 < INFINITY) && ((D2 - D1) <= p.margin * fmaxf(D2, xr));
+        if (near_tie) {
+          const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
+          p.flagged[slot] = (int32_t)row;
+        } else {
+          obj += (double)md;
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
+    if (lane == 0 && obj != 0.0) atomicAdd(&p.hdr->objective, obj);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+}
+
+// Exact re-score of near-tie rows: direct fp32 differences, squared and summed
+// per lane in fp32 (a sum of non-negative terms, relative error < 2^-17 for
+// d <= 16384 / 32 per lane), combined across the warp; ties to the lowest k.
+template <int DT>
+__global__ void __launch_bounds__(256) rescore_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                      const float *__restrict__ C, int K,
+                                                      const float *__restrict__ xn, int32_t *labels, float *mind,
+                                                      Header *hdr, const int32_t *__restrict__ flagged) {
+  const int lane = threadIdx.x & 31;
+  const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  const uint32_t count = *((volatile uint32_t *)&hdr->rescore_count);
+  double obj = 0.0;
+  for (uint32_t f = gw; f < count; f += nw) {
+    const int64_t row = flagged[f];
+    float best = INFINITY;
+    int arg = 0;
+    for (int k = 0; k < K; ++k) {
+      float s = 0.0f;
+      for (int j = lane; j < d; j += 32) {
+        float x, c;
+        if (DT == HME_BF16) {
+          x = __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(Xv)[row * ldx + j]);
+          c = __bfloat162float(__float2bfloat16_rn(C[(int64_t)k * d + j]));
+        } else {
+          x = reinterpret_cast<const float *>(Xv)[row * ldx + j];
+          c = C[(int64_t)k * d + j];
+        }
+        const float t = x - c;
+        s = fmaf(t, t, s);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      if (s < best) {
+        best = s;
+        arg = k;
+      }
+    }
+    if (lane == 0) {
+      labels[row] = arg;
+      if (mind) mind[row] = best;
+      obj += (double)best;
+    }
+  }
+  if (lane == 0 && obj != 0.0) atomicAdd(&hdr->objective, obj);
+  (void)xn;
+}
+
+// ---------------------------------------------------------------------------
+// host side: tensor maps and launch
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  return fn;
+}
+
+// bf16 matrix rows x cols (row stride ld elements), box = box_rows x 64 columns, 128-byte swizzle.
+int make_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return fail(HME_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(HME_ECUDA, "cuTensorMapEncodeTiled failed (%d) for %llu x %llu, ld %llu", (int)r,
+                (unsigned long long)rows, (unsigned long long)cols, (unsigned long long)ld);
+  return HME_OK;
+}
+
+}  // namespace
+
+int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
+                  const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
+                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, cudaStream_t s) {
+  if (N == 0) return HME_OK;
+  CUtensorMap mA0, mA1, mB0, mB1;
+  int rc;
+  if ((rc = make_map(&mA0, Xa, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
+  if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
+    return rc;
+  if (g.nprod == 4) {
+    if ((rc = make_map(&mA1, Xb, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
+    if ((rc = make_map(&mB1, clo, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
+      return rc;
+  } else {
+    mA1 = mA0;
+    mB1 = mB0;
+  }
+  AssignParams p;
+  p.N = N;
+  p.num_kb = (g.d + kBK - 1) / kBK;
+  p.BN = g.BN;
+  p.nchunks = g.nchunks;
+  p.num_tiles = (int)((N + kBM - 1) / kBM);
+  p.a_bytes = kBM * kBK * 2;
+  p.b_bytes = (uint32_t)g.BN * kBK * 2;
+  const int nops = g.nprod == 4 ? 2 : 1;
+  p.stage_bytes = nops * (p.a_bytes + p.b_bytes);
+  const size_t ctrl_bytes = 512 + 4 * kMaxBN * sizeof(float);
+  const size_t budget = 227 * 1024 - 1024 - ctrl_bytes;
+  int stages = (int)(budget / p.stage_bytes);
+  if (stages > 8) stages = 8;
+  if (stages < 2) return fail(HME_EINTERNAL, "assign: stage of %u bytes does not fit twice", p.stage_bytes);
+  p.stages = stages;
+  uint32_t stride = 32;
+  while (stride < (uint32_t)g.BN) stride <<= 1;
+  p.acc_stride = stride;
+  p.tmem_cols = 2 * stride;
+  p.xn = xn;
+  p.cn = cn;
+  p.labels = labels;
+  p.mind = mind;
+  p.hdr = hdr;
+  p.flagged = flagged;
+  p.limit_ns = wait_limit_ns();
+  p.margin = 2e-4f;
+  const size_t smem = (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
+  int grid = num_sms();
+  if (grid > p.num_tiles) grid = p.num_tiles;
+  cudaError_t e;
+  if (g.nprod == 4) {
+    e = cudaFuncSetAttribute(assign_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
+    assign_kernel<4><<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
+  } else {
+    e = cudaFuncSetAttribute(assign_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
+    assign_kernel<1><<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
+  }
+  count_launch();
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");
+  return HME_OK;
+}
+
+cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
+                           const float *xn, int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           cudaStream_t s) {
+  if (N == 0) return cudaSuccess;
+  const int grid = num_sms() * 4;
+  if (dtype == HME_BF16)
+    rescore_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, xn, labels, mind, hdr, flagged);
+  else
+    rescore_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, xn, labels, mind, hdr, flagged);
+  count_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace hme

@@ -1,0 +1,290 @@
+// hme_common.cuh -- internal declarations shared by the CUDA translation units
+// of libhme: workspace layout, status bits, launch bookkeeping and the inline
+// PTX wrappers (mbarrier, TMA, tcgen05) the sm_103a kernels use.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "../../include/hme.h"
+
+namespace hme {
+
+// ---------------------------------------------------------------------------
+// status word (first 256 bytes of every workspace)
+// ---------------------------------------------------------------------------
+enum : uint32_t {
+  kStatusBadLabel = 1u << 0,
+  kStatusTimeout = 1u << 1,
+};
+
+struct Header {          // lives at ws + 0, 256 bytes
+  uint32_t status;       // OR of kStatus* bits
+  uint32_t rescore_count;  // rows flagged by the assign margin test
+  uint32_t kpp_choice;   // k-means++: candidate picked in the current round
+  uint32_t pad0;
+  double objective;      // fp64 objective accumulator of hme_assign
+  uint32_t wait_where;   // which bounded wait expired (diagnostic)
+  uint32_t pad1[57];
+};
+static_assert(sizeof(Header) == 256, "header is 256 bytes");
+
+constexpr int kBM = 128;        // rows per assign tile (tcgen05 M)
+constexpr int kBK = 64;         // bf16 elements per stage k-block (one 128-byte swizzle row)
+constexpr int kMaxBN = 256;     // centres per tcgen05 N-chunk
+constexpr int kMaxK = 16384;
+constexpr int kMaxD = 16384;
+
+// ---------------------------------------------------------------------------
+// workspace layout
+// ---------------------------------------------------------------------------
+struct AssignGeom {
+  int d, K, dtype;
+  int ldp;        // row stride (elements) of the bf16 copies
+  int BN;         // centres per N-chunk (multiple of 16, <= 256)
+  int nchunks;    // ceil(K / BN)
+  int Kp;         // nchunks * BN
+  int nprod;      // 1 (bf16 features) or 4 (fp32 features, split products)
+};
+
+AssignGeom assign_geom(int d, int K, int dtype);
+
+struct PartLayout {
+  int64_t tile;     // items per partition tile (one warp each)
+  int64_t ntiles;
+  size_t tilecnt;   // int32[ntiles * K]
+  size_t hist;      // int64[K]
+  size_t offs;      // int64[K + 1]
+  size_t misc;      // int64 scratch for scans (block sums)
+  size_t end;
+};
+PartLayout part_layout(size_t base, int64_t N, int K);
+
+struct Layout {
+  size_t xn;        // f32[N]
+  size_t xhi, xlo;  // bf16[N * ldp] (fp32 features only)
+  size_t cb_hi, cb_lo;  // bf16[Kp * ldp]
+  size_t cn;        // f32[Kp]
+  size_t flagged;   // int32[N]: rows queued for the exact re-score
+  size_t perm, slab;  // int32[N] each: sorted order of the labels (update)
+  PartLayout part;  // partition scratch (update / route)
+  size_t sums;      // f64[K * d]
+  size_t kpp_rows;  // int32[m]
+  size_t kpp_d2;    // f64[m]
+  size_t kpp_part;  // f64[blocks]
+  size_t total;
+};
+Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m);
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---------------------------------------------------------------------------
+// host helpers (api.cu)
+// ---------------------------------------------------------------------------
+int fail(int code, const char *fmt, ...);
+int cuda_fail(cudaError_t e, const char *what);
+void count_launch(int n = 1);
+int num_sms();
+uint64_t wait_limit_ns();
+
+// ---------------------------------------------------------------------------
+// launchers (one per translation unit)
+// ---------------------------------------------------------------------------
+cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, int dtype, const AssignGeom &g,
+                                 float *xn, __nv_bfloat16 *xhi, __nv_bfloat16 *xlo, cudaStream_t s);
+cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
+                                float *cn, cudaStream_t s);
+int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
+                  const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
+                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, cudaStream_t s);
+cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
+                           const float *xn, int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           cudaStream_t s);
+cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
+                             int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,
+                             cudaStream_t s);
+// valid_total (device) = number of items with a label in [0, K) = offsets[K];
+// slots past it are never written by the partition and are not read.
+cudaError_t launch_tag_scatter(const int32_t *perm, int64_t N, const int64_t *valid_total, const int64_t *tag_off,
+                               const int32_t *tags, int64_t *tag_off_out, int32_t *tags_out, int64_t *scratch,
+                               int64_t nscratch, cudaStream_t s);
+cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *perm,
+                          const int32_t *sorted_labels, const int64_t *hist, const int64_t *valid_total,
+                          const float *mind, int K, double *sums, float *C, int64_t *counts_out, int32_t *n_reseeded,
+                          Header *hdr, cudaStream_t s);
+cudaError_t launch_kmeanspp(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, uint64_t seed,
+                            int64_t m, bool subsample, float *C_out, int32_t *rows, double *d2, double *part,
+                            Header *hdr, cudaStream_t s);
+cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
+int64_t kpp_candidates(int64_t N, int K, int method);
+int64_t kpp_blocks(int64_t m);
+
+// ---------------------------------------------------------------------------
+// device-side PTX wrappers
+// ---------------------------------------------------------------------------
+#ifdef __CUDACC__
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on an mbarrier phase.  Gives up after limit_ns of global time,
+// records kStatusTimeout (and where) in the header and returns false; the
+// caller then leaves its loop so that the kernel still ends.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns,
+                                                  Header *hdr, uint32_t where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  uint32_t spins = 0;
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((++spins & 63u) == 0 && global_timer_ns() - t0 > limit_ns) {
+      atomicOr(&hdr->status, (uint32_t)kStatusTimeout);
+      atomicExch(&hdr->wait_where, where);
+      return false;
+    }
+  }
+}
+
+// TMA: 2-D tiled bulk load global -> shared, completion counted on an mbarrier.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int32_t c0,
+                                            int32_t c1, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// ---- tcgen05 (5th-generation tensor cores, accumulators in TMEM) ----------
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem desc] x B[smem desc]^T, kind::f16 (bf16 in, fp32 accumulate).
+__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive (once) on an mbarrier when all previously issued tcgen05 ops of this thread complete.
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// 32 lanes x 32 bits, 16 consecutive columns: thread t of the warp gets lane
+// (quarter*32 + t), columns col .. col+15.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Shared-memory matrix descriptor for a K-major operand stored in the 128-byte
+// swizzled layout that TMA writes with CU_TENSOR_MAP_SWIZZLE_128B: rows of 128
+// bytes, 8-row groups 1024 bytes apart (stride byte offset), descriptor
+// version 1 (bit 46), layout type 2 = SWIZZLE_128B (bits 61-63).  The leading
+// byte offset is unused for this layout.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
+  uint64_t desc = 0;
+  desc |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  desc |= (uint64_t)(16u >> 4) << 16;
+  desc |= (uint64_t)(1024u >> 4) << 32;
+  desc |= (uint64_t)1 << 46;
+  desc |= (uint64_t)2 << 61;
+  return desc;
+}
+
+// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1),
+// B bf16 (bits 10-12 = 1), both K-major (bits 15, 16 = 0), N >> 3 at bits 17-22,
+// M >> 4 at bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+
+#endif  // __CUDACC__
+
+}  // namespace hme

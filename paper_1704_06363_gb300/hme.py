@@ -1,0 +1,185 @@
+"""ctypes binding of libhme (include/hme.h): argument marshalling only.
+
+Every function takes torch tensors that live on the current CUDA device,
+passes their data pointers and sizes to the C entry point of the same name,
+and raises ``HmeError`` on a non-zero status.  All arithmetic runs in the CUDA
+kernels of ``csrc/``; there is no CPU fallback: if ``lib/libhme.so`` has not
+been built (``paper_1704_06363_gb300._build.build()``), importing the library
+fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6)
+HME_F32, HME_BF16 = 0, 1
+HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE = range(4)
+HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
+HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED = 0, 1
+
+_NAMES = {0: "HME_OK", 1: "HME_EINVAL", 2: "HME_ENOMEM", 3: "HME_ECUDA", 4: "HME_ETIMEOUT", 5: "HME_EINTERNAL"}
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libhme.so")
+
+_lock = threading.Lock()
+_lib = None
+
+
+class HmeError(RuntimeError):
+    def __init__(self, code: int, fn: str, msg: str):
+        super().__init__(f"{fn}: {_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+def lib():
+    """The loaded libhme (built in-tree).  Raises if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libhme is not built ({LIB_PATH} missing): run paper_1704_06363_gb300._build.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        p, i64, i32, u64, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_uint64, ctypes.c_size_t
+        L.hme_workspace_bytes.restype = sz
+        L.hme_workspace_bytes.argtypes = [i32, i64, i32, i32, i32]
+        L.hme_last_error.restype = ctypes.c_char_p
+        L.hme_last_error.argtypes = []
+        L.hme_sync_status.restype = ctypes.c_int
+        L.hme_sync_status.argtypes = [p, p]
+        L.hme_kmeans_init.restype = ctypes.c_int
+        L.hme_kmeans_init.argtypes = [p, i64, i32, i64, i32, i32, u64, i32, p, p, sz, p]
+        L.hme_prepare_features.restype = ctypes.c_int
+        L.hme_prepare_features.argtypes = [p, i64, i32, i64, i32, i32, p, sz, p]
+        L.hme_assign.restype = ctypes.c_int
+        L.hme_assign.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
+        L.hme_update_centroids.restype = ctypes.c_int
+        L.hme_update_centroids.argtypes = [p, i64, i32, i64, i32, p, p, i32, p, p, p, p, p, sz, p]
+        L.hme_partition.restype = ctypes.c_int
+        L.hme_partition.argtypes = [p, i64, i32, p, p, p, p, p, p, p, p, p, sz, p]
+        L.hme_route.restype = ctypes.c_int
+        L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, p, p, p, p, sz, p]
+        L.hme_launch_count.restype = i64
+        L.hme_launch_count.argtypes = []
+        L.hme_debug_bounded_wait.restype = ctypes.c_int
+        L.hme_debug_bounded_wait.argtypes = [u64, p, sz, p]
+        _lib = L
+        return L
+
+
+def _check(rc: int, fn: str):
+    if rc != HME_OK:
+        raise HmeError(rc, fn, lib().hme_last_error().decode(errors="replace"))
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _features(X: torch.Tensor):
+    if X.dim() != 2 or X.stride(1) != 1:
+        raise ValueError("features must be a 2-D tensor with unit column stride")
+    if X.dtype == torch.float32:
+        dt = HME_F32
+    elif X.dtype == torch.bfloat16:
+        dt = HME_BF16
+    else:
+        raise TypeError(f"features must be float32 or bfloat16, got {X.dtype}")
+    return X.shape[0], X.shape[1], max(X.stride(0), X.shape[1]), dt
+
+
+def _ws(ws: torch.Tensor):
+    return ctypes.c_void_p(ws.data_ptr()), ws.numel() * ws.element_size()
+
+
+def hme_workspace_bytes(op: int, N: int, d: int, K: int, dtype: int) -> int:
+    return int(lib().hme_workspace_bytes(op, N, d, K, dtype))
+
+
+def workspace(op: int, N: int, d: int, K: int, dtype: int, device=None) -> torch.Tensor:
+    """A device byte tensor large enough for `op` (torch allocations are 512-byte aligned)."""
+    n = hme_workspace_bytes(op, N, d, K, dtype)
+    if n == 0:
+        raise HmeError(HME_EINVAL, "hme_workspace_bytes", lib().hme_last_error().decode(errors="replace"))
+    return torch.empty(n, dtype=torch.uint8, device=device if device is not None else "cuda")
+
+
+def hme_sync_status(ws: torch.Tensor, stream=None) -> int:
+    """Wait for the stream and return the device-side status of the last call on ws (no raise)."""
+    return int(lib().hme_sync_status(_ptr(ws), _stream(stream)))
+
+
+def hme_kmeans_init(X: torch.Tensor, K: int, seed: int, method: int, C_out: torch.Tensor, ws: torch.Tensor,
+                    stream=None):
+    N, d, ldx, dt = _features(X)
+    w, wb = _ws(ws)
+    _check(lib().hme_kmeans_init(_ptr(X), N, d, ldx, dt, K, seed & (2**64 - 1), method, _ptr(C_out), w, wb,
+                                 _stream(stream)), "hme_kmeans_init")
+
+
+def hme_prepare_features(X: torch.Tensor, K: int, ws: torch.Tensor, stream=None):
+    N, d, ldx, dt = _features(X)
+    w, wb = _ws(ws)
+    _check(lib().hme_prepare_features(_ptr(X), N, d, ldx, dt, K, w, wb, _stream(stream)), "hme_prepare_features")
+
+
+def hme_assign(X: torch.Tensor, C: torch.Tensor, labels_out: torch.Tensor, ws: torch.Tensor,
+               mind_out: Optional[torch.Tensor] = None, objective_out: Optional[torch.Tensor] = None,
+               flags: int = HME_ASSIGN_DEFAULT, stream=None):
+    N, d, ldx, dt = _features(X)
+    K = C.shape[0]
+    w, wb = _ws(ws)
+    _check(lib().hme_assign(_ptr(X), N, d, ldx, dt, _ptr(C), K, flags, _ptr(labels_out), _ptr(mind_out),
+                            _ptr(objective_out), w, wb, _stream(stream)), "hme_assign")
+
+
+def hme_update_centroids(X: torch.Tensor, labels: torch.Tensor, mind: Optional[torch.Tensor], C_inout: torch.Tensor,
+                         ws: torch.Tensor, counts_out: Optional[torch.Tensor] = None,
+                         n_reseeded_out: Optional[torch.Tensor] = None, objective_out: Optional[torch.Tensor] = None,
+                         stream=None):
+    N, d, ldx, dt = _features(X)
+    K = C_inout.shape[0]
+    w, wb = _ws(ws)
+    _check(lib().hme_update_centroids(_ptr(X), N, d, ldx, dt, _ptr(labels), _ptr(mind), K, _ptr(C_inout),
+                                      _ptr(counts_out), _ptr(n_reseeded_out), _ptr(objective_out), w, wb,
+                                      _stream(stream)),
+           "hme_update_centroids")
+
+
+def hme_partition(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_out: torch.Tensor,
+                  perm_out: torch.Tensor, ws: torch.Tensor, sorted_labels_out: Optional[torch.Tensor] = None,
+                  tag_off: Optional[torch.Tensor] = None, tags: Optional[torch.Tensor] = None,
+                  tag_off_out: Optional[torch.Tensor] = None, tags_out: Optional[torch.Tensor] = None, stream=None):
+    N = labels.shape[0]
+    w, wb = _ws(ws)
+    _check(lib().hme_partition(_ptr(labels), N, K, _ptr(hist_out), _ptr(offsets_out), _ptr(perm_out),
+                               _ptr(sorted_labels_out), _ptr(tag_off), _ptr(tags), _ptr(tag_off_out), _ptr(tags_out),
+                               w, wb, _stream(stream)), "hme_partition")
+
+
+def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offsets_out: torch.Tensor,
+              order_out: torch.Tensor, ws: torch.Tensor, stream=None):
+    B, d, ldq, dt = _features(Q)
+    K = C.shape[0]
+    w, wb = _ws(ws)
+    _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, _ptr(expert_out), _ptr(offsets_out), _ptr(order_out),
+                           w, wb, _stream(stream)), "hme_route")
+
+
+def hme_launch_count() -> int:
+    return int(lib().hme_launch_count())
+
+
+def hme_debug_bounded_wait(timeout_ns: int, ws: torch.Tensor, stream=None):
+    w, wb = _ws(ws)
+    _check(lib().hme_debug_bounded_wait(timeout_ns, w, wb, _stream(stream)), "hme_debug_bounded_wait")

@@ -1,0 +1,89 @@
+"""CPU-side checks of the C ABI: the library builds, loads without a GPU, exports
+every entry point that include/hme.h declares, and rejects bad arguments on the
+host before any CUDA call is made."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "hme.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_1704_06363_gb300 import _build
+    path = _build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_entry_points():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"HME_API\s+[\w\s\*]+?\b(hme_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_entry_points()
+    for required in ["hme_kmeans_init", "hme_assign", "hme_update_centroids", "hme_partition", "hme_route",
+                     "hme_workspace_bytes", "hme_last_error", "hme_sync_status", "hme_prepare_features"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_entry_points():
+        assert hasattr(lib, name), f"{name} declared in hme.h but not exported"
+
+
+def test_workspace_sizes(lib):
+    f = lib.hme_workspace_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    # fp32 features carry their bf16 split (4 bytes per element) in the workspace
+    assert f(1, 1_000_000, 2048, 64, 0) >= 1_000_000 * 2048 * 4
+    assert f(1, 1_000_000, 2048, 64, 1) < 1_000_000 * 2048  # bf16: no copy of X
+    assert f(2, 50_000_000, 256, 4096, 1) > 0
+    assert f(2, 0, 1, 1, 0) > 0
+    assert f(1, 10, 0, 4, 0) == 0  # d = 0 rejected
+    assert f(1, 10, 4, 0, 0) == 0  # K = 0 rejected
+    assert f(1, 10, 4, 4, 7) == 0  # unknown dtype
+    assert f(1, 2**31, 4, 4, 0) == 0
+
+
+def test_host_validation_rejects_before_launch(lib):
+    lib.hme_assign.restype = ctypes.c_int
+    lib.hme_last_error.restype = ctypes.c_char_p
+    p = ctypes.c_void_p
+    args = [p(16), ctypes.c_int64(10), ctypes.c_int32(8), ctypes.c_int64(8), ctypes.c_int32(0), p(16),
+            ctypes.c_int32(4), ctypes.c_int32(0), p(16), None, None, p(256), ctypes.c_size_t(1 << 30), None]
+    bad_k = list(args)
+    bad_k[6] = ctypes.c_int32(0)
+    assert lib.hme_assign(*bad_k) == 1 and b"K" in lib.hme_last_error()
+    bad_ld = list(args)
+    bad_ld[3] = ctypes.c_int64(4)
+    assert lib.hme_assign(*bad_ld) == 1
+    bad_ws = list(args)
+    bad_ws[11] = p(257)
+    assert lib.hme_assign(*bad_ws) == 1 and b"aligned" in lib.hme_last_error()
+    small_ws = list(args)
+    small_ws[12] = ctypes.c_size_t(16)
+    assert lib.hme_assign(*small_ws) == 2  # HME_ENOMEM
+    bf16_misaligned = list(args)
+    bf16_misaligned[4] = ctypes.c_int32(1)
+    bf16_misaligned[3] = ctypes.c_int64(12)
+    bf16_misaligned[2] = ctypes.c_int32(12)
+    assert lib.hme_assign(*bf16_misaligned) == 1 and b"TMA" in lib.hme_last_error()
+    lib.hme_partition.restype = ctypes.c_int
+    # tag arrays must be all or none
+    assert lib.hme_partition(p(16), ctypes.c_int64(4), ctypes.c_int32(2), p(16), p(16), p(16), None, p(16), None,
+                             None, None, p(256), ctypes.c_size_t(1 << 20), None) == 1
+
+
+def test_product_path_has_no_oracle_import():
+    """The product package never imports, links or runs the oracle."""
+    pkg = os.path.join(ROOT, "paper_1704_06363_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for fn in files:
+            if fn.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, fn)).read()
+                assert "import oracle" not in text and "from oracle" not in text and "liboracle" not in text, fn

@@ -1,0 +1,269 @@
+"""GPU parity of each C-ABI entry point against the fp64 oracle (small and ragged shapes)."""
+import numpy as np
+import pytest
+import torch
+
+import hme_synth
+import oracle
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+hme = pytest.importorskip("paper_1704_06363_gb300.hme")
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    d = torch.device("cuda:0")
+    torch.cuda.set_device(d)
+    return d
+
+
+def _mixture(N, d, K, dtype, seed, scale=3.0, relu=False, ld=None):
+    g = torch.Generator().manual_seed(seed)
+    centres = torch.randn(K, d, generator=g) * scale
+    comp = torch.randint(0, K, (N,), generator=g)
+    X = centres[comp] + torch.randn(N, d, generator=g)
+    if relu:
+        X.clamp_(min=0)
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    if ld is not None and ld != d:
+        buf = torch.zeros(N, ld, dtype=tdt)
+        buf[:, :d] = X.to(tdt)
+        X = buf[:, :d]
+    else:
+        X = X.to(tdt)
+    return X
+
+
+def _host(X, dtype):
+    return hme_synth.host_array(X.contiguous(), dtype)
+
+
+def _assign(X, C, dev, mind=True, prepared=False):
+    N, d = X.shape
+    K = C.shape[0]
+    Xg = X.to(dev) if X.is_contiguous() else _to_dev_strided(X, dev)
+    dt = hme.HME_F32 if X.dtype == torch.float32 else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+    lab = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    md = torch.empty(N, dtype=torch.float32, device=dev) if mind else None
+    obj = torch.zeros(1, dtype=torch.float64, device=dev)
+    Cg = C.to(dev)
+    if prepared:
+        hme.hme_prepare_features(Xg, K, ws)
+        hme.hme_assign(Xg, Cg, lab, ws, md, obj, flags=hme.HME_ASSIGN_PREPARED)
+    else:
+        hme.hme_assign(Xg, Cg, lab, ws, md, obj)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    return lab.cpu().numpy(), (md.cpu().numpy() if mind else None), obj.item()
+
+
+def _to_dev_strided(X, dev):
+    base = X.as_strided((X.shape[0], X.stride(0)), (X.stride(0), 1))
+    return base.to(dev)[:, : X.shape[1]]
+
+
+ASSIGN_CASES = [
+    # N, d, K, dtype, ld
+    (1000, 128, 16, "f32", None),
+    (1000, 128, 16, "bf16", None),
+    (777, 33, 5, "f32", None),
+    (777, 40, 5, "bf16", None),
+    (3000, 130, 300, "f32", None),
+    (3000, 130, 300, "bf16", 136),
+    (257, 1, 3, "f32", None),
+    (129, 64, 1, "f32", None),
+    (129, 64, 1, "bf16", None),
+    (2000, 512, 1024, "f32", None),
+    (2000, 256, 4096, "bf16", None),
+    (4100, 2048, 64, "f32", None),
+    (4100, 2048, 256, "bf16", None),
+    (50, 96, 200, "f32", None),
+]
+
+
+@pytest.mark.parametrize("N,d,K,dtype,ld", ASSIGN_CASES, ids=lambda v: str(v))
+def test_assign_parity(dev, N, d, K, dtype, ld):
+    X = _mixture(N, d, min(K, 64), dtype, seed=N + d + K, ld=ld)
+    C = hme_synth.random_centroids(K, d, seed=K + d, scale=3.0)
+    # half of the centres sit on data points so that the nearest one is meaningful
+    C[: K // 2] = X[: K // 2].float() if N >= K // 2 else C[: K // 2]
+    lab, md, obj = _assign(X, C, dev)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+
+
+def test_assign_prepared_equals_unprepared(dev):
+    X = _mixture(2000, 256, 32, "f32", seed=5)
+    C = hme_synth.random_centroids(32, 256, seed=9, scale=3.0)
+    a = _assign(X, C, dev, prepared=False)
+    b = _assign(X, C, dev, prepared=True)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1]) and a[2] == b[2]
+
+
+def test_assign_duplicate_centres_and_zero_rows(dev):
+    N, d, K = 600, 64, 8
+    X = _mixture(N, d, 4, "f32", seed=3, relu=True)
+    X[:50] = 0.0  # all-zero post-ReLU rows
+    C = hme_synth.random_centroids(K, d, seed=2)
+    C[3] = C[1]  # exact duplicates: ties go to the lower index
+    C[5] = C[1]
+    lab, md, obj = _assign(X, C, dev)
+    assert not np.any((lab == 3) | (lab == 5))
+    parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj)
+
+
+def test_assign_empty_input(dev):
+    X = torch.empty(0, 64, dtype=torch.float32)
+    C = hme_synth.random_centroids(4, 64, seed=1)
+    ws = hme.workspace(hme.HME_OP_ASSIGN, 0, 64, 4, hme.HME_F32, device=dev)
+    lab = torch.empty(0, dtype=torch.int32, device=dev)
+    obj = torch.full((1,), 7.0, dtype=torch.float64, device=dev)
+    hme.hme_assign(X.to(dev), C.to(dev), lab, ws, None, obj)
+    assert hme.hme_sync_status(ws) == hme.HME_OK and obj.item() == 0.0
+
+
+UPDATE_CASES = [
+    (1000, 128, 16, "f32", False),
+    (1000, 128, 16, "bf16", False),
+    (3001, 130, 37, "f32", True),
+    (3001, 136, 37, "bf16", True),
+    (5000, 2048, 64, "f32", False),
+    (5000, 256, 700, "bf16", True),
+    (300, 20, 500, "f32", True),  # more clusters than points: reseeds run out of rows
+]
+
+
+@pytest.mark.parametrize("N,d,K,dtype,holes", UPDATE_CASES, ids=lambda v: str(v))
+def test_update_parity(dev, N, d, K, dtype, holes):
+    X = _mixture(N, d, min(K, 50), dtype, seed=N * 7 + K)
+    g = torch.Generator().manual_seed(K)
+    w = torch.arange(1, K + 1, dtype=torch.float64) ** -1.1
+    labels = torch.multinomial(w, N, replacement=True, generator=g).to(torch.int32)
+    if holes:  # force empty clusters
+        labels[(labels % 5) == 2] = 0
+    mind = (torch.rand(N, generator=g) * 10).float()
+    mind[:7] = 5.0  # ties in the farthest-point order
+    C0 = hme_synth.random_centroids(K, d, seed=3)
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+    Cg = C0.to(dev)
+    counts = torch.empty(K, dtype=torch.int64, device=dev)
+    nres = torch.full((1,), -1, dtype=torch.int32, device=dev)
+    J = torch.zeros(1, dtype=torch.float64, device=dev)
+    hme.hme_update_centroids(X.to(dev), labels.to(dev), mind.to(dev), Cg, ws, counts, nres, J)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    parity.check_objective(J.item(), _host(X, dtype), dtype, C0.numpy(), labels.numpy())
+    Cref, cref, nref = oracle.update(_host(X, dtype), labels.numpy(), mind.double().numpy(), C0.numpy(), dtype)
+    assert np.array_equal(counts.cpu().numpy(), cref)
+    assert nres.item() == nref
+    parity.check_centres(Cg.cpu().numpy(), Cref)
+    # re-seeded centres are exact copies of rows
+    empty = np.nonzero(cref == 0)[0]
+    assert np.array_equal(Cg.cpu().numpy()[empty], Cref[empty])
+
+
+PART_CASES = [(0, 4), (1, 1), (31, 7), (1000, 64), (100003, 1000), (70000, 4096), (50000, 1), (12345, 16384)]
+
+
+@pytest.mark.parametrize("N,K", PART_CASES, ids=lambda v: str(v))
+def test_partition_bit_exact(dev, N, K):
+    g = torch.Generator().manual_seed(N + K)
+    w = torch.arange(1, K + 1, dtype=torch.float64) ** -1.0
+    labels = torch.multinomial(w, max(N, 1), replacement=True, generator=g).to(torch.int32)[:N]
+    ws = hme.workspace(hme.HME_OP_PARTITION, N, 1, K, hme.HME_F32, device=dev)
+    hist = torch.empty(K, dtype=torch.int64, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    perm = torch.empty(N, dtype=torch.int32, device=dev)
+    sl = torch.empty(N, dtype=torch.int32, device=dev)
+    hme.hme_partition(labels.to(dev), K, hist, offs, perm, ws, sl)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    parity.check_partition(dict(hist=hist.cpu().numpy(), offsets=offs.cpu().numpy(), perm=perm.cpu().numpy(),
+                                sorted_labels=sl.cpu().numpy()), labels.numpy(), K)
+
+
+def test_partition_tags_and_misaligned_labels(dev):
+    N, K = 20001, 33
+    w = hme_synth.WORKLOADS[4].with_rows(N)
+    tag_off, tags = hme_synth.make_tags(w)
+    g = torch.Generator().manual_seed(1)
+    full = torch.randint(0, K, (N + 1,), generator=g, dtype=torch.int32)
+    labels_d = full.to(dev)[1:]  # 4-byte offset: exercises the unaligned staging path
+    ws = hme.workspace(hme.HME_OP_PARTITION, N, 1, K, hme.HME_F32, device=dev)
+    hist = torch.empty(K, dtype=torch.int64, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    perm = torch.empty(N, dtype=torch.int32, device=dev)
+    too = torch.empty(N + 1, dtype=torch.int64, device=dev)
+    tgo = torch.empty(tags.numel(), dtype=torch.int32, device=dev)
+    hme.hme_partition(labels_d, K, hist, offs, perm, ws, None, tag_off.to(dev), tags.to(dev), too, tgo)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    parity.check_partition(dict(hist=hist.cpu().numpy(), offsets=offs.cpu().numpy(), perm=perm.cpu().numpy(),
+                                tag_off=too.cpu().numpy(), tags=tgo.cpu().numpy()),
+                           full[1:].numpy(), K, tag_off.numpy(), tags.numpy())
+
+
+def test_partition_bad_label_reports_einval(dev):
+    labels = torch.tensor([0, 1, 9, 2, -3, 1], dtype=torch.int32, device=dev)
+    K = 3
+    ws = hme.workspace(hme.HME_OP_PARTITION, 6, 1, K, hme.HME_F32, device=dev)
+    hist = torch.empty(K, dtype=torch.int64, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    perm = torch.full((6,), -1, dtype=torch.int32, device=dev)
+    hme.hme_partition(labels, K, hist, offs, perm, ws)
+    assert hme.hme_sync_status(ws) == hme.HME_EINVAL
+    assert hist.cpu().tolist() == [1, 2, 1]  # the valid labels are still counted
+    assert perm.cpu().tolist()[:4] == [0, 1, 5, 3]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_route_parity(dev, dtype):
+    B, d, K = 5000, 192, 40
+    Q = _mixture(B, d, K, dtype, seed=11)
+    C = hme_synth.random_centroids(K, d, seed=12, scale=3.0)
+    C[:20] = Q[:20].float()
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ROUTE, B, d, K, dt, device=dev)
+    expert = torch.empty(B, dtype=torch.int32, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    order = torch.empty(B, dtype=torch.int32, device=dev)
+    hme.hme_route(Q.to(dev), C.to(dev), expert, offs, order, ws)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    e = expert.cpu().numpy()
+    parity.check_assign(_host(Q, dtype), dtype, C.numpy(), e)
+    parity.check_partition(dict(offsets=offs.cpu().numpy(), perm=order.cpu().numpy()), e, K)
+
+
+@pytest.mark.parametrize("N,d,K,dtype,method", [
+    (10000, 128, 16, "f32", hme.HME_INIT_KMEANSPP),
+    (3000, 64, 9, "bf16", hme.HME_INIT_KMEANSPP),
+    (20000, 96, 8, "f32", hme.HME_INIT_KMEANSPP_SUBSAMPLE),
+    (7, 5, 7, "f32", hme.HME_INIT_KMEANSPP),
+])
+def test_kmeanspp_matches_oracle(dev, N, d, K, dtype, method):
+    X = _mixture(N, d, K, dtype, seed=N + K)
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_INIT, N, d, K, dt, device=dev)
+    C = torch.empty(K, d, dtype=torch.float32, device=dev)
+    for seed in (0, 1, 2**63 + 5):
+        hme.hme_kmeans_init(X.to(dev), K, seed, method, C, ws)
+        assert hme.hme_sync_status(ws) == hme.HME_OK
+        Cref, _ = oracle.kmeanspp(_host(X, dtype), K, seed, method == hme.HME_INIT_KMEANSPP_SUBSAMPLE, dtype)
+        assert np.array_equal(C.cpu().numpy(), Cref)
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(dev):
+    ws = torch.empty(256, dtype=torch.uint8, device=dev)
+    hme.hme_debug_bounded_wait(2_000_000, ws)  # 2 ms on a barrier nothing completes
+    assert hme.hme_sync_status(ws) == hme.HME_ETIMEOUT
+    x = torch.arange(10, device=dev).sum().item()  # the context is still usable
+    assert x == 45
+
+
+def test_launch_counter_moves(dev):
+    before = hme.hme_launch_count()
+    X = _mixture(300, 32, 4, "f32", seed=1)
+    _assign(X, hme_synth.random_centroids(4, 32, seed=1), dev)
+    assert hme.hme_launch_count() - before >= 3

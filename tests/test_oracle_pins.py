@@ -75,6 +75,7 @@ def test_hand_examples(case):
     assert labels.tolist() == case["labels"]
     assert d1.tolist() == case["d1"]
     assert J == case["objective"]
+    assert oracle.objective(X, C0, labels) == case["objective"]
     C1, counts, nr = oracle.update(X, labels, d1, C0)
     assert C1.tolist() == case["C1"]
     assert counts.tolist() == case["counts"]
@@ -266,6 +267,9 @@ def test_lloyd_invariants_random_data():
         # lowest index among exact minima
         for i in np.where(np.abs(Ds[:, 1] - Ds[:, 0]) <= scale)[0]:
             assert labels[i] == np.where(np.abs(D[i] - Ds[i, 0]) <= scale)[0].min()
+        # the objective of the assign's own labels is the assign's objective; any other labelling is not lower
+        assert oracle.objective(X, C, labels) == J
+        assert oracle.objective(X, C, (labels + 1) % K) >= J
         C_new, counts, nr = oracle.update(X, labels, d1, C)
         assert counts.sum() == 800
         assert counts.tolist() == np.bincount(labels, minlength=K).tolist()
