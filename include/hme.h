@@ -199,10 +199,13 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
  * receives a contiguous run of rows:
  *   expert_out[b] = label of Q row b (int32[B]), offsets_out (int64[K+1]),
  *   order_out (int32[B]) = rows of Q grouped by expert, ascending within one.
+ * flags: HME_ASSIGN_DEFAULT, or HME_ASSIGN_PREPARED when ws already holds Q
+ * prepared by hme_prepare_features (e.g. routing the training set with the
+ * workspace of the Lloyd loop: HME_OP_ROUTE and HME_OP_ASSIGN sizes agree).
  */
 HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
-              int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws, size_t ws_bytes,
-              void *stream);
+                      int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,
+                      size_t ws_bytes, void *stream);
 
 /* Number of kernels this library has launched in this process (diagnostic). */
 HME_API int64_t hme_launch_count(void);

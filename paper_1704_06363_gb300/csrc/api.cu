@@ -90,7 +90,7 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   L.cb_hi = take((size_t)g.Kp * g.ldp * 2);
   L.cb_lo = dtype == HME_F32 ? take((size_t)g.Kp * g.ldp * 2) : 0;
   L.cn = take((size_t)g.Kp * 4);
-  L.flagged = take((size_t)(N > 0 ? N : 1) * 4);
+  L.flagged = take((size_t)(N > 0 ? N : 1) * 12);  // (row, best, runner-up) per queued row
   L.perm = take((size_t)(N > 0 ? N : 1) * 4);
   L.slab = take((size_t)(N > 0 ? N : 1) * 4);
   L.part = part_layout(align_up(off, 256), N, K);
@@ -346,18 +346,19 @@ int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out
 }
 
 int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
-              int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws, size_t ws_bytes,
+              int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws, size_t ws_bytes,
               void *stream) {
   HME_TRY(check_common(B, d, K, dtype));
   HME_TRY(check_features(Q, B, d, ldq, dtype, true));
   if (!C) return fail(HME_EINVAL, "C is NULL");
   if (!offsets_out) return fail(HME_EINVAL, "offsets_out is NULL");
   if (B > 0 && (!expert_out || !order_out)) return fail(HME_EINVAL, "expert_out / order_out is NULL");
+  if (flags & ~HME_ASSIGN_PREPARED) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
   const Layout L = feature_layout(B, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_TRY(do_prepare(Q, B, d, ldq, dtype, K, L, ws, s));
+  if (!(flags & HME_ASSIGN_PREPARED)) HME_TRY(do_prepare(Q, B, d, ldq, dtype, K, L, ws, s));
   HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, s));
   HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
                             offsets_out, order_out, nullptr, at<Header>(ws, 0), s),

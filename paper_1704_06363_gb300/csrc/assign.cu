@@ -208,8 +208,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     double obj = 0.0;
     for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
-      float best1 = INFINITY, best2 = INFINITY;
-      int idx = 0;
+      float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
+      int idx1 = 0, idx2 = 0;
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
         __syncwarp();
         for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + ch * p.BN + t);
@@ -231,11 +231,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int j = 0; j < 16; ++j) {
             const float v = fmaf(-2.0f, __uint_as_float(r[j]), cb[c + j]);
             if (v < best1) {
+              best3 = best2;
               best2 = best1;
+              idx2 = idx1;
               best1 = v;
-              idx = kbase + c + j;
+              idx1 = kbase + c + j;
             } else if (v < best2) {
+              best3 = best2;
               best2 = v;
+              idx2 = kbase + c + j;
+            } else if (v < best3) {
+              best3 = v;
             }
           }
         }
@@ -249,13 +255,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float xr = __ldg(p.xn + row);
         const float D1 = xr + best1;
         const float D2 = xr + best2;
+        const float D3 = xr + best3;
         const float md = fmaxf(D1, 0.0f);
-        p.labels[row] = idx;
+        p.labels[row] = idx1;
         if (p.mind) p.mind[row] = md;
-        const bool near_tie = (best2 < INFINITY) && ((D2 - D1) <= p.margin * fmaxf(D2, xr));
-        if (near_tie) {
+        // Near tie: the runner-up (and maybe the third) could be the true nearest
+        // centre within the error of the tensor-core distances; queue the row for
+        // an exact comparison of the candidates (all K if a third one is close).
+        const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= p.margin * fmaxf(D2, xr));
+        if (near2) {
+          const bool near3 = (best3 < INFINITY) && ((D3 - D1) <= p.margin * fmaxf(D3, xr));
           const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
-          p.flagged[slot] = (int32_t)row;
+          p.flagged[3 * slot + 0] = (int32_t)row;
+          p.flagged[3 * slot + 1] = idx1;
+          p.flagged[3 * slot + 2] = near3 ? -1 : idx2;
         } else {
           obj += (double)md;
         }
@@ -275,41 +288,119 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Exact re-score of near-tie rows: direct fp32 differences, squared and summed
-// per lane in fp32 (a sum of non-negative terms, relative error < 2^-17 for
-// d <= 16384 / 32 per lane), combined across the warp; ties to the lowest k.
-template <int DT>
+// per lane in fp32 (a sum of non-negative terms), combined across the warp;
+// ties to the lowest k.  A queued row names its two candidates (best and
+// runner-up of the tensor-core pass), or -1 for "compare all K" when a third
+// centre was also within the margin.
+// Row segment loads: VW consecutive elements (16 bytes when vectorised).
+template <int DT, int VW>
+__device__ __forceinline__ void load_x(const void *Xv, int64_t off, float (&v)[VW]) {
+  if constexpr (DT == HME_F32) {
+    const float *p = reinterpret_cast<const float *>(Xv) + off;
+    if constexpr (VW == 4) {
+      const float4 f = __ldg(reinterpret_cast<const float4 *>(p));
+      v[0] = f.x, v[1] = f.y, v[2] = f.z, v[3] = f.w;
+    } else {
+#pragma unroll
+      for (int e = 0; e < VW; ++e) v[e] = __ldg(p + e);
+    }
+  } else {
+    const __nv_bfloat16 *p = reinterpret_cast<const __nv_bfloat16 *>(Xv) + off;
+    if constexpr (VW == 8) {
+      const uint4 u = __ldg(reinterpret_cast<const uint4 *>(p));
+      const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+      for (int t = 0; t < VW / 2; ++t) {
+        const float2 f = __bfloat1622float2(h[t]);
+        v[2 * t] = f.x, v[2 * t + 1] = f.y;
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < VW; ++e) v[e] = __bfloat162float(p[e]);
+    }
+  }
+}
+
+// Centre values the assign step compares against (bf16-rounded for bf16 features).
+template <int DT, int VW>
+__device__ __forceinline__ void load_c(const float *C, int64_t off, float (&v)[VW]) {
+  if constexpr (VW % 4 == 0) {
+#pragma unroll
+    for (int q = 0; q < VW / 4; ++q) {
+      const float4 f = __ldg(reinterpret_cast<const float4 *>(C + off) + q);
+      v[4 * q] = f.x, v[4 * q + 1] = f.y, v[4 * q + 2] = f.z, v[4 * q + 3] = f.w;
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < VW; ++e) v[e] = __ldg(C + off + e);
+  }
+  if constexpr (DT == HME_BF16) {
+#pragma unroll
+    for (int e = 0; e < VW; ++e) v[e] = __bfloat162float(__float2bfloat16_rn(v[e]));
+  }
+}
+
+__device__ __forceinline__ float warp_sum_f(float s) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  return s;
+}
+
+// sum_j (x_j - c_j)^2 over one row, lanes striding by 32 * VW elements (d % VW == 0).
+template <int DT, int VW>
+__device__ __forceinline__ float row_dist2(const void *Xv, int64_t xoff, const float *C, int64_t coff, int d,
+                                           int lane) {
+  float s = 0.0f;
+#pragma unroll 4
+  for (int j = lane * VW; j < d; j += 32 * VW) {
+    float x[VW], c[VW];
+    load_x<DT, VW>(Xv, xoff + j, x);
+    load_c<DT, VW>(C, coff + j, c);
+#pragma unroll
+    for (int e = 0; e < VW; ++e) {
+      const float t = x[e] - c[e];
+      s = fmaf(t, t, s);
+    }
+  }
+  return warp_sum_f(s);
+}
+
+// Exact re-score of near-tie rows: direct differences, squared and summed per
+// lane in fp32 (a sum of non-negative terms), combined across the warp; ties to
+// the lowest k.  A queued row names its two candidates (best and runner-up of
+// the tensor-core pass), or -1 for "compare all K" when a third centre was also
+// within the margin.  One warp per queued row, 16-byte loads when the layout
+// allows.
+template <int DT, int VW>
 __global__ void __launch_bounds__(256) rescore_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
-                                                      const float *__restrict__ C, int K,
-                                                      const float *__restrict__ xn, int32_t *labels, float *mind,
-                                                      Header *hdr, const int32_t *__restrict__ flagged) {
+                                                      const float *__restrict__ C, int K, int32_t *labels,
+                                                      float *mind, Header *hdr, const int32_t *__restrict__ flagged) {
   const int lane = threadIdx.x & 31;
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int nw = (gridDim.x * blockDim.x) >> 5;
   const uint32_t count = *((volatile uint32_t *)&hdr->rescore_count);
   double obj = 0.0;
   for (uint32_t f = gw; f < count; f += nw) {
-    const int64_t row = flagged[f];
-    float best = INFINITY;
-    int arg = 0;
-    for (int k = 0; k < K; ++k) {
-      float s = 0.0f;
-      for (int j = lane; j < d; j += 32) {
-        float x, c;
-        if (DT == HME_BF16) {
-          x = __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(Xv)[row * ldx + j]);
-          c = __bfloat162float(__float2bfloat16_rn(C[(int64_t)k * d + j]));
-        } else {
-          x = reinterpret_cast<const float *>(Xv)[row * ldx + j];
-          c = C[(int64_t)k * d + j];
+    const int64_t row = flagged[3 * f + 0];
+    const int i1 = flagged[3 * f + 1];
+    const int i2 = flagged[3 * f + 2];
+    float best;
+    int arg;
+    if (i2 >= 0) {
+      const float s1 = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)i1 * d, d, lane);
+      const float s2 = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)i2 * d, d, lane);
+      const bool first = s1 < s2 || (s1 == s2 && i1 < i2);
+      best = first ? s1 : s2;
+      arg = first ? i1 : i2;
+    } else {
+      best = INFINITY;
+      arg = 0;
+      for (int k = 0; k < K; ++k) {
+        const float s = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)k * d, d, lane);
+        if (s < best) {
+          best = s;
+          arg = k;
         }
-        const float t = x - c;
-        s = fmaf(t, t, s);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-      if (s < best) {
-        best = s;
-        arg = k;
       }
     }
     if (lane == 0) {
@@ -319,7 +410,6 @@ __global__ void __launch_bounds__(256) rescore_kernel(const void *__restrict__ X
     }
   }
   if (lane == 0 && obj != 0.0) atomicAdd(&hdr->objective, obj);
-  (void)xn;
 }
 
 // ---------------------------------------------------------------------------
@@ -429,12 +519,21 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            const float *xn, int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
                            cudaStream_t s) {
+  (void)xn;
   if (N == 0) return cudaSuccess;
   const int grid = num_sms() * 4;
-  if (dtype == HME_BF16)
-    rescore_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, xn, labels, mind, hdr, flagged);
-  else
-    rescore_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, xn, labels, mind, hdr, flagged);
+  const bool al = ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(C)) & 15u) == 0;
+  if (dtype == HME_BF16) {
+    if (al && d % 8 == 0 && ldx % 8 == 0)
+      rescore_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+    else
+      rescore_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+  } else {
+    if (al && d % 4 == 0 && ldx % 4 == 0)
+      rescore_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+    else
+      rescore_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+  }
   count_launch();
   return cudaGetLastError();
 }

@@ -68,7 +68,7 @@ struct Layout {
   size_t xhi, xlo;  // bf16[N * ldp] (fp32 features only)
   size_t cb_hi, cb_lo;  // bf16[Kp * ldp]
   size_t cn;        // f32[Kp]
-  size_t flagged;   // int32[N]: rows queued for the exact re-score
+  size_t flagged;   // int32[3N]: rows queued for the exact re-score, with their candidates
   size_t perm, slab;  // int32[N] each: sorted order of the labels (update)
   PartLayout part;  // partition scratch (update / route)
   size_t sums;      // f64[K * d]

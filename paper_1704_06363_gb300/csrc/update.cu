@@ -206,6 +206,13 @@ __global__ void __launch_bounds__(1024) update_reseed_kernel(const void *__restr
   __shared__ int64_t pick_i;
   __shared__ float pick_v;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // Nothing to do unless some cluster is empty (checked in parallel).
+  int any_empty = 0;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) any_empty |= (hist[k] == 0);
+  if (!__syncthreads_or(any_empty)) {
+    if (threadIdx.x == 0 && n_reseeded) *n_reseeded = 0;
+    return;
+  }
   float last_v = INFINITY;  // the previous pick; the next one comes strictly after it
   int64_t last_i = -1;
   int taken = 0;

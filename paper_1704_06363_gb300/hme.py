@@ -62,7 +62,7 @@ def lib():
         L.hme_partition.restype = ctypes.c_int
         L.hme_partition.argtypes = [p, i64, i32, p, p, p, p, p, p, p, p, p, sz, p]
         L.hme_route.restype = ctypes.c_int
-        L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, p, p, p, p, sz, p]
+        L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
         L.hme_launch_count.restype = i64
         L.hme_launch_count.argtypes = []
         L.hme_debug_bounded_wait.restype = ctypes.c_int
@@ -168,12 +168,12 @@ def hme_partition(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_
 
 
 def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offsets_out: torch.Tensor,
-              order_out: torch.Tensor, ws: torch.Tensor, stream=None):
+              order_out: torch.Tensor, ws: torch.Tensor, flags: int = HME_ASSIGN_DEFAULT, stream=None):
     B, d, ldq, dt = _features(Q)
     K = C.shape[0]
     w, wb = _ws(ws)
-    _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, _ptr(expert_out), _ptr(offsets_out), _ptr(order_out),
-                           w, wb, _stream(stream)), "hme_route")
+    _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, flags, _ptr(expert_out), _ptr(offsets_out),
+                           _ptr(order_out), w, wb, _stream(stream)), "hme_route")
 
 
 def hme_launch_count() -> int:

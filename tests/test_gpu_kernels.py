@@ -116,6 +116,40 @@ def test_assign_duplicate_centres_and_zero_rows(dev):
     parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_assign_near_ties_are_rescored_exactly(dev, dtype):
+    """Pairs of centres 1e-5 apart make most rows near ties: the exact re-score decides them."""
+    N, d, K = 3000, 256, 24
+    X = _mixture(N, d, 12, dtype, seed=21)
+    C = hme_synth.random_centroids(K, d, seed=4, scale=3.0)
+    C[:12] = X[:12].float()
+    g = torch.Generator().manual_seed(5)
+    C[12:] = C[:12] + 1e-5 * torch.randn(12, d, generator=g)  # near-duplicate partners
+    lab, md, obj = _assign(X, C, dev)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+
+
+def test_route_reuses_prepared_features(dev):
+    N, d, K = 4000, 128, 16
+    X = _mixture(N, d, K, "f32", seed=8)
+    C = hme_synth.random_centroids(K, d, seed=8, scale=3.0)
+    C[:8] = X[:8]
+    Xg, Cg = X.to(dev), C.to(dev)
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, hme.HME_F32, device=dev)
+    outs = []
+    for flags in (hme.HME_ASSIGN_DEFAULT, hme.HME_ASSIGN_PREPARED):
+        if flags == hme.HME_ASSIGN_PREPARED:
+            hme.hme_prepare_features(Xg, K, ws)
+        e = torch.empty(N, dtype=torch.int32, device=dev)
+        o = torch.empty(K + 1, dtype=torch.int64, device=dev)
+        r = torch.empty(N, dtype=torch.int32, device=dev)
+        hme.hme_route(Xg, Cg, e, o, r, ws, flags=flags)
+        assert hme.hme_sync_status(ws) == hme.HME_OK
+        outs.append((e.cpu(), o.cpu(), r.cpu()))
+    assert all(torch.equal(a, b) for a, b in zip(*outs))
+
+
 def test_assign_empty_input(dev):
     X = torch.empty(0, 64, dtype=torch.float32)
     C = hme_synth.random_centroids(4, 64, seed=1)
