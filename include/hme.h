@@ -207,6 +207,28 @@ HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t 
                       int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,
                       size_t ws_bytes, void *stream);
 
+/*
+ * hme_partition_noalloc -- the same stable partition as hme_partition (same
+ * outputs, bit for bit; no tag lists) for callers that cannot allocate device
+ * memory: code that must not call cudaMalloc/cudaFree where it routes a batch
+ * (they can synchronise the whole device, e.g. a serving loop), or code whose
+ * device memory is entirely owned by another framework's pool.  The paper has
+ * no counterpart; this is a deployment convenience.
+ *   No workspace: the scratch (status word + per-tile bucket counts) is a fixed
+ *   16 MiB array in device memory that every GPU loading the library holds
+ *   until exit.  The first call on a device, with that device current, looks up
+ *   the array's address (cudaGetSymbolAddress); make that first call before any
+ *   stream capture.  Calls share the array: calls that overlap on the GPU (two
+ *   streams, two host threads) race and must not be issued.  The tile length
+ *   grows so the counts fit; a size that still does not fit returns HME_EINVAL.
+ *   *status_out (device int32, may be NULL) = 0, or 1 if a label outside
+ *   [0, K) was seen and skipped.  Calls no cudaMalloc, cudaFree or allocating
+ *   library routine.
+ */
+HME_API int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out,
+                                  int64_t *offsets_out, int32_t *perm_out, int32_t *sorted_labels_out,
+                                  int32_t *status_out, void *stream);
+
 /* Number of kernels this library has launched in this process (diagnostic). */
 HME_API int64_t hme_launch_count(void);
 

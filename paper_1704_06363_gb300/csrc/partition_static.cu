@@ -1,0 +1,103 @@
+// partition_static.cu -- hme_partition_noalloc: the expert partition for
+// callers that cannot allocate device memory.
+//
+// Some callers cannot hand this library a workspace: a serving loop that must
+// not call cudaMalloc/cudaFree on its request path (both can synchronise the
+// whole device), or an application whose device memory is entirely owned by
+// another framework's pool.  This entry point needs no workspace: its only
+// scratch (a status word and the per-tile bucket counts of the stable
+// counting sort) lives in a fixed array in device global memory that is part
+// of the library image.
+//
+// - The array is kStaticScratchBytes = 16 MiB.  Every GPU that loads the
+//   library holds it until the process exits.
+// - Set-up: the first call on each device, with that device current, looks up
+//   the array's device address with cudaGetSymbolAddress (host code cannot use
+//   the array's name as a device address).  Make that first call before any
+//   stream capture.
+// - Every call shares the array and it keeps the last call's contents: the
+//   status word is cleared at the start of each call; the tile counts are fully
+//   rewritten.  Calls that overlap on the GPU (different streams, or several
+//   host threads) race on the array and must not be issued.
+// - Sizes: the tile length grows so that the ntiles x K counts always fit; a
+//   size that would still not fit is rejected with HME_EINVAL.
+// - No cudaMalloc, cudaFree or allocating library routine is called.
+#include "hme_common.cuh"
+
+#include <mutex>
+
+namespace hme {
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;
+constexpr int64_t kStaticTileRound = 512;
+
+static __device__ __align__(256) unsigned char g_partition_scratch[kStaticScratchBytes];
+
+std::mutex g_scratch_mu;
+void *g_scratch_ptr[64] = {};
+
+// Device address of g_partition_scratch on the current device (set-up on first use).
+int static_scratch(void **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(HME_EINTERNAL, "hme_partition_noalloc: device %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_partition_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: cudaGetSymbolAddress");
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return HME_OK;
+}
+
+}  // namespace
+}  // namespace hme
+
+using namespace hme;
+
+extern "C" int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out,
+                                     int64_t *offsets_out, int32_t *perm_out, int32_t *sorted_labels_out,
+                                     int32_t *status_out, void *stream) {
+  if (N < 0 || N > (int64_t)0x7FFFFFFF) return fail(HME_EINVAL, "N = %lld out of range", (long long)N);
+  if (K < 1 || K > kMaxK) return fail(HME_EINVAL, "K = %d out of range [1, %d]", K, kMaxK);
+  if (!hist_out || !offsets_out) return fail(HME_EINVAL, "hist_out / offsets_out is NULL");
+  if (N > 0 && (!labels || !perm_out)) return fail(HME_EINVAL, "labels / perm_out is NULL");
+
+  // Tile counts go right after the 256-byte header; lengthen tiles until they fit.
+  PartLayout pl = part_layout(sizeof(Header), N, K);
+  const size_t room = kStaticScratchBytes - sizeof(Header);
+  const int64_t max_tiles = (int64_t)(room / ((size_t)K * sizeof(int32_t)));
+  if (max_tiles < 1) return fail(HME_EINVAL, "K = %d needs more than %zu bytes of static scratch", K, room);
+  if (pl.ntiles > max_tiles) {
+    int64_t tile = (N + max_tiles - 1) / max_tiles;
+    tile = (tile + kStaticTileRound - 1) / kStaticTileRound * kStaticTileRound;
+    pl.tile = tile;
+    pl.ntiles = (N + tile - 1) / tile;
+  }
+  pl.tilecnt = sizeof(Header);
+  const size_t need = sizeof(Header) + (size_t)pl.ntiles * K * sizeof(int32_t);
+  if (need > kStaticScratchBytes)
+    return fail(HME_EINVAL, "N = %lld, K = %d needs %zu bytes of static scratch; the maximum is %zu", (long long)N, K,
+                need, kStaticScratchBytes);
+
+  void *scratch = nullptr;
+  int rc = static_scratch(&scratch);
+  if (rc != HME_OK) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Header *hdr = static_cast<Header *>(scratch);
+  cudaError_t e = cudaMemsetAsync(hdr, 0, sizeof(Header), s);  // the status word must start at zero
+  if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: clear status");
+  e = launch_partition(labels, N, K, pl, static_cast<char *>(scratch), hist_out, offsets_out, perm_out,
+                       sorted_labels_out, hdr, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc");
+  if (status_out) {
+    e = cudaMemcpyAsync(status_out, &hdr->status, sizeof(int32_t), cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: copy status");
+  }
+  return HME_OK;
+}

@@ -63,6 +63,8 @@ def lib():
         L.hme_partition.argtypes = [p, i64, i32, p, p, p, p, p, p, p, p, p, sz, p]
         L.hme_route.restype = ctypes.c_int
         L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
+        L.hme_partition_noalloc.restype = ctypes.c_int
+        L.hme_partition_noalloc.argtypes = [p, i64, i32, p, p, p, p, p, p]
         L.hme_launch_count.restype = i64
         L.hme_launch_count.argtypes = []
         L.hme_debug_bounded_wait.restype = ctypes.c_int
@@ -174,6 +176,16 @@ def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offset
     w, wb = _ws(ws)
     _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, flags, _ptr(expert_out), _ptr(offsets_out),
                            _ptr(order_out), w, wb, _stream(stream)), "hme_route")
+
+
+def hme_partition_noalloc(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_out: torch.Tensor,
+                          perm_out: torch.Tensor, sorted_labels_out: Optional[torch.Tensor] = None,
+                          status_out: Optional[torch.Tensor] = None, stream=None):
+    """hme_partition without a workspace (for callers that cannot allocate device memory)."""
+    N = labels.shape[0]
+    _check(lib().hme_partition_noalloc(_ptr(labels), N, K, _ptr(hist_out), _ptr(offsets_out), _ptr(perm_out),
+                                       _ptr(sorted_labels_out), _ptr(status_out), _stream(stream)),
+           "hme_partition_noalloc")
 
 
 def hme_launch_count() -> int:
