@@ -66,7 +66,7 @@ def _load():
         lib.orc_bf16_to_f32.argtypes = [ctypes.c_uint16]
         lib.orc_kmeanspp.restype = i32
         lib.orc_kmeanspp.argtypes = [p, i64, i64, i64, i32, i64, u64, i32, p, p]
-        lib.orc_assign.restype = None
+        lib.orc_assign.restype = i32
         lib.orc_assign.argtypes = [p, i64, i64, i64, i32, p, i64, p, p, p, p]
         lib.orc_objective.restype = i32
         lib.orc_objective.argtypes = [p, i64, i64, i64, i32, p, i64, p, p]
@@ -146,7 +146,8 @@ def assign(X, C, dtype: str = "f32"):
     d1 = np.zeros(N, np.float64)
     d2 = np.zeros(N, np.float64)
     J = ctypes.c_double(0.0)
-    _load().orc_assign(_ptr(X), N, d, d, code, _ptr(C), K, _ptr(labels), _ptr(d1), _ptr(d2), ctypes.byref(J))
+    if _load().orc_assign(_ptr(X), N, d, d, code, _ptr(C), K, _ptr(labels), _ptr(d1), _ptr(d2), ctypes.byref(J)):
+        raise MemoryError("orc_assign: allocation failed")
     return labels, d1, d2, J.value
 
 

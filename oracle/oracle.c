@@ -105,14 +105,19 @@ static double feat(const void *X, int dtype, int64_t ldx, int64_t i, int64_t j)
     return (double)((const float *)X)[i * ldx + j];
 }
 
-/* The centre coordinate the assign step compares against: the stored fp32
- * value, or its bf16 rounding when the features are bf16. */
-static double centre(const float *C, int64_t d, int dtype, int64_t k, int64_t j)
+/* The centre coordinates the assign step compares against, as fp64: the stored
+ * fp32 values, or their bf16 rounding when the features are bf16.  Returns a
+ * malloc'd K x d table (NULL on allocation failure). */
+static double *centre_table(const float *C, int64_t K, int64_t d, int dtype)
 {
-    float c = C[k * d + j];
-    if (dtype == ORC_BF16)
-        return (double)orc_bf16_to_f32(orc_f32_to_bf16_rne(c));
-    return (double)c;
+    double *T = (double *)malloc((size_t)(K * d > 0 ? K * d : 1) * sizeof(double));
+    if (!T)
+        return NULL;
+    for (int64_t i = 0; i < K * d; ++i) {
+        float c = C[i];
+        T[i] = (dtype == ORC_BF16) ? (double)orc_bf16_to_f32(orc_f32_to_bf16_rne(c)) : (double)c;
+    }
+    return T;
 }
 
 /* ||x_i - y||^2 by the direct sum, j ascending, fp64. */
@@ -198,6 +203,7 @@ int orc_kmeanspp(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
             picked_out[k] = row;
         for (int64_t j = 0; j < d; ++j)
             C_out[k * d + j] = (float)feat(X, dtype, ldx, row, j);
+#pragma omp parallel for schedule(static)
         for (int64_t j = 0; j < m; ++j) {
             double dj = dist2_row_row(X, dtype, ldx, d, rows[j], row);
             if (k == 0 || dj < D2[j])
@@ -217,10 +223,13 @@ int orc_kmeanspp(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
 /* objective = sum_i d1[i], summed in ascending i.  Rows are independent,   */
 /* so the loop over i may run on several threads without changing a value. */
 /* ---------------------------------------------------------------------- */
-void orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
-                const float *C, int64_t K,
-                int32_t *labels, double *d1, double *d2, double *objective)
+int orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
+               const float *C, int64_t K,
+               int32_t *labels, double *d1, double *d2, double *objective)
 {
+    double *Ct = centre_table(C, K, d, dtype);
+    if (!Ct)
+        return -1;
 #pragma omp parallel for schedule(dynamic, 64)
     for (int64_t i = 0; i < N; ++i) {
         double best = INFINITY, second = INFINITY;
@@ -228,7 +237,7 @@ void orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
         for (int64_t k = 0; k < K; ++k) {
             double s = 0.0;
             for (int64_t j = 0; j < d; ++j) {
-                double t = feat(X, dtype, ldx, i, j) - centre(C, d, dtype, k, j);
+                double t = feat(X, dtype, ldx, i, j) - Ct[k * d + j];
                 s += t * t;
             }
             if (s < best) {
@@ -253,6 +262,8 @@ void orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
         }
         *objective = J;
     }
+    free(Ct);
+    return 0;
 }
 
 /* ---------------------------------------------------------------------- */
@@ -263,17 +274,22 @@ void orc_assign(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
 int orc_objective(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
                   const float *C, int64_t K, const int32_t *labels, double *objective)
 {
-    double J = 0.0;
-    for (int64_t i = 0; i < N; ++i) {
+    for (int64_t i = 0; i < N; ++i)
         if (labels[i] < 0 || labels[i] >= K)
             return -1;
+    double *Ct = centre_table(C, K, d, dtype);
+    if (!Ct)
+        return -1;
+    double J = 0.0;
+    for (int64_t i = 0; i < N; ++i) {
         double s = 0.0;
         for (int64_t j = 0; j < d; ++j) {
-            double t = feat(X, dtype, ldx, i, j) - centre(C, d, dtype, labels[i], j);
+            double t = feat(X, dtype, ldx, i, j) - Ct[(int64_t)labels[i] * d + j];
             s += t * t;
         }
         J += s;
     }
+    free(Ct);
     *objective = J;
     return 0;
 }
@@ -416,7 +432,9 @@ int orc_lloyd(const void *X, int64_t N, int64_t d, int64_t ldx, int dtype,
     int rc = 0;
     for (int64_t t = 0; t < T && rc == 0; ++t) {
         double J = 0.0;
-        orc_assign(X, N, d, ldx, dtype, C_inout, K, labels_out, d1, NULL, &J);
+        rc = orc_assign(X, N, d, ldx, dtype, C_inout, K, labels_out, d1, NULL, &J);
+        if (rc != 0)
+            break;
         if (objectives)
             objectives[t] = J;
         if (changed) {
