@@ -260,6 +260,7 @@ def run_ours(args, w):
     torch.cuda.synchronize(dev)
     launches = hme.hme_launch_count() - launches0
     ck = clocks.stop()
+    rescored = int(ws[4:8].view(torch.int32).item())  # rows queued by the last assign (the route's)
     ms = e0.elapsed_time(e1)
     if world > 1:
         t = torch.tensor([ms], device=dev, dtype=torch.float64)
@@ -350,6 +351,7 @@ def run_ours(args, w):
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches,
+            "rescored_rows_last_assign": rescored,
             "clocks": ck,
         }
         print(json.dumps(line), flush=True)

@@ -139,10 +139,13 @@ HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ld
  * cores (fp32 accumulate): for HME_BF16 features, x.bf16(c) with c rounded to
  * bf16 (round to nearest even); for HME_F32, the bf16 split x = xh + xl,
  * c = ch + cl and the four products xh.ch + xh.cl + xl.ch + xl.cl, with the
- * norms taken of the same split values.  Rows whose two best distances lie within a
- * relative 2e-4 of each other (of max(D2, ||x||^2)) are re-scored against
- * every centre with direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of
- * non-negative terms).  The N x K distance matrix is never written.
+ * norms taken of the same split values.  A row whose runner-up distance is
+ * within E of its best, E a bound on the error of a difference of two computed
+ * distances (ceil(d/16) * nprod * 2^-22 (||x||^2 + max_k ||c_k||^2), plus
+ * 2^-14 (||x|| + max ||c||) sqrt(D2) for split fp32 operands), is re-scored
+ * exactly on its candidates (all K when a third centre is also within E) with
+ * direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of non-negative
+ * terms).  The N x K distance matrix is never written.
  * X: N x d (ldx, dtype); C: K x d float32 (read only); labels_out: int32[N].
  * flags: HME_ASSIGN_DEFAULT, or HME_ASSIGN_PREPARED (skip the per-call
  * hme_prepare_features pass; ws must hold this X's preparation).

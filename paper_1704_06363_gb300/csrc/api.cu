@@ -178,7 +178,7 @@ int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const flo
   const AssignGeom g = assign_geom(d, K, dtype);
   Header *hdr = at<Header>(ws, 0);
   HME_CUDA(launch_prep_centres(C, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
-                               at<float>(ws, L.cn), s),
+                               at<float>(ws, L.cn), hdr, s),
            "prepare centres");
   const void *Xa = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xhi) : X;
   const void *Xb = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;

@@ -52,11 +52,51 @@ struct AssignParams {
   Header *hdr;
   int32_t *flagged;
   uint64_t limit_ns;
-  float margin;
+  float err_acc;    // ceil(d/16) * nprod * 2^-22 + 2^-20: accumulation + epilogue rounding
+  float err_split;  // 2^-14 for split fp32 operands, else 0
 };
 
 constexpr int kThreads = 192;
 constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4;
+
+// One group of 16 accumulator columns of one row: v_j = ||c_j||^2 - 2 x.c_j.
+// The running best three values (and the indices of the best two) change only
+// when the group's minimum is below the third best, which after the first few
+// groups is rare; that test is one compare per 16 columns.
+__device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const float *cn16, int k0, float &best1,
+                                               float &best2, float &best3, int &idx1, int &idx2) {
+  float v[16];
+  const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
+  float m = INFINITY;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 cc = c4[q];
+    v[4 * q + 0] = fmaf(-2.0f, __uint_as_float(r[4 * q + 0]), cc.x);
+    v[4 * q + 1] = fmaf(-2.0f, __uint_as_float(r[4 * q + 1]), cc.y);
+    v[4 * q + 2] = fmaf(-2.0f, __uint_as_float(r[4 * q + 2]), cc.z);
+    v[4 * q + 3] = fmaf(-2.0f, __uint_as_float(r[4 * q + 3]), cc.w);
+    m = fminf(m, fminf(fminf(v[4 * q], v[4 * q + 1]), fminf(v[4 * q + 2], v[4 * q + 3])));
+  }
+  if (m < best3) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const float x = v[j];
+      if (x < best1) {
+        best3 = best2;
+        best2 = best1;
+        idx2 = idx1;
+        best1 = x;
+        idx1 = k0 + j;
+      } else if (x < best2) {
+        best3 = best2;
+        best2 = x;
+        idx2 = k0 + j;
+      } else if (x < best3) {
+        best3 = x;
+      }
+    }
+  }
+}
 
 template <int NPROD>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -203,6 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue: argmin over the accumulator rows ----------------
     const int q = warp & 3;          // TMEM lane quarter this warp may access
     float *cb = cnbuf + (warp - 2) * kMaxBN;  // this warp's copy of ||c||^2 for the chunk
+    const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
+    const float sqrt_cn_max = sqrtf(cn_max);
     const int row_in_tile = q * 32 + lane;
     uint32_t acc_it = 0;
     bool ok = true;
@@ -223,26 +265,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
         const int kbase = ch * p.BN;
-        for (int c = 0; c < p.BN; c += 16) {
-          uint32_t r[16];
-          tmem_ld16(taddr + (uint32_t)c, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float v = fmaf(-2.0f, __uint_as_float(r[j]), cb[c + j]);
-            if (v < best1) {
-              best3 = best2;
-              best2 = best1;
-              idx2 = idx1;
-              best1 = v;
-              idx1 = kbase + c + j;
-            } else if (v < best2) {
-              best3 = best2;
-              best2 = v;
-              idx2 = kbase + c + j;
-            } else if (v < best3) {
-              best3 = v;
-            }
+        // 16 columns per step; the next step's tcgen05.ld is in flight while this
+        // step's distances are formed.  Fast path: the minimum of the 16 values
+        // (branch-free); the top-3 insertion only runs when it beats the third best.
+        uint32_t ra[16], rb[16];
+        tmem_ld16(taddr, ra);
+        tmem_ld_wait(ra);
+        for (int c = 0; c < p.BN; c += 32) {
+          const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+          if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
+          epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
+          if (more1) {
+            tmem_ld_wait(rb);
+            if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
+            epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
+            if (more2) tmem_ld_wait(ra);
           }
         }
         tc_fence_before();
@@ -259,12 +296,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float md = fmaxf(D1, 0.0f);
         p.labels[row] = idx1;
         if (p.mind) p.mind[row] = md;
-        // Near tie: the runner-up (and maybe the third) could be the true nearest
-        // centre within the error of the tensor-core distances; queue the row for
-        // an exact comparison of the candidates (all K if a third one is close).
-        const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= p.margin * fmaxf(D2, xr));
+        // Near tie: a centre whose tensor-core distance is within E of the best
+        // could be the true nearest one.  E bounds the error of a difference of
+        // two computed distances: each fp32 accumulation step of x.c errs by at
+        // most one ulp of the accumulator (|x.c| <= (||x||^2 + ||c||^2) / 2),
+        // the split operands of fp32 features by 2^-16 per element, and the
+        // epilogue adds a few roundings.  Such rows are queued for an exact
+        // comparison of the candidates (all K if a third one is also within E).
+        const float E = p.err_acc * (xr + cn_max) +
+                        p.err_split * (sqrtf(xr) + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f));
+        const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
         if (near2) {
-          const bool near3 = (best3 < INFINITY) && ((D3 - D1) <= p.margin * fmaxf(D3, xr));
+          const bool near3 = (best3 < INFINITY) && ((D3 - D1) <= E);
           const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
           p.flagged[3 * slot + 0] = (int32_t)row;
           p.flagged[3 * slot + 1] = idx1;
@@ -496,7 +539,8 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.hdr = hdr;
   p.flagged = flagged;
   p.limit_ns = wait_limit_ns();
-  p.margin = 2e-4f;
+  p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
+  p.err_split = g.nprod == 4 ? 0x1p-14f : 0.0f;
   const size_t smem = (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
   int grid = num_sms();
   if (grid > p.num_tiles) grid = p.num_tiles;

@@ -28,7 +28,8 @@ struct Header {          // lives at ws + 0, 256 bytes
   uint32_t pad0;
   double objective;      // fp64 objective accumulator of hme_assign
   uint32_t wait_where;   // which bounded wait expired (diagnostic)
-  uint32_t pad1[57];
+  uint32_t cn_max_bits;  // max_k ||c_k||^2 of the prepared centres (float bits; values are >= 0)
+  uint32_t pad1[56];
 };
 static_assert(sizeof(Header) == 256, "header is 256 bytes");
 
@@ -96,7 +97,7 @@ uint64_t wait_limit_ns();
 cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, int dtype, const AssignGeom &g,
                                  float *xn, __nv_bfloat16 *xhi, __nv_bfloat16 *xlo, cudaStream_t s);
 cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
-                                float *cn, cudaStream_t s);
+                                float *cn, Header *hdr, cudaStream_t s);
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, cudaStream_t s);
@@ -262,6 +263,16 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
 }
 
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Wait for outstanding tcgen05.ld and tie the 16 destination registers to the
+// wait, so that no use of them can be scheduled before it.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
 
 // Shared-memory matrix descriptor for a K-major operand stored in the 128-byte
 // swizzled layout that TMA writes with CU_TENSOR_MAP_SWIZZLE_128B: rows of 128

@@ -11,7 +11,9 @@
 //                  vector loads, read once (HBM-bound).
 //   prep_centres   every iteration: bf16(c) (bf16 features) or the split
 //                  ch, cl (fp32 features), and cn[k] = ||c_eff||^2 of exactly
-//                  the values the MMA consumes; cn = +inf for padding centres.
+//                  the values the MMA consumes; cn = +inf for padding centres;
+//                  max_k cn[k] goes to the workspace header (error bound of the
+//                  assign step's near-tie test).
 #include "hme_common.cuh"
 
 namespace hme {
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(256) prep_bf16_kernel(const __nv_bfloat16 *__r
 __global__ void __launch_bounds__(256) prep_centres_kernel(const float *__restrict__ C, int K, int Kp, int d,
                                                            int ldp, int nprod, __nv_bfloat16 *__restrict__ chi,
                                                            __nv_bfloat16 *__restrict__ clo,
-                                                           float *__restrict__ cn) {
+                                                           float *__restrict__ cn, Header *hdr) {
   const int lane = threadIdx.x & 31;
   const int k = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
   if (k >= Kp) return;
@@ -157,7 +159,10 @@ __global__ void __launch_bounds__(256) prep_centres_kernel(const float *__restri
     s = fmaf(ce, ce, s);
   }
   s = warp_sum(s);
-  if (lane == 0) cn[k] = s;
+  if (lane == 0) {
+    cn[k] = s;
+    atomicMax(&hdr->cn_max_bits, __float_as_uint(s));  // s >= 0: integer order is float order
+  }
 }
 
 }  // namespace
@@ -184,9 +189,9 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
 }
 
 cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
-                                float *cn, cudaStream_t s) {
+                                float *cn, Header *hdr, cudaStream_t s) {
   const int blocks = (g.Kp + 7) / 8;
-  prep_centres_kernel<<<blocks, 256, 0, s>>>(C, g.K, g.Kp, g.d, g.ldp, g.nprod, chi, clo, cn);
+  prep_centres_kernel<<<blocks, 256, 0, s>>>(C, g.K, g.Kp, g.d, g.ldp, g.nprod, chi, clo, cn, hdr);
   count_launch();
   return cudaGetLastError();
 }
