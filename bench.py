@@ -122,6 +122,17 @@ class Clocks:
                 "samples": len(sm)}
 
 
+def max_over_ranks(ms: float, device=None) -> float:
+    """Slowest rank's time: the whole job ends when the last replica ends."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle baseline (also the --impl reference arm)
 # ---------------------------------------------------------------------------
@@ -261,11 +272,7 @@ def run_ours(args, w):
     launches = hme.hme_launch_count() - launches0
     ck = clocks.stop()
     rescored = int(ws[4:8].view(torch.int32).item())  # rows queued by the last assign (the route's)
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
     assert hme.hme_sync_status(ws) == hme.HME_OK
 
     iters_total = T * args.steps * world
@@ -318,11 +325,7 @@ def run_ours(args, w):
             e2e_step()
         f1.record(stream)
         torch.cuda.synchronize(dev)
-        ms_e2e = f0.elapsed_time(f1)
-        if world > 1:
-            t = torch.tensor([ms_e2e], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms_e2e = float(t.item())
+        ms_e2e = max_over_ranks(f0.elapsed_time(f1), dev)
         e2e = {"value": iters_total / (ms_e2e / 1000.0), "unit": UNIT, "h2d_bytes_per_step": X.numel() * e,
                "d2h_bytes_per_step": 4 * N + 4 * N + 8 * (K + 1) + 4 * K * d, "ms_per_step": ms_e2e / args.steps}
         del Xh, Xd
