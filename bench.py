@@ -271,7 +271,8 @@ def run_ours(args, w):
     torch.cuda.synchronize(dev)
     launches = hme.hme_launch_count() - launches0
     ck = clocks.stop()
-    rescored = int(ws[4:8].view(torch.int32).item())  # rows queued by the last assign (the route's)
+    hdr = ws[:16].view(torch.int32).cpu()  # queues of the last assign (the route's): pairs, all-K
+    rescored = {"pair": int(hdr[1]), "all_k": int(hdr[3])}
     ms = max_over_ranks(e0.elapsed_time(e1), dev)
     assert hme.hme_sync_status(ws) == hme.HME_OK
 

@@ -91,6 +91,7 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   L.cb_lo = dtype == HME_F32 ? take((size_t)g.Kp * g.ldp * 2) : 0;
   L.cn = take((size_t)g.Kp * 4);
   L.flagged = take((size_t)(N > 0 ? N : 1) * 12);  // (row, best, runner-up) per queued row
+  L.full_rows = take((size_t)(N > 0 ? N : 1) * 4);
   L.perm = take((size_t)(N > 0 ? N : 1) * 4);
   L.slab = take((size_t)(N > 0 ? N : 1) * 4);
   L.part = part_layout(align_up(off, 256), N, K);
@@ -184,9 +185,10 @@ int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const flo
   const void *Xb = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;
   const int64_t lda = dtype == HME_F32 ? g.ldp : ldx;
   HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
-                        at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged), s));
-  HME_CUDA(launch_rescore(X, N, d, ldx, dtype, C, K, at<float>(ws, L.xn), labels, mind, hdr,
-                          at<int32_t>(ws, L.flagged), s),
+                        at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged),
+                        at<int32_t>(ws, L.full_rows), s));
+  HME_CUDA(launch_rescore(X, N, d, ldx, dtype, C, K, labels, mind, hdr, at<int32_t>(ws, L.flagged),
+                          at<int32_t>(ws, L.full_rows), s),
            "re-score");
   return HME_OK;
 }

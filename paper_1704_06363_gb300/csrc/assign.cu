@@ -50,7 +50,8 @@ struct AssignParams {
   int32_t *labels;
   float *mind;
   Header *hdr;
-  int32_t *flagged;
+  int32_t *flagged;    // (row, best, runner-up) of near-tie rows with two candidates
+  int32_t *full_rows;  // near-tie rows to compare with all K centres
   uint64_t limit_ns;
   float err_acc;    // ceil(d/16) * nprod * 2^-22 + 2^-20: accumulation + epilogue rounding
   float err_split;  // 2^-14 for split fp32 operands, else 0
@@ -98,7 +99,33 @@ __device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const fl
   }
 }
 
-template <int NPROD>
+// Lean variant for many centres (several N-chunks): per column
+// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
+// min(best, v), and the best's column -- six instructions, no branches.  jl is
+// the column of the best within this group; i1 moves only if the group
+// improved the best, so ties keep the lowest index.
+__device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float *cn16, int k0, float &b1, float &b2,
+                                           int &i1) {
+  const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
+  const float before = b1;
+  int jl = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 cc = c4[q];
+    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = 4 * q + e;
+      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[e]);
+      b2 = fminf(b2, fmaxf(b1, v));
+      jl = (v < b1) ? j : jl;
+      b1 = fminf(b1, v);
+    }
+  }
+  i1 = (b1 < before) ? k0 + jl : i1;
+}
+
+template <int NPROD, bool LEAN>
 __global__ void __launch_bounds__(kThreads, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
@@ -252,6 +279,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
       int idx1 = 0, idx2 = 0;
+      float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
+      int li1 = 0;
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
         __syncwarp();
         for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + ch * p.BN + t);
@@ -266,19 +295,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
         const int kbase = ch * p.BN;
         // 16 columns per step; the next step's tcgen05.ld is in flight while this
-        // step's distances are formed.  Fast path: the minimum of the 16 values
-        // (branch-free); the top-3 insertion only runs when it beats the third best.
+        // step's distances are formed.
         uint32_t ra[16], rb[16];
         tmem_ld16(taddr, ra);
         tmem_ld_wait(ra);
         for (int c = 0; c < p.BN; c += 32) {
           const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
           if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
-          epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
+          if (LEAN)
+            lean_group(ra, cb + c, kbase + c, best1, best2, idx1);
+          else
+            epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
           if (more1) {
             tmem_ld_wait(rb);
             if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
-            epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
+            if (LEAN)
+              lean_group(rb, cb + c + 16, kbase + c + 16, lb1, lb2, li1);
+            else
+              epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
             if (more2) tmem_ld_wait(ra);
           }
         }
@@ -287,6 +321,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
       }
       if (!ok) break;
+      if (LEAN) {  // merge the two lean states: lowest value, then lowest index
+        const bool take_b = lb1 < best1 || (lb1 == best1 && li1 < idx1);
+        best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
+        best1 = take_b ? lb1 : best1;
+        idx1 = take_b ? li1 : idx1;
+      }
       const int64_t row = (int64_t)tile * kBM + row_in_tile;
       if (row < p.N) {
         const float xr = __ldg(p.xn + row);
@@ -302,16 +342,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         // most one ulp of the accumulator (|x.c| <= (||x||^2 + ||c||^2) / 2),
         // the split operands of fp32 features by 2^-16 per element, and the
         // epilogue adds a few roundings.  Such rows are queued for an exact
-        // comparison of the candidates (all K if a third one is also within E).
+        // comparison: of the two candidates, or of all K when a third centre is
+        // also within E (or, in the lean scan, whenever the runner-up is).
         const float E = p.err_acc * (xr + cn_max) +
                         p.err_split * (sqrtf(xr) + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f));
         const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
         if (near2) {
-          const bool near3 = (best3 < INFINITY) && ((D3 - D1) <= E);
-          const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
-          p.flagged[3 * slot + 0] = (int32_t)row;
-          p.flagged[3 * slot + 1] = idx1;
-          p.flagged[3 * slot + 2] = near3 ? -1 : idx2;
+          const bool near3 = LEAN || ((best3 < INFINITY) && ((D3 - D1) <= E));
+          if (near3) {
+            const uint32_t slot = atomicAdd(&p.hdr->rescore_full_count, 1u);
+            p.full_rows[slot] = (int32_t)row;
+          } else {
+            const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
+            p.flagged[3 * slot + 0] = (int32_t)row;
+            p.flagged[3 * slot + 1] = idx1;
+            p.flagged[3 * slot + 2] = idx2;
+          }
         } else {
           obj += (double)md;
         }
@@ -389,35 +435,14 @@ __device__ __forceinline__ float warp_sum_f(float s) {
   return s;
 }
 
-// sum_j (x_j - c_j)^2 over one row, lanes striding by 32 * VW elements (d % VW == 0).
-template <int DT, int VW>
-__device__ __forceinline__ float row_dist2(const void *Xv, int64_t xoff, const float *C, int64_t coff, int d,
-                                           int lane) {
-  float s = 0.0f;
-#pragma unroll 4
-  for (int j = lane * VW; j < d; j += 32 * VW) {
-    float x[VW], c[VW];
-    load_x<DT, VW>(Xv, xoff + j, x);
-    load_c<DT, VW>(C, coff + j, c);
-#pragma unroll
-    for (int e = 0; e < VW; ++e) {
-      const float t = x[e] - c[e];
-      s = fmaf(t, t, s);
-    }
-  }
-  return warp_sum_f(s);
-}
 
-// Exact re-score of near-tie rows: direct differences, squared and summed per
-// lane in fp32 (a sum of non-negative terms), combined across the warp; ties to
-// the lowest k.  A queued row names its two candidates (best and runner-up of
-// the tensor-core pass), or -1 for "compare all K" when a third centre was also
-// within the margin.  One warp per queued row, 16-byte loads when the layout
-// allows.
+// Exact re-score of near-tie rows with two candidates: one warp per row, one
+// pass over the row computing both sums of squared differences (fp32 per lane,
+// a sum of non-negative terms, then across the warp); ties to the lower index.
 template <int DT, int VW>
-__global__ void __launch_bounds__(256) rescore_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
-                                                      const float *__restrict__ C, int K, int32_t *labels,
-                                                      float *mind, Header *hdr, const int32_t *__restrict__ flagged) {
+__global__ void __launch_bounds__(256) rescore_pair_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                           const float *__restrict__ C, int32_t *labels, float *mind,
+                                                           Header *hdr, const int32_t *__restrict__ flagged) {
   const int lane = threadIdx.x & 31;
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int nw = (gridDim.x * blockDim.x) >> 5;
@@ -427,32 +452,216 @@ __global__ void __launch_bounds__(256) rescore_kernel(const void *__restrict__ X
     const int64_t row = flagged[3 * f + 0];
     const int i1 = flagged[3 * f + 1];
     const int i2 = flagged[3 * f + 2];
-    float best;
-    int arg;
-    if (i2 >= 0) {
-      const float s1 = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)i1 * d, d, lane);
-      const float s2 = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)i2 * d, d, lane);
-      const bool first = s1 < s2 || (s1 == s2 && i1 < i2);
-      best = first ? s1 : s2;
-      arg = first ? i1 : i2;
-    } else {
-      best = INFINITY;
-      arg = 0;
-      for (int k = 0; k < K; ++k) {
-        const float s = row_dist2<DT, VW>(Xv, row * ldx, C, (int64_t)k * d, d, lane);
-        if (s < best) {
-          best = s;
-          arg = k;
-        }
+    float s1 = 0.0f, s2 = 0.0f;
+#pragma unroll 4
+    for (int j = lane * VW; j < d; j += 32 * VW) {
+      float x[VW], c1[VW], c2[VW];
+      load_x<DT, VW>(Xv, row * ldx + j, x);
+      load_c<DT, VW>(C, (int64_t)i1 * d + j, c1);
+      load_c<DT, VW>(C, (int64_t)i2 * d + j, c2);
+#pragma unroll
+      for (int e = 0; e < VW; ++e) {
+        const float t1 = x[e] - c1[e], t2 = x[e] - c2[e];
+        s1 = fmaf(t1, t1, s1);
+        s2 = fmaf(t2, t2, s2);
       }
     }
+    s1 = warp_sum_f(s1);
+    s2 = warp_sum_f(s2);
+    const bool first = s1 < s2 || (s1 == s2 && i1 < i2);
     if (lane == 0) {
-      labels[row] = arg;
-      if (mind) mind[row] = best;
-      obj += (double)best;
+      labels[row] = first ? i1 : i2;
+      if (mind) mind[row] = first ? s1 : s2;
+      obj += (double)(first ? s1 : s2);
     }
   }
   if (lane == 0 && obj != 0.0) atomicAdd(&hdr->objective, obj);
+}
+
+// Exact re-score against all K centres when K is small (one N-chunk): one block
+// per queued row; the row is cached in shared memory and the 8 warps split the
+// centres, each lane summing (x_j - c_j)^2 over its strided elements in fp32
+// (16-byte loads of c), then across the warp and across the warps; ties to the
+// lowest index.  Latency is about K/8 passes over one centre row.
+template <int DT, int VW>
+__global__ void __launch_bounds__(256) rescore_row_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                          const float *__restrict__ C, int K, int32_t *labels,
+                                                          float *mind, Header *hdr,
+                                                          const int32_t *__restrict__ full_rows) {
+  extern __shared__ float xrow[];
+  __shared__ float wv[8];
+  __shared__ int wk[8];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint32_t count = *((volatile uint32_t *)&hdr->rescore_full_count);
+  double obj = 0.0;
+  for (uint32_t f = blockIdx.x; f < count; f += gridDim.x) {
+    const int64_t row = full_rows[f];
+    for (int j = threadIdx.x; j < d; j += blockDim.x) {
+      float x;
+      if (DT == HME_BF16)
+        x = __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(Xv)[row * ldx + j]);
+      else
+        x = reinterpret_cast<const float *>(Xv)[row * ldx + j];
+      xrow[j] = x;
+    }
+    __syncthreads();
+    float bv = INFINITY;
+    int bk = 0x7fffffff;
+    for (int k = warp; k < K; k += 8) {
+      float sacc = 0.0f;
+#pragma unroll 4
+      for (int j = lane * VW; j < d; j += 32 * VW) {
+        float c[VW];
+        load_c<DT, VW>(C, (int64_t)k * d + j, c);
+#pragma unroll
+        for (int e = 0; e < VW; ++e) {
+          const float t = xrow[j + e] - c[e];
+          sacc = fmaf(t, t, sacc);
+        }
+      }
+      sacc = warp_sum_f(sacc);
+      if (sacc < bv) {  // k ascends within a warp
+        bv = sacc;
+        bk = k;
+      }
+    }
+    if (lane == 0) {
+      wv[warp] = bv;
+      wk[warp] = bk;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float v = wv[0];
+      int kk = wk[0];
+      for (int w = 1; w < 8; ++w)
+        if (wv[w] < v || (wv[w] == v && wk[w] < kk)) {
+          v = wv[w];
+          kk = wk[w];
+        }
+      labels[row] = kk;
+      if (mind) mind[row] = v;
+      obj += (double)v;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && obj != 0.0) atomicAdd(&hdr->objective, obj);
+}
+
+// Exact re-score of near-tie rows against all K centres: a small tiled
+// "distance GEMM" on the CUDA cores.  A block takes 32 queued rows and walks
+// the centres 64 at a time and the dimensions 32 at a time through shared
+// memory; thread (ty, tx) of a 16 x 16 grid owns rows {ty, ty+16} and centres
+// {tx, tx+16, tx+32, tx+48}.  sum_j (x_j - c_j)^2 is formed in fp32 per 32-wide
+// chunk and the chunk sums are added in fp32 (relative error below
+// (32 + d/32) 2^-24, all terms non-negative); the minimum over centres keeps
+// the lowest index among equal values.
+constexpr int kFR = 32, kFC = 64, kFD = 32;
+
+template <int DT>
+__global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                           const float *__restrict__ C, int K, int32_t *labels,
+                                                           float *mind, Header *hdr,
+                                                           const int32_t *__restrict__ full_rows) {
+  __shared__ float xs[kFR][kFD + 1];
+  __shared__ float cs[kFC][kFD + 1];
+  __shared__ float best_v[kFR];
+  __shared__ int best_k[kFR];
+  __shared__ int64_t rows[kFR];
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const uint32_t count = *((volatile uint32_t *)&hdr->rescore_full_count);
+  double obj = 0.0;
+  for (uint32_t b0 = blockIdx.x * kFR; b0 < count; b0 += gridDim.x * kFR) {
+    const int nr = (int)min((uint32_t)kFR, count - b0);
+    if (threadIdx.x < kFR) {
+      rows[threadIdx.x] = threadIdx.x < nr ? (int64_t)full_rows[b0 + threadIdx.x] : -1;
+      best_v[threadIdx.x] = INFINITY;
+      best_k[threadIdx.x] = 0;
+    }
+    __syncthreads();
+    for (int k0 = 0; k0 < K; k0 += kFC) {
+      float tot[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+      for (int j0 = 0; j0 < d; j0 += kFD) {
+        for (int e = threadIdx.x; e < kFR * kFD; e += 256) {
+          const int r = e / kFD, j = e - r * kFD;
+          const int64_t row = rows[r];
+          float x = 0.0f;
+          if (row >= 0 && j0 + j < d) {
+            if (DT == HME_BF16)
+              x = __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(Xv)[row * ldx + j0 + j]);
+            else
+              x = reinterpret_cast<const float *>(Xv)[row * ldx + j0 + j];
+          }
+          xs[r][j] = x;
+        }
+        for (int e = threadIdx.x; e < kFC * kFD; e += 256) {
+          const int c = e / kFD, j = e - c * kFD;
+          const int k = k0 + c;
+          float v = 0.0f;
+          if (k < K && j0 + j < d) {
+            v = __ldg(C + (int64_t)k * d + j0 + j);
+            if (DT == HME_BF16) v = __bfloat162float(__float2bfloat16_rn(v));
+          }
+          cs[c][j] = v;
+        }
+        __syncthreads();
+        float part[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll 8
+        for (int j = 0; j < kFD; ++j) {
+          const float x0 = xs[ty][j], x1 = xs[ty + 16][j];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float c = cs[tx + 16 * q][j];
+            const float t0 = x0 - c, t1 = x1 - c;
+            part[0][q] = fmaf(t0, t0, part[0][q]);
+            part[1][q] = fmaf(t1, t1, part[1][q]);
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) tot[r][q] += part[r][q];
+        __syncthreads();
+      }
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        float v = INFINITY;
+        int kk = 0x7fffffff;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int k = k0 + tx + 16 * q;
+          if (k < K && tot[r][q] < v) {
+            v = tot[r][q];
+            kk = k;
+          }
+        }
+#pragma unroll
+        for (int o = 8; o > 0; o >>= 1) {  // the 16 threads of one ty share a half-warp
+          const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+          const int ok = __shfl_xor_sync(0xffffffffu, kk, o);
+          if (ov < v || (ov == v && ok < kk)) {
+            v = ov;
+            kk = ok;
+          }
+        }
+        const int rl = ty + 16 * r;
+        if (tx == 0 && (v < best_v[rl] || (v == best_v[rl] && kk < best_k[rl]))) {
+          best_v[rl] = v;
+          best_k[rl] = kk;
+        }
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x < nr) {
+      const int64_t row = rows[threadIdx.x];
+      labels[row] = best_k[threadIdx.x];
+      if (mind) mind[row] = best_v[threadIdx.x];
+      obj += (double)best_v[threadIdx.x];
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
+  if ((threadIdx.x & 31) == 0 && obj != 0.0) atomicAdd(&hdr->objective, obj);
 }
 
 // ---------------------------------------------------------------------------
@@ -497,7 +706,7 @@ int make_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint
 
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
-                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, cudaStream_t s) {
+                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
   if (N == 0) return HME_OK;
   CUtensorMap mA0, mA1, mB0, mB1;
   int rc;
@@ -538,6 +747,7 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.mind = mind;
   p.hdr = hdr;
   p.flagged = flagged;
+  p.full_rows = full_rows;
   p.limit_ns = wait_limit_ns();
   p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
   p.err_split = g.nprod == 4 ? 0x1p-14f : 0.0f;
@@ -545,15 +755,12 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   int grid = num_sms();
   if (grid > p.num_tiles) grid = p.num_tiles;
   cudaError_t e;
-  if (g.nprod == 4) {
-    e = cudaFuncSetAttribute(assign_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
-    assign_kernel<4><<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
-  } else {
-    e = cudaFuncSetAttribute(assign_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
-    assign_kernel<1><<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
-  }
+  const bool lean = g.nchunks > 1;
+  auto kern = g.nprod == 4 ? (lean ? assign_kernel<4, true> : assign_kernel<4, false>)
+                           : (lean ? assign_kernel<1, true> : assign_kernel<1, false>);
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
+  kern<<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
   count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");
@@ -561,24 +768,44 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
 }
 
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
-                           const float *xn, int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
-                           cudaStream_t s) {
-  (void)xn;
+                           int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           const int32_t *full_rows, cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   const int grid = num_sms() * 4;
   const bool al = ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(C)) & 15u) == 0;
+  // all-K rows: block per row for few centres (low latency), tiled otherwise
+  const bool row_path = K <= 128;
+  const bool cvec = (reinterpret_cast<uintptr_t>(C) & 15u) == 0 && d % 4 == 0;
+  const size_t row_smem = (size_t)d * sizeof(float);
+  if (row_path && row_smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(dtype == HME_BF16 ? rescore_row_kernel<HME_BF16, 1>
+                                                           : (cvec ? rescore_row_kernel<HME_F32, 4>
+                                                                   : rescore_row_kernel<HME_F32, 1>),
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)row_smem);
+    if (e != cudaSuccess) return e;
+  }
   if (dtype == HME_BF16) {
     if (al && d % 8 == 0 && ldx % 8 == 0)
-      rescore_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
     else
-      rescore_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+    if (row_path)
+      rescore_row_kernel<HME_BF16, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+    else
+      rescore_full_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
   } else {
     if (al && d % 4 == 0 && ldx % 4 == 0)
-      rescore_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
     else
-      rescore_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+    if (row_path && cvec)
+      rescore_row_kernel<HME_F32, 4><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+    else if (row_path)
+      rescore_row_kernel<HME_F32, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+    else
+      rescore_full_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
   }
-  count_launch();
+  count_launch(2);
   return cudaGetLastError();
 }
 

@@ -23,9 +23,9 @@ enum : uint32_t {
 
 struct Header {          // lives at ws + 0, 256 bytes
   uint32_t status;       // OR of kStatus* bits
-  uint32_t rescore_count;  // rows flagged by the assign margin test
+  uint32_t rescore_count;  // near-tie rows queued with their two candidates
   uint32_t kpp_choice;   // k-means++: candidate picked in the current round
-  uint32_t pad0;
+  uint32_t rescore_full_count;  // near-tie rows queued for a comparison with all K centres
   double objective;      // fp64 objective accumulator of hme_assign
   uint32_t wait_where;   // which bounded wait expired (diagnostic)
   uint32_t cn_max_bits;  // max_k ||c_k||^2 of the prepared centres (float bits; values are >= 0)
@@ -69,7 +69,8 @@ struct Layout {
   size_t xhi, xlo;  // bf16[N * ldp] (fp32 features only)
   size_t cb_hi, cb_lo;  // bf16[Kp * ldp]
   size_t cn;        // f32[Kp]
-  size_t flagged;   // int32[3N]: rows queued for the exact re-score, with their candidates
+  size_t flagged;   // int32[3N]: near-tie rows queued with their two candidates
+  size_t full_rows; // int32[N]: near-tie rows queued for all K centres
   size_t perm, slab;  // int32[N] each: sorted order of the labels (update)
   PartLayout part;  // partition scratch (update / route)
   size_t sums;      // f64[K * d]
@@ -100,10 +101,10 @@ cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat
                                 float *cn, Header *hdr, cudaStream_t s);
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
-                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, cudaStream_t s);
+                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s);
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
-                           const float *xn, int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
-                           cudaStream_t s);
+                           int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           const int32_t *full_rows, cudaStream_t s);
 cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
                              int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,
                              cudaStream_t s);

@@ -116,15 +116,22 @@ def test_assign_duplicate_centres_and_zero_rows(dev):
     parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj)
 
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_assign_near_ties_are_rescored_exactly(dev, dtype):
-    """Pairs of centres 1e-5 apart make most rows near ties: the exact re-score decides them."""
-    N, d, K = 3000, 256, 24
-    X = _mixture(N, d, 12, dtype, seed=21)
+@pytest.mark.parametrize("dtype,K,copies", [("f32", 24, 2), ("bf16", 24, 2), ("f32", 24, 3), ("bf16", 600, 2),
+                                            ("f32", 600, 3)])
+def test_assign_near_ties_are_rescored_exactly(dev, dtype, K, copies):
+    """Groups of centres 1e-5 apart make most rows near ties: the exact re-score decides them.
+
+    Two copies exercise the two-candidate re-score, three the all-K one; K = 600
+    (three N-chunks) exercises the lean scan, whose near ties all go to all K.
+    """
+    N, d = 3000, 256
+    base = K // copies
+    X = _mixture(N, d, min(base, 64), dtype, seed=21 + K)
     C = hme_synth.random_centroids(K, d, seed=4, scale=3.0)
-    C[:12] = X[:12].float()
+    C[:base] = X[:base].float()
     g = torch.Generator().manual_seed(5)
-    C[12:] = C[:12] + 1e-5 * torch.randn(12, d, generator=g)  # near-duplicate partners
+    for r in range(1, copies):
+        C[r * base:(r + 1) * base] = C[:base] + 1e-5 * torch.randn(base, d, generator=g)
     lab, md, obj = _assign(X, C, dev)
     st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
     assert st["mismatches"] <= st["near_ties"]
