@@ -158,13 +158,23 @@ HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t
  * hme_update_centroids -- the K-means centre step (Section 2, "K-means
  * clustering" of the z_j):
  *   counts_out[k] = |{i : labels[i] = k}| (int64, may be NULL),
- *   C_inout[k]    = (sum_{labels[i]=k} x_i) / counts[k], summed by segment in
- *                   fp32 and across segments in fp64, stored as float32,
+ *   C_inout[k]    = (sum_{labels[i]=k} x_i) / counts[k] (fp64 sums, stored as
+ *                   float32),
  *   *objective_out = sum_i ||x_i - c_{labels[i]}||^2 for the centres as they
  *                   were on entry (bf16-rounded for HME_BF16 features, as in
- *                   hme_assign), by direct differences in the same pass over X
- *                   (one device double, may be NULL).  With the labels of the
- *                   preceding hme_assign this is the Lloyd objective J_t.
+ *                   hme_assign), evaluated in fp64 as sum ||x||^2
+ *                   - 2 sum_k c_k . S_k + sum_k n_k ||c_k||^2 from the
+ *                   per-cluster sums S_k (one device double, may be NULL).
+ *                   With the labels of the preceding hme_assign this is the
+ *                   Lloyd objective J_t.
+ * The per-cluster sums, counts and sum ||x||^2 stay in ws after the call.
+ * prev_labels == NULL: they are recomputed from all N rows (segmented sums in
+ * label order).  prev_labels != NULL: ws must hold the state left by the
+ * previous hme_update_centroids call on the same X and ws, made with labels
+ * equal to prev_labels (and no other call with this ws in between but
+ * hme_assign / hme_prepare_features); only rows whose label differs from
+ * prev_labels are read and moved between clusters.  Both give Lloyd's centres
+ * (the same sums up to fp64 rounding order).
  * Empty clusters (the paper is silent; Section 4.5 reports every cluster used)
  * are re-seeded in ascending k: each takes the not-yet-taken row with the
  * largest mind[i], ties to the lowest i, as its centre (copied exactly); that
@@ -174,9 +184,9 @@ HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t
  * Labels outside [0, K) are skipped and reported by hme_sync_status.
  */
 HME_API int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
-                         const int32_t *labels, const float *mind, int32_t K, float *C_inout,
-                         int64_t *counts_out, int32_t *n_reseeded_out, double *objective_out, void *ws,
-                         size_t ws_bytes, void *stream);
+                                 const int32_t *labels, const int32_t *prev_labels, const float *mind, int32_t K,
+                                 float *C_inout, int64_t *counts_out, int32_t *n_reseeded_out,
+                                 double *objective_out, void *ws, size_t ws_bytes, void *stream);
 
 /*
  * hme_partition -- each expert's share of the training set (Section 2: "each

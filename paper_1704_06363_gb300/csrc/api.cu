@@ -56,17 +56,36 @@ uint64_t wait_limit_ns() {
   return v;
 }
 
+// Tile shape of the assign kernel.  Every 128-row tile re-reads all centre
+// tiles from L2, so for bf16 features (one product, tensor-bound when K is
+// large) two row tiles share each centre stage (MT = 2): up to 256 centres per
+// N-chunk, single-buffered in TMEM when 2 x BN needs all 512 columns.  With
+// several N-chunks and few dimensions the CTA's 256 rows stay resident in
+// shared memory (ARES) and the chunks hold 128 centres (double-buffered).  fp32
+// features (four products, 2 operands per side) keep MT = 1.
 AssignGeom assign_geom(int d, int K, int dtype) {
   AssignGeom g;
   g.d = d;
   g.K = K;
   g.dtype = dtype;
   g.ldp = (d + 7) / 8 * 8;
-  g.nchunks = (K + kMaxBN - 1) / kMaxBN;
+  g.nprod = dtype == HME_F32 ? 4 : 1;
+  const int num_kb = (d + kBK - 1) / kBK;
+  int max_bn = kMaxBN;
+  g.mt = 1;
+  g.ares = false;
+  if (g.nprod == 1) {
+    g.mt = 2;
+    if (K > kMaxBN && 2 * num_kb * (kBM * kBK * 2) <= 128 * 1024) {
+      g.ares = true;
+      max_bn = 128;
+    }
+  }
+  g.nchunks = (K + max_bn - 1) / max_bn;
   const int per = (K + g.nchunks - 1) / g.nchunks;
   g.BN = (per + 15) / 16 * 16;
   g.Kp = g.BN * g.nchunks;
-  g.nprod = dtype == HME_F32 ? 4 : 1;
+  g.nbuf = (g.mt * g.BN <= 256) ? 2 : 1;
   return g;
 }
 
@@ -97,6 +116,10 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   L.part = part_layout(align_up(off, 256), N, K);
   off = L.part.end;
   L.sums = take((size_t)K * d * 8);
+  L.counts = take((size_t)K * 8);
+  L.x2sum = take(8);
+  L.delta_k = take((size_t)4 * K * 4 + 16);
+  L.reseed = take((size_t)kMaxSms * 2 * 8 * 64 * 8);  // (2 blocks x 8 warps per SM) x 64 keys
   if (kpp_m > 0) {
     L.kpp_rows = take((size_t)kpp_m * 4);
     L.kpp_d2 = take((size_t)kpp_m * 8);
@@ -296,8 +319,9 @@ int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, 
 }
 
 int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const int32_t *labels,
-                         const float *mind, int32_t K, float *C_inout, int64_t *counts_out, int32_t *n_reseeded_out,
-                         double *objective_out, void *ws, size_t ws_bytes, void *stream) {
+                         const int32_t *prev_labels, const float *mind, int32_t K, float *C_inout,
+                         int64_t *counts_out, int32_t *n_reseeded_out, double *objective_out, void *ws,
+                         size_t ws_bytes, void *stream) {
   HME_TRY(check_common(N, d, K, dtype));
   HME_TRY(check_features(X, N, d, ldx, dtype, false));
   if (!C_inout) return fail(HME_EINVAL, "C_inout is NULL");
@@ -311,10 +335,16 @@ int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32
   int64_t *offs = at<int64_t>(ws, L.part.offs);
   int32_t *perm = at<int32_t>(ws, L.perm);
   int32_t *slab = at<int32_t>(ws, L.slab);
-  HME_CUDA(launch_partition(labels, N, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab, hdr, s),
-           "update: sort labels");
-  HME_CUDA(launch_update(X, N, d, ldx, dtype, perm, slab, hist, offs + K, mind, K, at<double>(ws, L.sums), C_inout,
-                         counts_out, n_reseeded_out, hdr, s),
+  if (!prev_labels)
+    HME_CUDA(launch_partition(labels, N, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab, hdr, s),
+             "update: sort labels");
+  UpdateState st{at<double>(ws, L.sums), at<int64_t>(ws, L.counts), at<double>(ws, L.x2sum)};
+  int32_t *dk = at<int32_t>(ws, L.delta_k);
+  int32_t *fl = at<int32_t>(ws, L.flagged);  // int32[3N]; free while no assign is in flight on this ws
+  DeltaScratch ds{dk, dk + K, dk + 2 * K, dk + 3 * K, reinterpret_cast<int64_t *>(dk + 4 * K),
+                  perm, slab, fl, fl + N, at<unsigned long long>(ws, L.reseed)};
+  HME_CUDA(launch_update(X, N, d, ldx, dtype, labels, prev_labels, perm, slab, hist, offs + K, mind, K, st, ds,
+                         C_inout, counts_out, n_reseeded_out, hdr, s),
            "update: centres");
   if (objective_out)
     HME_CUDA(cudaMemcpyAsync(objective_out, &hdr->objective, sizeof(double), cudaMemcpyDeviceToDevice, s),

@@ -44,7 +44,9 @@ struct AssignParams {
   uint32_t b_bytes;    // one B operand per stage (BN rows x 128 bytes)
   uint32_t stage_bytes;
   uint32_t tmem_cols;  // allocated TMEM columns
-  uint32_t acc_stride; // columns between the two accumulators
+  uint32_t acc_stride; // columns between accumulator buffers
+  int nbuf;            // accumulator buffers (2: epilogue overlaps the next MMAs)
+  uint32_t a_res_bytes;  // resident A region (0 unless the A rows stay resident)
   const float *xn;
   const float *cn;     // Kp entries, +inf past K
   int32_t *labels;
@@ -57,7 +59,6 @@ struct AssignParams {
   float err_split;  // 2^-14 for split fp32 operands, else 0
 };
 
-constexpr int kThreads = 192;
 constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4;
 
 // One group of 16 accumulator columns of one row: v_j = ||c_j||^2 - 2 x.c_j.
@@ -125,12 +126,20 @@ __device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float 
   i1 = (b1 < before) ? k0 + jl : i1;
 }
 
-template <int NPROD, bool LEAN>
-__global__ void __launch_bounds__(kThreads, 1)
+// The fused assign kernel.
+//   NPROD  1: bf16 operands; 4: fp32 features as bf16 hi/lo pairs (four products)
+//   LEAN   several N-chunks: lean epilogue scan (best, index, runner-up)
+//   MT     row tiles of 128 per CTA sharing each B (centre) stage: 1 or 2
+//   ARES   the CTA's A rows (all k-blocks) stay resident in shared memory for
+//          all N-chunks; only B streams through the ring
+// Threads: warp 0 TMA, warp 1 MMA, 4*MT epilogue warps.
+template <int NPROD, bool LEAN, int MT, bool ARES>
+__global__ void __launch_bounds__(64 + 128 * MT, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
                   const AssignParams p) {
   constexpr int NOPS = (NPROD == 4) ? 2 : 1;  // operands per side (hi[, lo])
+  constexpr int BMT = kBM * MT;               // rows per CTA tile
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms.
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -138,17 +147,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t *smem = smem_raw + (base - raw_addr);
 
   const int S = p.stages;
-  uint8_t *ctrl = smem + (size_t)S * p.stage_bytes;
+  const uint32_t ares = base;                         // resident A region (ARES)
+  const uint32_t ring = base + p.a_res_bytes;         // stage ring
+  uint8_t *ctrl = smem + p.a_res_bytes + (size_t)S * p.stage_bytes;
   uint64_t *full = reinterpret_cast<uint64_t *>(ctrl);
   uint64_t *empty = full + S;
   uint64_t *tfull = empty + S;
   uint64_t *tempty = tfull + 2;
   uint64_t *drain = tempty + 2;
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+  uint64_t *a_full = drain + 1;
+  uint64_t *a_empty = a_full + 1;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(a_empty + 1);
   float *cnbuf = reinterpret_cast<float *>(ctrl + 512);  // one 256-float buffer per epilogue warp
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int nbuf = p.nbuf;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -157,9 +171,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&tempty[a]), 4 * MT);
     }
     mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(a_full), 1);
+    mbar_init(smem_u32(a_empty), 1);
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -179,15 +195,39 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
+  // shared-memory addresses of the operands of stage s / k-block kb
+  auto a_addr = [&](int op, int mt, int kb, uint32_t st) -> uint32_t {
+    if (ARES) return ares + (uint32_t)(((mt * p.num_kb + kb) * NOPS + op)) * p.a_bytes;
+    return st + (uint32_t)(op * MT + mt) * p.a_bytes;
+  };
+  auto b_addr = [&](int op, uint32_t st) -> uint32_t {
+    return st + (ARES ? 0u : (uint32_t)(NOPS * MT) * p.a_bytes) + (uint32_t)op * p.b_bytes;
+  };
+
   if (warp == 0) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       const uint64_t pol_a = l2_policy_evict_first();
       const uint64_t pol_b = l2_policy_evict_last();
-      uint32_t it = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
-        const int32_t row0 = tile * kBM;
+      uint32_t it = 0, tile_it = 0;
+      bool ok = true, a_pending = false;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+        const int32_t row0 = tile * BMT;
+        if (ARES) {
+          // the previous tile's MMAs must be done with the resident A rows
+          if (!mbar_wait_bounded(smem_u32(a_empty), (tile_it & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereProducer)) {
+            ok = false;
+            break;
+          }
+          const uint32_t ab = smem_u32(a_full);
+          mbar_arrive_expect_tx(ab, p.a_res_bytes);
+          for (int mt = 0; mt < MT; ++mt)
+            for (int kb = 0; kb < p.num_kb; ++kb) {
+              tma_load_2d(a_addr(0, mt, kb, 0), &tmA0, ab, kb * kBK, row0 + mt * kBM, pol_a);
+              if (NPROD == 4) tma_load_2d(a_addr(1, mt, kb, 0), &tmA1, ab, kb * kBK, row0 + mt * kBM, pol_a);
+            }
+          a_pending = true;
+        }
         for (int ch = 0; ch < p.nchunks && ok; ++ch) {
           for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
             const int s = it % S;
@@ -198,34 +238,45 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const uint32_t fb = smem_u32(&full[s]);
             mbar_arrive_expect_tx(fb, p.stage_bytes);
-            const uint32_t st = base + (uint32_t)s * p.stage_bytes;
+            const uint32_t st = ring + (uint32_t)s * p.stage_bytes;
             const int32_t kx = kb * kBK;
-            tma_load_2d(st, &tmA0, fb, kx, row0, pol_a);
-            if (NPROD == 4) tma_load_2d(st + p.a_bytes, &tmA1, fb, kx, row0, pol_a);
-            const uint32_t sb = st + NOPS * p.a_bytes;
-            tma_load_2d(sb, &tmB0, fb, kx, ch * p.BN, pol_b);
-            if (NPROD == 4) tma_load_2d(sb + p.b_bytes, &tmB1, fb, kx, ch * p.BN, pol_b);
+            if (!ARES) {
+              for (int mt = 0; mt < MT; ++mt) {
+                tma_load_2d(a_addr(0, mt, kb, st), &tmA0, fb, kx, row0 + mt * kBM, pol_a);
+                if (NPROD == 4) tma_load_2d(a_addr(1, mt, kb, st), &tmA1, fb, kx, row0 + mt * kBM, pol_a);
+              }
+            }
+            tma_load_2d(b_addr(0, st), &tmB0, fb, kx, ch * p.BN, pol_b);
+            if (NPROD == 4) tma_load_2d(b_addr(1, st), &tmB1, fb, kx, ch * p.BN, pol_b);
           }
         }
       }
-      // Drain: every stage issued must land before the CTA may end.
+      // Drain: every copy issued must land before the CTA may end.
       if (!ok) {
         const uint32_t issued = it;
-        for (uint32_t j = (issued > (uint32_t)S ? issued - S : 0); j < issued; ++j) {
+        for (uint32_t j = (issued > (uint32_t)S ? issued - S : 0); j < issued; ++j)
           mbar_wait_bounded(smem_u32(&full[j % S]), (j / S) & 1u, 200000000ull, p.hdr, kWhereProducer);
-        }
+        if (ARES && a_pending && tile_it > 0)
+          mbar_wait_bounded(smem_u32(a_full), (tile_it - 1) & 1u, 200000000ull, p.hdr, kWhereProducer);
       }
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(kBM, (uint32_t)p.BN);
-      uint32_t it = 0, acc_it = 0;
+      uint32_t it = 0, acc_it = 0, tile_it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+        if (ARES) {
+          if (!mbar_wait_bounded(smem_u32(a_full), tile_it & 1u, p.limit_ns, p.hdr, kWhereMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+        }
         for (int ch = 0; ch < p.nchunks && ok; ++ch, ++acc_it) {
-          const uint32_t a = acc_it & 1u;
-          const uint32_t aph = (acc_it >> 1) & 1u;
+          const uint32_t a = acc_it % (uint32_t)nbuf;
+          const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
           if (!mbar_wait_bounded(smem_u32(&tempty[a]), aph ^ 1u, p.limit_ns, p.hdr, kWhereMmaAcc)) {
             ok = false;
             break;
@@ -240,25 +291,29 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t st = base + (uint32_t)s * p.stage_bytes;
-            const uint32_t sb = st + NOPS * p.a_bytes;
+            const uint32_t st = ring + (uint32_t)s * p.stage_bytes;
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k) {
-              const uint64_t ad0 = smem_desc_sw128(st + k * 32);
-              const uint64_t bd0 = smem_desc_sw128(sb + k * 32);
-              tc_mma_bf16(dt, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-              if (NPROD == 4) {
-                const uint64_t ad1 = smem_desc_sw128(st + p.a_bytes + k * 32);
-                const uint64_t bd1 = smem_desc_sw128(sb + p.b_bytes + k * 32);
-                tc_mma_bf16(dt, ad0, bd1, idesc, 1u);  // xh . cl
-                tc_mma_bf16(dt, ad1, bd0, idesc, 1u);  // xl . ch
-                tc_mma_bf16(dt, ad1, bd1, idesc, 1u);  // xl . cl
+              const uint64_t bd0 = smem_desc_sw128(b_addr(0, st) + k * 32);
+              const uint64_t bd1 = NPROD == 4 ? smem_desc_sw128(b_addr(1, st) + k * 32) : 0;
+#pragma unroll
+              for (int mt = 0; mt < MT; ++mt) {
+                const uint32_t dtm = dt + (uint32_t)(mt * p.BN);
+                const uint64_t ad0 = smem_desc_sw128(a_addr(0, mt, kb, st) + k * 32);
+                tc_mma_bf16(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                if (NPROD == 4) {
+                  const uint64_t ad1 = smem_desc_sw128(a_addr(1, mt, kb, st) + k * 32);
+                  tc_mma_bf16(dtm, ad0, bd1, idesc, 1u);  // xh . cl
+                  tc_mma_bf16(dtm, ad1, bd0, idesc, 1u);  // xl . ch
+                  tc_mma_bf16(dtm, ad1, bd1, idesc, 1u);  // xl . cl
+                }
               }
             }
             tc_commit(smem_u32(&empty[s]));  // frees the stage once these MMAs finish
           }
-          if (ok) tc_commit(smem_u32(&tfull[a]));  // accumulator a is complete
+          if (ok) tc_commit(smem_u32(&tfull[a]));  // accumulators of buffer a are complete
         }
+        if (ARES && ok) tc_commit(smem_u32(a_empty));  // the resident A rows may be replaced
       }
       if (!ok) {
         // Let the MMAs already issued finish before TMEM is released.
@@ -268,11 +323,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- epilogue: argmin over the accumulator rows ----------------
+    const int e = warp - 2;          // 0 .. 4*MT-1
+    const int mt = e >> 2;           // which row tile (accumulator) of the CTA tile
     const int q = warp & 3;          // TMEM lane quarter this warp may access
-    float *cb = cnbuf + (warp - 2) * kMaxBN;  // this warp's copy of ||c||^2 for the chunk
+    float *cb = cnbuf + e * kMaxBN;  // this warp's copy of ||c||^2 for the chunk
     const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
     const float sqrt_cn_max = sqrtf(cn_max);
-    const int row_in_tile = q * 32 + lane;
+    const int row_in_tile = mt * kBM + q * 32 + lane;
     uint32_t acc_it = 0;
     bool ok = true;
     double obj = 0.0;
@@ -285,14 +342,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + ch * p.BN + t);
         __syncwarp();
-        const uint32_t a = acc_it & 1u;
-        const uint32_t aph = (acc_it >> 1) & 1u;
+        const uint32_t a = acc_it % (uint32_t)nbuf;
+        const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
         if (!mbar_wait_bounded(smem_u32(&tfull[a]), aph, p.limit_ns, p.hdr, kWhereEpi)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
+        const uint32_t taddr =
+            tmem_base + a * p.acc_stride + (uint32_t)(mt * p.BN) + ((uint32_t)(q * 32) << 16);
         const int kbase = ch * p.BN;
         // 16 columns per step; the next step's tcgen05.ld is in flight while this
         // step's distances are formed.
@@ -327,7 +385,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         best1 = take_b ? lb1 : best1;
         idx1 = take_b ? li1 : idx1;
       }
-      const int64_t row = (int64_t)tile * kBM + row_in_tile;
+      const int64_t row = (int64_t)tile * BMT + row_in_tile;
       if (row < p.N) {
         const float xr = __ldg(p.xn + row);
         const float D1 = xr + best1;
@@ -726,21 +784,24 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.num_kb = (g.d + kBK - 1) / kBK;
   p.BN = g.BN;
   p.nchunks = g.nchunks;
-  p.num_tiles = (int)((N + kBM - 1) / kBM);
+  p.num_tiles = (int)((N + kBM * g.mt - 1) / (kBM * g.mt));
   p.a_bytes = kBM * kBK * 2;
   p.b_bytes = (uint32_t)g.BN * kBK * 2;
   const int nops = g.nprod == 4 ? 2 : 1;
-  p.stage_bytes = nops * (p.a_bytes + p.b_bytes);
-  const size_t ctrl_bytes = 512 + 4 * kMaxBN * sizeof(float);
-  const size_t budget = 227 * 1024 - 1024 - ctrl_bytes;
+  p.a_res_bytes = g.ares ? (uint32_t)(g.mt * p.num_kb * nops) * p.a_bytes : 0u;
+  p.stage_bytes = nops * ((g.ares ? 0u : (uint32_t)g.mt * p.a_bytes) + p.b_bytes);
+  const size_t ctrl_bytes = 512 + (size_t)4 * g.mt * kMaxBN * sizeof(float);
+  const size_t budget = 227 * 1024 - 1024 - ctrl_bytes - p.a_res_bytes;
   int stages = (int)(budget / p.stage_bytes);
   if (stages > 8) stages = 8;
   if (stages < 2) return fail(HME_EINTERNAL, "assign: stage of %u bytes does not fit twice", p.stage_bytes);
   p.stages = stages;
+  p.nbuf = g.nbuf;
   uint32_t stride = 32;
-  while (stride < (uint32_t)g.BN) stride <<= 1;
+  while (stride < (uint32_t)(g.mt * g.BN)) stride <<= 1;
   p.acc_stride = stride;
-  p.tmem_cols = 2 * stride;
+  p.tmem_cols = (uint32_t)g.nbuf * stride;
+  if (p.tmem_cols > 512) return fail(HME_EINTERNAL, "assign: %u TMEM columns", p.tmem_cols);
   p.xn = xn;
   p.cn = cn;
   p.labels = labels;
@@ -751,16 +812,22 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.limit_ns = wait_limit_ns();
   p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
   p.err_split = g.nprod == 4 ? 0x1p-14f : 0.0f;
-  const size_t smem = (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
+  const size_t smem = (size_t)p.a_res_bytes + (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
   int grid = num_sms();
   if (grid > p.num_tiles) grid = p.num_tiles;
   cudaError_t e;
   const bool lean = g.nchunks > 1;
-  auto kern = g.nprod == 4 ? (lean ? assign_kernel<4, true> : assign_kernel<4, false>)
-                           : (lean ? assign_kernel<1, true> : assign_kernel<1, false>);
+  using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
+  Kern kern;
+  if (g.nprod == 4)
+    kern = lean ? assign_kernel<4, true, 1, false> : assign_kernel<4, false, 1, false>;
+  else if (g.ares)
+    kern = assign_kernel<1, true, 2, true>;
+  else
+    kern = lean ? assign_kernel<1, true, 2, false> : assign_kernel<1, false, 2, false>;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
-  kern<<<grid, kThreads, smem, s>>>(mA0, mA1, mB0, mB1, p);
+  kern<<<grid, 64 + 128 * g.mt, smem, s>>>(mA0, mA1, mB0, mB1, p);
   count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");

@@ -29,7 +29,8 @@ struct Header {          // lives at ws + 0, 256 bytes
   double objective;      // fp64 objective accumulator of hme_assign
   uint32_t wait_where;   // which bounded wait expired (diagnostic)
   uint32_t cn_max_bits;  // max_k ||c_k||^2 of the prepared centres (float bits; values are >= 0)
-  uint32_t pad1[56];
+  uint32_t moved_rows;   // incremental centre update: rows that changed label (diagnostic)
+  uint32_t pad1[55];
 };
 static_assert(sizeof(Header) == 256, "header is 256 bytes");
 
@@ -49,6 +50,9 @@ struct AssignGeom {
   int nchunks;    // ceil(K / BN)
   int Kp;         // nchunks * BN
   int nprod;      // 1 (bf16 features) or 4 (fp32 features, split products)
+  int mt;         // 128-row tiles per CTA sharing each centre stage (1 or 2)
+  bool ares;      // A rows resident in shared memory across N-chunks
+  int nbuf;       // TMEM accumulator buffers (1 or 2)
 };
 
 AssignGeom assign_geom(int d, int K, int dtype);
@@ -73,7 +77,11 @@ struct Layout {
   size_t full_rows; // int32[N]: near-tie rows queued for all K centres
   size_t perm, slab;  // int32[N] each: sorted order of the labels (update)
   PartLayout part;  // partition scratch (update / route)
-  size_t sums;      // f64[K * d]
+  size_t sums;      // f64[K * d]: per-cluster sums (kept between centre updates)
+  size_t counts;    // i64[K]: per-cluster counts (kept between centre updates)
+  size_t x2sum;     // f64: sum of ||x||^2 (kept between centre updates)
+  size_t delta_k;   // int32[4K] + int64[2]: counts, cursors and totals of the incremental update
+  size_t reseed;    // u64[64 * selecting warps]: re-seed candidate keys
   size_t kpp_rows;  // int32[m]
   size_t kpp_d2;    // f64[m]
   size_t kpp_part;  // f64[blocks]
@@ -113,15 +121,35 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
 cudaError_t launch_tag_scatter(const int32_t *perm, int64_t N, const int64_t *valid_total, const int64_t *tag_off,
                                const int32_t *tags, int64_t *tag_off_out, int32_t *tags_out, int64_t *scratch,
                                int64_t nscratch, cudaStream_t s);
-cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *perm,
-                          const int32_t *sorted_labels, const int64_t *hist, const int64_t *valid_total,
-                          const float *mind, int K, double *sums, float *C, int64_t *counts_out, int32_t *n_reseeded,
+// Per-cluster state carried by the workspace from one centre update to the next.
+struct UpdateState {
+  double *sums;     // fp64[K * d]: S_k = sum of the rows with label k
+  int64_t *counts;  // int64[K]: n_k
+  double *x2sum;    // sum_i ||x_i||^2 of the rows with a valid label
+};
+// Scratch of the incremental update (regions the assign queues and the sort
+// order also use; never live at the same time).
+struct DeltaScratch {
+  int32_t *hist_add, *hist_sub;  // int32[K] each, adjacent (hist_sub = hist_add + K)
+  int32_t *cur_add, *cur_sub;    // int32[K] each
+  int64_t *totals;               // int64[2]: rows to add, rows to subtract
+  int32_t *add_rows, *add_lab, *sub_rows, *sub_lab;  // int32[N] each
+  unsigned long long *cand;      // re-seed candidates: 64 keys per selecting warp
+};
+// prev_labels == nullptr: full pass (perm / sorted_labels / hist / valid_total
+// from the partition of labels); otherwise an incremental update from the
+// state left by a call with prev_labels.
+cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *labels,
+                          const int32_t *prev_labels, const int32_t *perm, const int32_t *sorted_labels,
+                          const int64_t *hist, const int64_t *valid_total, const float *mind, int K,
+                          UpdateState st, DeltaScratch ds, float *C, int64_t *counts_out, int32_t *n_reseeded,
                           Header *hdr, cudaStream_t s);
 cudaError_t launch_kmeanspp(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, uint64_t seed,
                             int64_t m, bool subsample, float *C_out, int32_t *rows, double *d2, double *part,
                             Header *hdr, cudaStream_t s);
 cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
 int64_t kpp_candidates(int64_t N, int K, int method);
+constexpr int kMaxSms = 256;  // bound used to size the re-seed candidate region
 int64_t kpp_blocks(int64_t m);
 
 // ---------------------------------------------------------------------------

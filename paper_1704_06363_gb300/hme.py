@@ -58,7 +58,7 @@ def lib():
         L.hme_assign.restype = ctypes.c_int
         L.hme_assign.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
         L.hme_update_centroids.restype = ctypes.c_int
-        L.hme_update_centroids.argtypes = [p, i64, i32, i64, i32, p, p, i32, p, p, p, p, p, sz, p]
+        L.hme_update_centroids.argtypes = [p, i64, i32, i64, i32, p, p, p, i32, p, p, p, p, p, sz, p]
         L.hme_partition.restype = ctypes.c_int
         L.hme_partition.argtypes = [p, i64, i32, p, p, p, p, p, p, p, p, p, sz, p]
         L.hme_route.restype = ctypes.c_int
@@ -148,11 +148,13 @@ def hme_assign(X: torch.Tensor, C: torch.Tensor, labels_out: torch.Tensor, ws: t
 def hme_update_centroids(X: torch.Tensor, labels: torch.Tensor, mind: Optional[torch.Tensor], C_inout: torch.Tensor,
                          ws: torch.Tensor, counts_out: Optional[torch.Tensor] = None,
                          n_reseeded_out: Optional[torch.Tensor] = None, objective_out: Optional[torch.Tensor] = None,
-                         stream=None):
+                         prev_labels: Optional[torch.Tensor] = None, stream=None):
+    """Centre step.  prev_labels: the labels of the previous call on this ws (incremental update)."""
     N, d, ldx, dt = _features(X)
     K = C_inout.shape[0]
     w, wb = _ws(ws)
-    _check(lib().hme_update_centroids(_ptr(X), N, d, ldx, dt, _ptr(labels), _ptr(mind), K, _ptr(C_inout),
+    _check(lib().hme_update_centroids(_ptr(X), N, d, ldx, dt, _ptr(labels), _ptr(prev_labels), _ptr(mind), K,
+                                      _ptr(C_inout),
                                       _ptr(counts_out), _ptr(n_reseeded_out), _ptr(objective_out), w, wb,
                                       _stream(stream)),
            "hme_update_centroids")

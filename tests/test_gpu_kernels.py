@@ -175,6 +175,8 @@ UPDATE_CASES = [
     (5000, 2048, 64, "f32", False),
     (5000, 256, 700, "bf16", True),
     (300, 20, 500, "f32", True),  # more clusters than points: reseeds run out of rows
+    (20000, 64, 90, "f32", True),  # about 18 empty clusters: one-pass selection
+    (20000, 64, 400, "bf16", True),  # about 80 empty clusters: the general path
 ]
 
 
@@ -205,6 +207,40 @@ def test_update_parity(dev, N, d, K, dtype, holes):
     # re-seeded centres are exact copies of rows
     empty = np.nonzero(cref == 0)[0]
     assert np.array_equal(Cg.cpu().numpy()[empty], Cref[empty])
+
+
+@pytest.mark.parametrize("N,d,K,dtype,frac", [(4000, 256, 24, "f32", 0.05), (4000, 136, 24, "bf16", 0.3),
+                                              (3001, 130, 300, "f32", 0.02), (2000, 64, 40, "bf16", 1.0)])
+def test_update_incremental_matches_oracle(dev, N, d, K, dtype, frac):
+    """An update from the previous call's state, reading only rows whose label changed,
+    gives the oracle's centres, counts and objective for the new labels."""
+    X = _mixture(N, d, min(K, 30), dtype, seed=N + K + 7)
+    g = torch.Generator().manual_seed(11)
+    lab0 = torch.randint(0, K, (N,), generator=g, dtype=torch.int32)
+    lab0[lab0 == 5] = 6  # cluster 5 empty at first: re-seeded, then filled
+    lab1 = lab0.clone()
+    moved = torch.rand(N, generator=g) < frac
+    lab1[moved] = torch.randint(0, K, (int(moved.sum()),), generator=g, dtype=torch.int32)
+    lab1[lab1 == 7] = 8  # cluster 7 empties in the second call
+    mind = (torch.rand(N, generator=g) * 10).float()
+    C0 = hme_synth.random_centroids(K, d, seed=6)
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+    Xg, md = X.to(dev), mind.to(dev)
+    Cg = C0.to(dev)
+    counts = torch.empty(K, dtype=torch.int64, device=dev)
+    nres = torch.zeros(1, dtype=torch.int32, device=dev)
+    J = torch.zeros(1, dtype=torch.float64, device=dev)
+    hme.hme_update_centroids(Xg, lab0.to(dev), md, Cg, ws, counts, nres, J)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    C1 = Cg.cpu().numpy()
+    Xh = _host(X, dtype)
+    hme.hme_update_centroids(Xg, lab1.to(dev), md, Cg, ws, counts, nres, J, prev_labels=lab0.to(dev))
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    Cref, cref, nref = oracle.update(Xh, lab1.numpy(), mind.double().numpy(), C1, dtype)
+    assert np.array_equal(counts.cpu().numpy(), cref) and nres.item() == nref
+    parity.check_centres(Cg.cpu().numpy(), Cref)
+    parity.check_objective(J.item(), Xh, dtype, C1, lab1.numpy())
 
 
 PART_CASES = [(0, 4), (1, 1), (31, 7), (1000, 64), (100003, 1000), (70000, 4096), (50000, 1), (12345, 16384)]

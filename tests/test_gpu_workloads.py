@@ -50,6 +50,7 @@ class Lloyd:
         self.J = torch.zeros(1, dtype=torch.float64, device=dev)
         self.counts = torch.empty(K, dtype=torch.int64, device=dev)
         self.nres = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.prev = None  # labels of the previous centre update: later updates are incremental
         hme.hme_prepare_features(X, K, self.ws)
 
     def init(self, seed, method):
@@ -64,8 +65,10 @@ class Lloyd:
         assert hme.hme_sync_status(self.ws) == hme.HME_OK
 
     def update(self, C):
-        hme.hme_update_centroids(self.X, self.labels, self.mind, C, self.ws, self.counts, self.nres, self.J)
+        hme.hme_update_centroids(self.X, self.labels, self.mind, C, self.ws, self.counts, self.nres, self.J,
+                                 prev_labels=self.prev)
         assert hme.hme_sync_status(self.ws) == hme.HME_OK
+        self.prev = self.labels.clone()
 
 
 def _teacher_forced(w, Xh, L, C, iters):
