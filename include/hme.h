@@ -138,11 +138,13 @@ HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ld
  * The distance is ||x||^2 - 2 x.c + ||c||^2 with x.c on the tcgen05 tensor
  * cores (fp32 accumulate): for HME_BF16 features, x.bf16(c) with c rounded to
  * bf16 (round to nearest even); for HME_F32, the bf16 split x = xh + xl,
- * c = ch + cl and the four products xh.ch + xh.cl + xl.ch + xl.cl, with the
- * norms taken of the same split values.  A row whose runner-up distance is
- * within E of its best, E a bound on the error of a difference of two computed
- * distances (ceil(d/16) * nprod * 2^-22 (||x||^2 + max_k ||c_k||^2), plus
- * 2^-14 (||x|| + max ||c||) sqrt(D2) for split fp32 operands), is re-scored
+ * c = ch + cl and the three products xh.ch + xh.cl + xl.ch (nprod = 3; the
+ * dropped xl.cl is at most 2^-16 (1 + 2^-8)^2 ||x|| ||c||), with the norms
+ * taken of the same split values.  A row whose runner-up distance is within E
+ * of its best, E a bound on the error of a difference of two computed
+ * distances (ceil(d/16) * nprod * 2^-22 (||x||^2 + max_k ||c_k||^2), plus, for
+ * split fp32 operands, 2^-14 (||x|| + max ||c||) sqrt(D2) and
+ * 1.0625 * 2^-14 ||x|| max ||c||), is re-scored
  * exactly on its candidates (all K when a third centre is also within E) with
  * direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of non-negative
  * terms).  The N x K distance matrix is never written.

@@ -62,14 +62,14 @@ uint64_t wait_limit_ns() {
 // N-chunk, single-buffered in TMEM when 2 x BN needs all 512 columns.  With
 // several N-chunks and few dimensions the CTA's 256 rows stay resident in
 // shared memory (ARES) and the chunks hold 128 centres (double-buffered).  fp32
-// features (four products, 2 operands per side) keep MT = 1.
+// features (three products, 2 operands per side) keep MT = 1.
 AssignGeom assign_geom(int d, int K, int dtype) {
   AssignGeom g;
   g.d = d;
   g.K = K;
   g.dtype = dtype;
   g.ldp = (d + 7) / 8 * 8;
-  g.nprod = dtype == HME_F32 ? 4 : 1;
+  g.nprod = dtype == HME_F32 ? 3 : 1;
   const int num_kb = (d + kBK - 1) / kBK;
   int max_bn = kMaxBN;
   g.mt = 1;
@@ -83,7 +83,9 @@ AssignGeom assign_geom(int d, int K, int dtype) {
   }
   g.nchunks = (K + max_bn - 1) / max_bn;
   const int per = (K + g.nchunks - 1) / g.nchunks;
-  g.BN = (per + 15) / 16 * 16;
+  // The lean scan (several chunks) reads 32 accumulator columns per step.
+  const int gran = g.nchunks > 1 ? 32 : 16;
+  g.BN = (per + gran - 1) / gran * gran;
   g.Kp = g.BN * g.nchunks;
   g.nbuf = (g.mt * g.BN <= 256) ? 2 : 1;
   return g;

@@ -12,10 +12,14 @@
 //
 // Operands: for bf16 features, A = X (bf16) and B = bf16(C); for fp32
 // features the split x = xh + xl, c = ch + cl (all bf16, 16 significant bits
-// together) gives x_eff.c_eff = xh.ch + xh.cl + xl.ch + xl.cl (four MMAs per
-// k-step).  With ||x_eff||^2 and ||c_eff||^2 from the same split values the
-// computed distance is ||x_eff - c_eff||^2 up to fp32 accumulation, whose
-// difference from ||x - c||^2 is O(2^-16 |x - c| (|x| + |c|)) per element.
+// together) gives x_eff.c_eff = xh.ch + xh.cl + xl.ch + xl.cl.  The kernel
+// issues the first three (three MMAs per k-step): |xl| <= 2^-8 (1 + 2^-8) |x|
+// elementwise and likewise for cl, so the dropped xl.cl is at most
+// 2^-16 (1 + 2^-8)^2 ||x|| ||c|| and enters the near-tie bound as its own
+// term.  With ||x_eff||^2 and ||c_eff||^2 from the same split values the
+// computed distance is ||x_eff - c_eff||^2 + 2 xl.cl up to fp32 accumulation;
+// ||x_eff - c_eff||^2 differs from ||x - c||^2 by O(2^-16 |x - c| (|x| + |c|))
+// per element.
 //
 // Warp roles (192 threads, one CTA per SM, persistent over row tiles):
 //   warp 0      TMA producer: A and B k-blocks into an S-stage ring,
@@ -57,6 +61,7 @@ struct AssignParams {
   uint64_t limit_ns;
   float err_acc;    // ceil(d/16) * nprod * 2^-22 + 2^-20: accumulation + epilogue rounding
   float err_split;  // 2^-14 for split fp32 operands, else 0
+  float err_ll;     // 1.0625 * 2^-14 for split fp32 operands (the dropped xl.cl), else 0
 };
 
 constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4;
@@ -100,45 +105,68 @@ __device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const fl
   }
 }
 
-// Lean variant for many centres (several N-chunks): per column
-// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
-// min(best, v), and the best's column -- six instructions, no branches.  jl is
-// the column of the best within this group; i1 moves only if the group
-// improved the best, so ties keep the lowest index.
-__device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float *cn16, int k0, float &b1, float &b2,
-                                           int &i1) {
-  const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
-  const float before = b1;
-  int jl = 0;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const float4 cc = c4[q];
-    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int j = 4 * q + e;
-      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[e]);
-      b2 = fminf(b2, fmaxf(b1, v));
-      jl = (v < b1) ? j : jl;
-      b1 = fminf(b1, v);
-    }
-  }
-  i1 = (b1 < before) ? k0 + jl : i1;
-}
-
 // The fused assign kernel.
-//   NPROD  1: bf16 operands; 4: fp32 features as bf16 hi/lo pairs (four products)
+//   NPROD  1: bf16 operands; 3: fp32 features as bf16 hi/lo pairs (three products)
 //   LEAN   several N-chunks: lean epilogue scan (best, index, runner-up)
 //   MT     row tiles of 128 per CTA sharing each B (centre) stage: 1 or 2
 //   ARES   the CTA's A rows (all k-blocks) stay resident in shared memory for
 //          all N-chunks; only B streams through the ring
 // Threads: warp 0 TMA, warp 1 MMA, 4*MT epilogue warps.
+// Lean scan for many centres (several N-chunks): per column
+// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
+// min(best, v), and the best's column moves only on a strict improvement, so
+// ties keep the lowest index.  Four independent states per thread (column j of
+// a 32-column group feeds state j % 4) let four dependency chains of
+// min/select run side by side; they are merged once per row tile.
+struct Lean4 {
+  float b1[4], b2[4];
+  int i1[4];
+  __device__ __forceinline__ void reset() {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      b1[u] = INFINITY;
+      b2[u] = INFINITY;
+      i1[u] = 0;
+    }
+  }
+  // Merge into (best, runner-up, index): lowest value, then lowest index.
+  __device__ __forceinline__ void merge(float &best, float &second, int &idx) const {
+    best = b1[0];
+    idx = i1[0];
+    second = b2[0];
+#pragma unroll
+    for (int u = 1; u < 4; ++u) {
+      const bool take = b1[u] < best || (b1[u] == best && i1[u] < idx);
+      second = fminf(fmaxf(best, b1[u]), fminf(second, b2[u]));
+      best = take ? b1[u] : best;
+      idx = take ? i1[u] : idx;
+    }
+  }
+};
+
+__device__ __forceinline__ void lean_group32(const uint32_t (&r)[32], const float *cn32, int k0, Lean4 &st) {
+  const float4 *c4 = reinterpret_cast<const float4 *>(cn32);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 cc = c4[q];
+    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int j = 4 * q + u;
+      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[u]);
+      st.b2[u] = fminf(st.b2[u], fmaxf(st.b1[u], v));
+      st.i1[u] = (v < st.b1[u]) ? k0 + j : st.i1[u];
+      st.b1[u] = fminf(st.b1[u], v);
+    }
+  }
+}
+
 template <int NPROD, bool LEAN, int MT, bool ARES>
 __global__ void __launch_bounds__(64 + 128 * MT, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
                   const AssignParams p) {
-  constexpr int NOPS = (NPROD == 4) ? 2 : 1;  // operands per side (hi[, lo])
+  constexpr int NOPS = (NPROD == 3) ? 2 : 1;  // operands per side (hi[, lo])
   constexpr int BMT = kBM * MT;               // rows per CTA tile
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms.
@@ -181,7 +209,7 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmA0);
     prefetch_tensormap(&tmB0);
-    if (NPROD == 4) {
+    if (NPROD == 3) {
       prefetch_tensormap(&tmA1);
       prefetch_tensormap(&tmB1);
     }
@@ -224,7 +252,7 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
           for (int mt = 0; mt < MT; ++mt)
             for (int kb = 0; kb < p.num_kb; ++kb) {
               tma_load_2d(a_addr(0, mt, kb, 0), &tmA0, ab, kb * kBK, row0 + mt * kBM, pol_a);
-              if (NPROD == 4) tma_load_2d(a_addr(1, mt, kb, 0), &tmA1, ab, kb * kBK, row0 + mt * kBM, pol_a);
+              if (NPROD == 3) tma_load_2d(a_addr(1, mt, kb, 0), &tmA1, ab, kb * kBK, row0 + mt * kBM, pol_a);
             }
           a_pending = true;
         }
@@ -243,11 +271,11 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
             if (!ARES) {
               for (int mt = 0; mt < MT; ++mt) {
                 tma_load_2d(a_addr(0, mt, kb, st), &tmA0, fb, kx, row0 + mt * kBM, pol_a);
-                if (NPROD == 4) tma_load_2d(a_addr(1, mt, kb, st), &tmA1, fb, kx, row0 + mt * kBM, pol_a);
+                if (NPROD == 3) tma_load_2d(a_addr(1, mt, kb, st), &tmA1, fb, kx, row0 + mt * kBM, pol_a);
               }
             }
             tma_load_2d(b_addr(0, st), &tmB0, fb, kx, ch * p.BN, pol_b);
-            if (NPROD == 4) tma_load_2d(b_addr(1, st), &tmB1, fb, kx, ch * p.BN, pol_b);
+            if (NPROD == 3) tma_load_2d(b_addr(1, st), &tmB1, fb, kx, ch * p.BN, pol_b);
           }
         }
       }
@@ -295,17 +323,16 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k) {
               const uint64_t bd0 = smem_desc_sw128(b_addr(0, st) + k * 32);
-              const uint64_t bd1 = NPROD == 4 ? smem_desc_sw128(b_addr(1, st) + k * 32) : 0;
+              const uint64_t bd1 = NPROD == 3 ? smem_desc_sw128(b_addr(1, st) + k * 32) : 0;
 #pragma unroll
               for (int mt = 0; mt < MT; ++mt) {
                 const uint32_t dtm = dt + (uint32_t)(mt * p.BN);
                 const uint64_t ad0 = smem_desc_sw128(a_addr(0, mt, kb, st) + k * 32);
                 tc_mma_bf16(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
-                if (NPROD == 4) {
+                if (NPROD == 3) {
                   const uint64_t ad1 = smem_desc_sw128(a_addr(1, mt, kb, st) + k * 32);
                   tc_mma_bf16(dtm, ad0, bd1, idesc, 1u);  // xh . cl
                   tc_mma_bf16(dtm, ad1, bd0, idesc, 1u);  // xl . ch
-                  tc_mma_bf16(dtm, ad1, bd1, idesc, 1u);  // xl . cl
                 }
               }
             }
@@ -333,15 +360,36 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
     uint32_t acc_it = 0;
     bool ok = true;
     double obj = 0.0;
+    // ||c||^2 of the next chunk is fetched into registers while the current
+    // chunk is scanned; with a single chunk the buffer is filled once.
+    constexpr int kCnRegs = kMaxBN / 32;
+    float cn_next[kCnRegs];
+    auto fetch_cn = [&](int ch) {
+#pragma unroll
+      for (int r = 0; r < kCnRegs; ++r) {
+        const int t = lane + 32 * r;
+        cn_next[r] = (t < p.BN) ? __ldg(p.cn + ch * p.BN + t) : 0.0f;
+      }
+    };
+    fetch_cn(0);
+    bool cb_filled = false;
     for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
       int idx1 = 0, idx2 = 0;
-      float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
-      int li1 = 0;
+      Lean4 lst;  // lean scan states
+      lst.reset();
+      const int64_t row = (int64_t)tile * BMT + row_in_tile;
+      const float xr = row < p.N ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
-        __syncwarp();
-        for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + ch * p.BN + t);
-        __syncwarp();
+        if (p.nchunks > 1 || !cb_filled) {
+          __syncwarp();
+#pragma unroll
+          for (int r = 0; r < kCnRegs; ++r)
+            if (lane + 32 * r < p.BN) cb[lane + 32 * r] = cn_next[r];
+          __syncwarp();
+          cb_filled = true;
+          if (p.nchunks > 1) fetch_cn(ch + 1 < p.nchunks ? ch + 1 : 0);
+        }
         const uint32_t a = acc_it % (uint32_t)nbuf;
         const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
         if (!mbar_wait_bounded(smem_u32(&tfull[a]), aph, p.limit_ns, p.hdr, kWhereEpi)) {
@@ -352,26 +400,38 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         const uint32_t taddr =
             tmem_base + a * p.acc_stride + (uint32_t)(mt * p.BN) + ((uint32_t)(q * 32) << 16);
         const int kbase = ch * p.BN;
-        // 16 columns per step; the next step's tcgen05.ld is in flight while this
-        // step's distances are formed.
-        uint32_t ra[16], rb[16];
-        tmem_ld16(taddr, ra);
-        tmem_ld_wait(ra);
-        for (int c = 0; c < p.BN; c += 32) {
-          const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
-          if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
-          if (LEAN)
-            lean_group(ra, cb + c, kbase + c, best1, best2, idx1);
-          else
+        if (LEAN) {
+          // 32 columns per step, the next 32 in flight; four chains per thread.
+          uint32_t ra[32], rb[32];
+          tmem_ld32(taddr, ra);
+          tmem_ld_wait(ra);
+          for (int c = 0; c < p.BN; c += 64) {
+            const bool more1 = c + 32 < p.BN, more2 = c + 64 < p.BN;
+            if (more1) tmem_ld32(taddr + (uint32_t)(c + 32), rb);
+            lean_group32(ra, cb + c, kbase + c, lst);
+            if (more1) {
+              tmem_ld_wait(rb);
+              if (more2) tmem_ld32(taddr + (uint32_t)(c + 64), ra);
+              lean_group32(rb, cb + c + 32, kbase + c + 32, lst);
+              if (more2) tmem_ld_wait(ra);
+            }
+          }
+        } else {
+          // 16 columns per step; the next step's tcgen05.ld is in flight while this
+          // step's distances are formed.
+          uint32_t ra[16], rb[16];
+          tmem_ld16(taddr, ra);
+          tmem_ld_wait(ra);
+          for (int c = 0; c < p.BN; c += 32) {
+            const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+            if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
             epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
-          if (more1) {
-            tmem_ld_wait(rb);
-            if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
-            if (LEAN)
-              lean_group(rb, cb + c + 16, kbase + c + 16, lb1, lb2, li1);
-            else
+            if (more1) {
+              tmem_ld_wait(rb);
+              if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
               epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
-            if (more2) tmem_ld_wait(ra);
+              if (more2) tmem_ld_wait(ra);
+            }
           }
         }
         tc_fence_before();
@@ -379,15 +439,8 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
       }
       if (!ok) break;
-      if (LEAN) {  // merge the two lean states: lowest value, then lowest index
-        const bool take_b = lb1 < best1 || (lb1 == best1 && li1 < idx1);
-        best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
-        best1 = take_b ? lb1 : best1;
-        idx1 = take_b ? li1 : idx1;
-      }
-      const int64_t row = (int64_t)tile * BMT + row_in_tile;
+      if (LEAN) lst.merge(best1, best2, idx1);
       if (row < p.N) {
-        const float xr = __ldg(p.xn + row);
         const float D1 = xr + best1;
         const float D2 = xr + best2;
         const float D3 = xr + best3;
@@ -399,11 +452,14 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         // two computed distances: each fp32 accumulation step of x.c errs by at
         // most one ulp of the accumulator (|x.c| <= (||x||^2 + ||c||^2) / 2),
         // the split operands of fp32 features by 2^-16 per element, and the
-        // epilogue adds a few roundings.  Such rows are queued for an exact
+        // epilogue adds a few roundings; the dropped xl.cl moves each distance by
+        // at most 2^-15 (1 + 2^-8)^2 ||x|| ||c||.  Such rows are queued for an exact
         // comparison: of the two candidates, or of all K when a third centre is
         // also within E (or, in the lean scan, whenever the runner-up is).
+        const float sqrt_xr = sqrtf(xr);
         const float E = p.err_acc * (xr + cn_max) +
-                        p.err_split * (sqrtf(xr) + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f));
+                        p.err_split * (sqrt_xr + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f)) +
+                        p.err_ll * sqrt_xr * sqrt_cn_max;
         const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
         if (near2) {
           const bool near3 = LEAN || ((best3 < INFINITY) && ((D3 - D1) <= E));
@@ -771,7 +827,7 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   if ((rc = make_map(&mA0, Xa, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
   if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
     return rc;
-  if (g.nprod == 4) {
+  if (g.nprod == 3) {
     if ((rc = make_map(&mA1, Xb, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
     if ((rc = make_map(&mB1, clo, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
       return rc;
@@ -787,7 +843,7 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.num_tiles = (int)((N + kBM * g.mt - 1) / (kBM * g.mt));
   p.a_bytes = kBM * kBK * 2;
   p.b_bytes = (uint32_t)g.BN * kBK * 2;
-  const int nops = g.nprod == 4 ? 2 : 1;
+  const int nops = g.nprod == 3 ? 2 : 1;
   p.a_res_bytes = g.ares ? (uint32_t)(g.mt * p.num_kb * nops) * p.a_bytes : 0u;
   p.stage_bytes = nops * ((g.ares ? 0u : (uint32_t)g.mt * p.a_bytes) + p.b_bytes);
   const size_t ctrl_bytes = 512 + (size_t)4 * g.mt * kMaxBN * sizeof(float);
@@ -811,16 +867,18 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.full_rows = full_rows;
   p.limit_ns = wait_limit_ns();
   p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
-  p.err_split = g.nprod == 4 ? 0x1p-14f : 0.0f;
+  p.err_split = g.nprod == 3 ? 0x1p-14f : 0.0f;
+  p.err_ll = g.nprod == 3 ? 0x1.1p-14f : 0.0f;
   const size_t smem = (size_t)p.a_res_bytes + (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
   int grid = num_sms();
   if (grid > p.num_tiles) grid = p.num_tiles;
   cudaError_t e;
   const bool lean = g.nchunks > 1;
+  if (lean && g.BN % 32 != 0) return fail(HME_EINTERNAL, "assign: lean scan needs BN %% 32 == 0 (BN = %d)", g.BN);
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
-  if (g.nprod == 4)
-    kern = lean ? assign_kernel<4, true, 1, false> : assign_kernel<4, false, 1, false>;
+  if (g.nprod == 3)
+    kern = lean ? assign_kernel<3, true, 1, false> : assign_kernel<3, false, 1, false>;
   else if (g.ares)
     kern = assign_kernel<1, true, 2, true>;
   else

@@ -8,7 +8,9 @@ The oracle (fp64, direct sums) is the reference; the bars are:
     ceil(d/16) * nprod * 2^-23 (||x||^2 + ||c||^2)  [one ulp of the fp32
     accumulator per accumulation step, the observed accumulation rounds
     towards zero]  + 2^-15 (||x|| + ||c||) ||x - c||  [fp32 features: the
-    16-bit split, |x - x_eff| <= 2^-16 |x| per element]  + 1e-5 D; the sum of
+    16-bit split, |x - x_eff| <= 2^-16 |x| per element]  + 2^-14 ||x|| ||c||
+    [fp32 features: the product xl.cl of the split is not formed,
+    2 |xl.cl| <= 2^-15 (1 + 2^-8)^2 ||x|| ||c||]  + 1e-5 D; the sum of
     those distances (hme_assign's objective estimate) within the sum of the
     per-row bounds + 1e-5 J;
   - objective of hme_update_centroids (direct differences): within 1e-5
@@ -44,12 +46,13 @@ def features_f64(Xh: np.ndarray, dtype: str) -> np.ndarray:
 def distance_bound(Xd, Cd, labels, D, dtype):
     """Per-row bound on |D_gpu - D| for hme_assign's distances (see the module docstring)."""
     d = Xd.shape[1]
-    nprod = 4 if dtype == "f32" else 1
+    nprod = 3 if dtype == "f32" else 1
     xn = (Xd ** 2).sum(1)
     cn = (Cd ** 2).sum(1)[labels]
     b = np.ceil(d / 16) * nprod * 2.0 ** -23 * (xn + cn) + 1e-5 * D
     if dtype == "f32":
         b += 2.0 ** -15 * (np.sqrt(xn) + np.sqrt(cn)) * np.sqrt(np.maximum(D, 0))
+        b += 2.0 ** -14 * np.sqrt(xn) * np.sqrt(cn)
     return b
 
 
