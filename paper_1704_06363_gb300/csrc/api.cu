@@ -83,9 +83,7 @@ AssignGeom assign_geom(int d, int K, int dtype) {
   }
   g.nchunks = (K + max_bn - 1) / max_bn;
   const int per = (K + g.nchunks - 1) / g.nchunks;
-  // The lean scan (several chunks) reads 32 accumulator columns per step.
-  const int gran = g.nchunks > 1 ? 32 : 16;
-  g.BN = (per + gran - 1) / gran * gran;
+  g.BN = (per + 15) / 16 * 16;
   g.Kp = g.BN * g.nchunks;
   g.nbuf = (g.mt * g.BN <= 256) ? 2 : 1;
   return g;

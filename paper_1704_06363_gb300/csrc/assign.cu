@@ -105,6 +105,32 @@ __device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const fl
   }
 }
 
+// Lean variant for many centres (several N-chunks): per column
+// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
+// min(best, v), and the best's column -- six instructions, no branches.  jl is
+// the column of the best within this group; i1 moves only if the group
+// improved the best, so ties keep the lowest index.
+__device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float *cn16, int k0, float &b1, float &b2,
+                                           int &i1) {
+  const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
+  const float before = b1;
+  int jl = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 cc = c4[q];
+    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = 4 * q + e;
+      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[e]);
+      b2 = fminf(b2, fmaxf(b1, v));
+      jl = (v < b1) ? j : jl;
+      b1 = fminf(b1, v);
+    }
+  }
+  i1 = (b1 < before) ? k0 + jl : i1;
+}
+
 // The fused assign kernel.
 //   NPROD  1: bf16 operands; 3: fp32 features as bf16 hi/lo pairs (three products)
 //   LEAN   several N-chunks: lean epilogue scan (best, index, runner-up)
@@ -112,55 +138,6 @@ __device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const fl
 //   ARES   the CTA's A rows (all k-blocks) stay resident in shared memory for
 //          all N-chunks; only B streams through the ring
 // Threads: warp 0 TMA, warp 1 MMA, 4*MT epilogue warps.
-// Lean scan for many centres (several N-chunks): per column
-// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
-// min(best, v), and the best's column moves only on a strict improvement, so
-// ties keep the lowest index.  Four independent states per thread (column j of
-// a 32-column group feeds state j % 4) let four dependency chains of
-// min/select run side by side; they are merged once per row tile.
-struct Lean4 {
-  float b1[4], b2[4];
-  int i1[4];
-  __device__ __forceinline__ void reset() {
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      b1[u] = INFINITY;
-      b2[u] = INFINITY;
-      i1[u] = 0;
-    }
-  }
-  // Merge into (best, runner-up, index): lowest value, then lowest index.
-  __device__ __forceinline__ void merge(float &best, float &second, int &idx) const {
-    best = b1[0];
-    idx = i1[0];
-    second = b2[0];
-#pragma unroll
-    for (int u = 1; u < 4; ++u) {
-      const bool take = b1[u] < best || (b1[u] == best && i1[u] < idx);
-      second = fminf(fmaxf(best, b1[u]), fminf(second, b2[u]));
-      best = take ? b1[u] : best;
-      idx = take ? i1[u] : idx;
-    }
-  }
-};
-
-__device__ __forceinline__ void lean_group32(const uint32_t (&r)[32], const float *cn32, int k0, Lean4 &st) {
-  const float4 *c4 = reinterpret_cast<const float4 *>(cn32);
-#pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    const float4 cc = c4[q];
-    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int j = 4 * q + u;
-      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[u]);
-      st.b2[u] = fminf(st.b2[u], fmaxf(st.b1[u], v));
-      st.i1[u] = (v < st.b1[u]) ? k0 + j : st.i1[u];
-      st.b1[u] = fminf(st.b1[u], v);
-    }
-  }
-}
-
 template <int NPROD, bool LEAN, int MT, bool ARES>
 __global__ void __launch_bounds__(64 + 128 * MT, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
@@ -376,8 +353,8 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
     for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
       int idx1 = 0, idx2 = 0;
-      Lean4 lst;  // lean scan states
-      lst.reset();
+      float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
+      int li1 = 0;
       const int64_t row = (int64_t)tile * BMT + row_in_tile;
       const float xr = row < p.N ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
@@ -400,38 +377,26 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         const uint32_t taddr =
             tmem_base + a * p.acc_stride + (uint32_t)(mt * p.BN) + ((uint32_t)(q * 32) << 16);
         const int kbase = ch * p.BN;
-        if (LEAN) {
-          // 32 columns per step, the next 32 in flight; four chains per thread.
-          uint32_t ra[32], rb[32];
-          tmem_ld32(taddr, ra);
-          tmem_ld_wait(ra);
-          for (int c = 0; c < p.BN; c += 64) {
-            const bool more1 = c + 32 < p.BN, more2 = c + 64 < p.BN;
-            if (more1) tmem_ld32(taddr + (uint32_t)(c + 32), rb);
-            lean_group32(ra, cb + c, kbase + c, lst);
-            if (more1) {
-              tmem_ld_wait(rb);
-              if (more2) tmem_ld32(taddr + (uint32_t)(c + 64), ra);
-              lean_group32(rb, cb + c + 32, kbase + c + 32, lst);
-              if (more2) tmem_ld_wait(ra);
-            }
-          }
-        } else {
-          // 16 columns per step; the next step's tcgen05.ld is in flight while this
-          // step's distances are formed.
-          uint32_t ra[16], rb[16];
-          tmem_ld16(taddr, ra);
-          tmem_ld_wait(ra);
-          for (int c = 0; c < p.BN; c += 32) {
-            const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
-            if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
+        // 16 columns per step; the next step's tcgen05.ld is in flight while this
+        // step's distances are formed.
+        uint32_t ra[16], rb[16];
+        tmem_ld16(taddr, ra);
+        tmem_ld_wait(ra);
+        for (int c = 0; c < p.BN; c += 32) {
+          const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+          if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
+          if (LEAN)
+            lean_group(ra, cb + c, kbase + c, best1, best2, idx1);
+          else
             epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
-            if (more1) {
-              tmem_ld_wait(rb);
-              if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
+          if (more1) {
+            tmem_ld_wait(rb);
+            if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
+            if (LEAN)
+              lean_group(rb, cb + c + 16, kbase + c + 16, lb1, lb2, li1);
+            else
               epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
-              if (more2) tmem_ld_wait(ra);
-            }
+            if (more2) tmem_ld_wait(ra);
           }
         }
         tc_fence_before();
@@ -439,7 +404,12 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
       }
       if (!ok) break;
-      if (LEAN) lst.merge(best1, best2, idx1);
+      if (LEAN) {  // merge the two lean states: lowest value, then lowest index
+        const bool take_b = lb1 < best1 || (lb1 == best1 && li1 < idx1);
+        best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
+        best1 = take_b ? lb1 : best1;
+        idx1 = take_b ? li1 : idx1;
+      }
       if (row < p.N) {
         const float D1 = xr + best1;
         const float D2 = xr + best2;
@@ -596,7 +566,10 @@ __global__ void __launch_bounds__(256) rescore_pair_kernel(const void *__restric
 // per queued row; the row is cached in shared memory and the 8 warps split the
 // centres, each lane summing (x_j - c_j)^2 over its strided elements in fp32
 // (16-byte loads of c), then across the warp and across the warps; ties to the
-// lowest index.  Latency is about K/8 passes over one centre row.
+// lowest index.  Each warp streams kRowKB centre rows at a time, so the
+// latency is about K / (8 kRowKB) passes over one centre row.
+constexpr int kRowKB = 4;
+
 template <int DT, int VW>
 __global__ void __launch_bounds__(256) rescore_row_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
                                                           const float *__restrict__ C, int K, int32_t *labels,
@@ -621,22 +594,32 @@ __global__ void __launch_bounds__(256) rescore_row_kernel(const void *__restrict
     __syncthreads();
     float bv = INFINITY;
     int bk = 0x7fffffff;
-    for (int k = warp; k < K; k += 8) {
-      float sacc = 0.0f;
-#pragma unroll 4
-      for (int j = lane * VW; j < d; j += 32 * VW) {
-        float c[VW];
-        load_c<DT, VW>(C, (int64_t)k * d + j, c);
+    // each warp takes kRowKB centres at a time (their loads in flight together);
+    // k ascends within a warp
+    for (int k0 = warp * kRowKB; k0 < K; k0 += 8 * kRowKB) {
+      float sacc[kRowKB];
 #pragma unroll
-        for (int e = 0; e < VW; ++e) {
-          const float t = xrow[j + e] - c[e];
-          sacc = fmaf(t, t, sacc);
+      for (int b = 0; b < kRowKB; ++b) sacc[b] = 0.0f;
+#pragma unroll 2
+      for (int j = lane * VW; j < d; j += 32 * VW) {
+#pragma unroll
+        for (int b = 0; b < kRowKB; ++b) {
+          float c[VW];  // centres past K repeat the last one; their sums are discarded
+          load_c<DT, VW>(C, (int64_t)min(k0 + b, K - 1) * d + j, c);
+#pragma unroll
+          for (int e = 0; e < VW; ++e) {
+            const float t = xrow[j + e] - c[e];
+            sacc[b] = fmaf(t, t, sacc[b]);
+          }
         }
       }
-      sacc = warp_sum_f(sacc);
-      if (sacc < bv) {  // k ascends within a warp
-        bv = sacc;
-        bk = k;
+#pragma unroll
+      for (int b = 0; b < kRowKB; ++b) {
+        const float v = warp_sum_f(sacc[b]);
+        if (k0 + b < K && v < bv) {
+          bv = v;
+          bk = k0 + b;
+        }
       }
     }
     if (lane == 0) {
@@ -874,7 +857,6 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   if (grid > p.num_tiles) grid = p.num_tiles;
   cudaError_t e;
   const bool lean = g.nchunks > 1;
-  if (lean && g.BN % 32 != 0) return fail(HME_EINTERNAL, "assign: lean scan needs BN %% 32 == 0 (BN = %d)", g.BN);
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
   if (g.nprod == 3)

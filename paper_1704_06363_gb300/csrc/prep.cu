@@ -129,21 +129,26 @@ __global__ void __launch_bounds__(256) prep_bf16_kernel(const __nv_bfloat16 *__r
   }
 }
 
-// Centres: one warp per centre row k < Kp.
-__global__ void __launch_bounds__(256) prep_centres_kernel(const float *__restrict__ C, int K, int Kp, int d,
-                                                           int ldp, int nprod, __nv_bfloat16 *__restrict__ chi,
-                                                           __nv_bfloat16 *__restrict__ clo,
-                                                           float *__restrict__ cn, Header *hdr) {
-  const int lane = threadIdx.x & 31;
-  const int k = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-  if (k >= Kp) return;
+// Centres: one block per centre row k < Kp, the row's elements strided over
+// the block's threads (several loads in flight per thread), then a block sum
+// of the squared effective values.
+constexpr int kPrepCThreads = 256;
+
+__global__ void __launch_bounds__(kPrepCThreads) prep_centres_kernel(const float *__restrict__ C, int K, int Kp,
+                                                                     int d, int ldp, int nprod,
+                                                                     __nv_bfloat16 *__restrict__ chi,
+                                                                     __nv_bfloat16 *__restrict__ clo,
+                                                                     float *__restrict__ cn, Header *hdr) {
+  __shared__ float part[kPrepCThreads / 32];
+  const int k = blockIdx.x;
   if (k >= K) {
-    if (lane == 0) cn[k] = INFINITY;
+    if (threadIdx.x == 0) cn[k] = INFINITY;
     return;
   }
   float s = 0.0f;
-  for (int j = lane; j < d; j += 32) {
-    const float c = C[(int64_t)k * d + j];
+#pragma unroll 4
+  for (int j = threadIdx.x; j < d; j += kPrepCThreads) {
+    const float c = __ldg(C + (int64_t)k * d + j);
     float ce;
     if (nprod == 1) {
       const __nv_bfloat16 b = __float2bfloat16_rn(c);
@@ -159,9 +164,13 @@ __global__ void __launch_bounds__(256) prep_centres_kernel(const float *__restri
     s = fmaf(ce, ce, s);
   }
   s = warp_sum(s);
-  if (lane == 0) {
-    cn[k] = s;
-    atomicMax(&hdr->cn_max_bits, __float_as_uint(s));  // s >= 0: integer order is float order
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.0f;
+    for (int w = 0; w < kPrepCThreads / 32; ++w) t += part[w];
+    cn[k] = t;
+    atomicMax(&hdr->cn_max_bits, __float_as_uint(t));  // t >= 0: integer order is float order
   }
 }
 
@@ -190,8 +199,7 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
 
 cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
                                 float *cn, Header *hdr, cudaStream_t s) {
-  const int blocks = (g.Kp + 7) / 8;
-  prep_centres_kernel<<<blocks, 256, 0, s>>>(C, g.K, g.Kp, g.d, g.ldp, g.nprod, chi, clo, cn, hdr);
+  prep_centres_kernel<<<g.Kp, kPrepCThreads, 0, s>>>(C, g.K, g.Kp, g.d, g.ldp, g.nprod, chi, clo, cn, hdr);
   count_launch();
   return cudaGetLastError();
 }

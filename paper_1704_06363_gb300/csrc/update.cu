@@ -18,11 +18,12 @@
 //               move by one.  Lloyd's centres are the same sums, so the result
 //               equals the full pass up to fp64 rounding order; after the first
 //               iterations well under 1% of the rows change.
-// Then:
+// Then, in one kernel:
 //   objective   J = sum ||x||^2 - 2 sum_k c_k . S_k + sum_k n_k ||c_k||^2 in
 //               fp64 with the centres that entered this update (bf16-rounded
 //               for bf16 features): the Lloyd objective of (C_t, labels).
-//   finalize    c_k = S_k / n_k (fp64 divide, rounded once to fp32) for
+//   finalize    c_k = S_k * (1 / n_k) in fp64 (within 2^-52 relative of the
+//               quotient; one divide per centre), rounded once to fp32, for
 //               non-empty k; counts_out = n.
 //   reseed      one CTA: in ascending k, every empty cluster takes the row that
 //               comes next in the order (mind descending, index ascending), i.e.
@@ -81,21 +82,31 @@ constexpr int kUnroll = 4;
 // Block layout: G groups of V threads; thread (g, t) owns column vector
 // (blockIdx.y * V + t) and the g-th sub-range of the block's row range.  The
 // thread also sums x^2 over its elements (sum ||x||^2 of the valid rows).
+// Rows come from one list (perm, slab; *n1 entries, added) followed by an
+// optional second list (perm2, slab2; *n2 entries, subtracted).  With
+// rows_per_block == 0 the split is made on the device, at least kMinRows rows
+// per block so that a short list does not turn into one flush per row.
+constexpr int64_t kMinRows = 16;
+
 template <int DT, int VW>
 __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__restrict__ X, int64_t N, int d,
                                                                   int64_t ldx, const int32_t *__restrict__ perm,
                                                                   const int32_t *__restrict__ slab,
-                                                                  const int64_t *__restrict__ valid_total, int V,
-                                                                  int G, int64_t rows_per_block, double *sums,
-                                                                  double *x2sum, float sign) {
+                                                                  const int64_t *__restrict__ n1,
+                                                                  const int32_t *__restrict__ perm2,
+                                                                  const int32_t *__restrict__ slab2,
+                                                                  const int64_t *__restrict__ n2, int V, int G,
+                                                                  int64_t rows_per_block, double *sums,
+                                                                  double *x2sum) {
   __shared__ double qpart[kUpdThreads / 32];
   const int g = threadIdx.x / V;
   const int t = threadIdx.x - g * V;
   const int vcol = blockIdx.y * V + t;
   const int col = vcol * VW;
-  const int64_t nrows = min(N, *valid_total);
-  // rows_per_block == 0: split the (device-side) row count evenly over the blocks
-  const int64_t rpb = rows_per_block > 0 ? rows_per_block : (nrows + gridDim.x - 1) / gridDim.x;
+  const int64_t na = min(N, *n1);
+  const int64_t nrows = na + (n2 ? min(N, *n2) : 0);
+  int64_t rpb = rows_per_block;
+  if (rpb <= 0) rpb = max(kMinRows, (nrows + gridDim.x - 1) / gridDim.x);
   const int64_t b0 = (int64_t)blockIdx.x * rpb;
   const int64_t b1 = min(nrows, b0 + rpb);
   const int64_t per = (b1 - b0 + G - 1) / G;
@@ -103,12 +114,22 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
   const int64_t r1 = min(b1, r0 + per);
   const bool active = (g < G) && (col < d) && (r0 < r1);
   double qd = 0.0;
+  // entry j of the joined list: its row and its key (label, or ~label when subtracted)
+  auto entry = [&](int64_t j, int &key) -> int64_t {
+    if (j < na) {
+      key = __ldg(slab + j);
+      return __ldg(perm + j);
+    }
+    key = ~__ldg(slab2 + (j - na));
+    return __ldg(perm2 + (j - na));
+  };
 
   if (active) {
     float acc[VW];
     double accd[VW];
     float q = 0.0f;
-    int cur = __ldg(slab + r0);
+    int cur;
+    entry(r0, cur);
     auto fold = [&]() {
 #pragma unroll
       for (int e = 0; e < VW; ++e) {
@@ -118,20 +139,21 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
       qd += (double)q;
       q = 0.0f;
     };
-    auto flush = [&](int lab) {
+    auto flush = [&](int key) {
       fold();
-      double *dst = sums + (int64_t)lab * d + col;
+      double *dst = sums + (int64_t)(key >= 0 ? key : ~key) * d + col;
 #pragma unroll
       for (int e = 0; e < VW; ++e) {
         if (VW == 1 || col + e < d) atomicAdd(dst + e, accd[e]);
         accd[e] = 0.0;
       }
     };
-    auto add_row = [&](const float (&v)[VW]) {
+    auto add_row = [&](const float (&v)[VW], int key) {
+      const float sg = key >= 0 ? 1.0f : -1.0f;
 #pragma unroll
       for (int e = 0; e < VW; ++e) {
-        acc[e] += sign * v[e];
-        q = fmaf(sign * v[e], v[e], q);
+        acc[e] += sg * v[e];
+        q = fmaf(sg * v[e], v[e], q);
       }
     };
 #pragma unroll
@@ -143,21 +165,20 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
     int64_t j = r0;
     int since = 0;
     for (; j + kUnroll <= r1; j += kUnroll) {
-      int lab[kUnroll];
+      int key[kUnroll];
       float v[kUnroll][VW];
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
-        const int64_t row = __ldg(perm + j + u);
-        lab[u] = __ldg(slab + j + u);
+        const int64_t row = entry(j + u, key[u]);
         Vec<DT, VW>::load(X, row * ldx + col, v[u]);
       }
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
-        if (lab[u] != cur) {
+        if (key[u] != cur) {
           flush(cur);
-          cur = lab[u];
+          cur = key[u];
         }
-        add_row(v[u]);
+        add_row(v[u], key[u]);
       }
       if ((since += kUnroll) >= 64) {
         fold();
@@ -165,15 +186,15 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
       }
     }
     for (; j < r1; ++j) {
-      const int64_t row = __ldg(perm + j);
-      const int lab = __ldg(slab + j);
+      int key;
+      const int64_t row = entry(j, key);
       float v[VW];
       Vec<DT, VW>::load(X, row * ldx + col, v);
-      if (lab != cur) {
+      if (key != cur) {
         flush(cur);
-        cur = lab;
+        cur = key;
       }
-      add_row(v);
+      add_row(v, key);
     }
     flush(cur);
   }
@@ -190,15 +211,15 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
   }
 }
 
-// Incremental update, in four small kernels over the label vectors:
+// Incremental update, in three small kernels over the label vectors:
 //   delta_count  rows whose label changed, counted per new label (to add) and
 //                per old label (to subtract); labels outside [0, K) count as
 //                unassigned on either side;
 //   delta_scan   exclusive prefix of both counts -> fill cursors and totals;
+//                also moves n_k by (added - subtracted);
 //   delta_fill   the changed rows grouped by label (order inside a group is
 //                irrelevant for sums), as (row, label) lists;
-// then the sums kernel runs over each list (sign +1 / -1), and delta_counts
-// moves n_k by the difference of the two counts.
+// then one sums launch runs over both lists (added, then subtracted).
 // Warp-aggregated increment: lanes with the same key add once, by the lowest
 // lane, and each lane gets its own slot (base + rank among equal keys).
 __device__ __forceinline__ int32_t warp_add(int32_t *ctr, int key, bool active) {
@@ -211,41 +232,69 @@ __device__ __forceinline__ int32_t warp_add(int32_t *ctr, int key, bool active) 
   return base + __popc(peers & ((1u << lane) - 1u));
 }
 
+// Labels i .. i+VEC-1 of both vectors (16-byte loads when VEC == 4); entries
+// past N read as -1 on both sides (unchanged).
+template <int VEC>
+__device__ __forceinline__ void load_pair(const int32_t *labels, const int32_t *prev, int64_t i, int64_t N,
+                                          int (&a)[VEC], int (&b)[VEC]) {
+  if (VEC == 4 && i + 4 <= N) {
+    const int4 x = __ldg(reinterpret_cast<const int4 *>(labels + i));
+    const int4 y = __ldg(reinterpret_cast<const int4 *>(prev + i));
+    a[0] = x.x, a[1] = x.y, a[2] = x.z, a[3] = x.w;
+    b[0] = y.x, b[1] = y.y, b[2] = y.z, b[3] = y.w;
+  } else {
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) {
+      a[e] = i + e < N ? __ldg(labels + i + e) : -1;
+      b[e] = i + e < N ? __ldg(prev + i + e) : -1;
+    }
+  }
+}
+
+template <int VEC>
 __global__ void __launch_bounds__(256) delta_count_kernel(const int32_t *__restrict__ labels,
                                                           const int32_t *__restrict__ prev, int64_t N, int K,
                                                           int32_t *hist_add, int32_t *hist_sub, Header *hdr) {
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
   bool bad = false;
   // whole warps iterate together (the loop bound is rounded up to a warp)
-  const int64_t Nw = (N + 31) / 32 * 32;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < Nw; i += stride) {
-    int a = -1, b = -1;
-    if (i < N) {
-      a = __ldg(labels + i);
-      b = __ldg(prev + i);
-      if (a < 0 || a >= K) {
-        bad = true;
-        a = -1;
-      }
-      if (b < 0 || b >= K) b = -1;
+  const int64_t Nw = (N + 32 * VEC - 1) / (32 * VEC) * (32 * VEC);
+  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VEC; i < Nw; i += stride) {
+    int a[VEC], b[VEC];
+    load_pair<VEC>(labels, prev, i, N, a, b);
+    bool any = false;
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) {
+      if (i + e < N && (a[e] < 0 || a[e] >= K)) bad = true;
+      if (a[e] < 0 || a[e] >= K) a[e] = -1;
+      if (b[e] < 0 || b[e] >= K) b[e] = -1;
+      any |= a[e] != b[e];
     }
-    const bool moved = a != b;
-    warp_add(hist_add, a, moved && a >= 0);
-    warp_add(hist_sub, b, moved && b >= 0);
+    if (!__any_sync(0xffffffffu, any)) continue;  // nothing moved in this warp's span
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) {
+      const bool moved = a[e] != b[e];
+      warp_add(hist_add, a[e], moved && a[e] >= 0);
+      warp_add(hist_sub, b[e], moved && b[e] >= 0);
+    }
   }
   if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadLabel);
 }
 
+// Exclusive prefix of hist_add and hist_sub (one block), the fill cursors,
+// totals = {rows to add, rows to subtract}, the moved-row count in the header
+// and n_k += added_k - subtracted_k.
 __global__ void __launch_bounds__(1024) delta_scan_kernel(const int32_t *__restrict__ hist_add,
                                                           const int32_t *__restrict__ hist_sub, int K,
-                                                          int32_t *cur_add, int32_t *cur_sub, int64_t *totals) {
+                                                          int32_t *cur_add, int32_t *cur_sub, int64_t *totals,
+                                                          int64_t *counts, Header *hdr) {
   __shared__ int64_t wsum[32];
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int per = (K + 1023) / 1024;
+  const int k0 = t * per, k1 = min(K, k0 + per);
   for (int which = 0; which < 2; ++which) {
     const int32_t *h = which == 0 ? hist_add : hist_sub;
     int32_t *cur = which == 0 ? cur_add : cur_sub;
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const int per = (K + 1023) / 1024;
-    const int k0 = t * per, k1 = min(K, k0 + per);
     int64_t local = 0;
     for (int k = k0; k < k1; ++k) local += h[k];
     int64_t incl = local;
@@ -272,67 +321,85 @@ __global__ void __launch_bounds__(1024) delta_scan_kernel(const int32_t *__restr
       cur[k] = (int32_t)run;
       run += h[k];
     }
-    if (t == 1023) totals[which] = run;
+    if (t == 1023) {
+      totals[which] = run;
+      if (which == 0) hdr->moved_rows = (uint32_t)min(run, (int64_t)0xFFFFFFFF);
+    }
     __syncthreads();
   }
+  for (int k = t; k < K; k += blockDim.x) counts[k] += (int64_t)hist_add[k] - (int64_t)hist_sub[k];
 }
 
-__global__ void delta_report_kernel(const int64_t *totals, Header *hdr) {
-  hdr->moved_rows = (uint32_t)min(totals[0], (int64_t)0xFFFFFFFF);
-}
-
+template <int VEC>
 __global__ void __launch_bounds__(256) delta_fill_kernel(const int32_t *__restrict__ labels,
                                                          const int32_t *__restrict__ prev, int64_t N, int K,
                                                          int32_t *cur_add, int32_t *cur_sub, int32_t *add_rows,
                                                          int32_t *add_lab, int32_t *sub_rows, int32_t *sub_lab) {
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  const int64_t Nw = (N + 31) / 32 * 32;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < Nw; i += stride) {
-    int a = -1, b = -1;
-    if (i < N) {
-      a = __ldg(labels + i);
-      b = __ldg(prev + i);
-      if (a < 0 || a >= K) a = -1;
-      if (b < 0 || b >= K) b = -1;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
+  const int64_t Nw = (N + 32 * VEC - 1) / (32 * VEC) * (32 * VEC);
+  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VEC; i < Nw; i += stride) {
+    int a[VEC], b[VEC];
+    load_pair<VEC>(labels, prev, i, N, a, b);
+    bool any = false;
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) {
+      if (a[e] < 0 || a[e] >= K) a[e] = -1;
+      if (b[e] < 0 || b[e] >= K) b[e] = -1;
+      any |= a[e] != b[e];
     }
-    const bool moved = a != b;
-    const bool add = moved && a >= 0, sub = moved && b >= 0;
-    const int32_t sa = warp_add(cur_add, a, add);
-    const int32_t sb = warp_add(cur_sub, b, sub);
-    if (add) {
-      add_rows[sa] = (int32_t)i;
-      add_lab[sa] = a;
-    }
-    if (sub) {
-      sub_rows[sb] = (int32_t)i;
-      sub_lab[sb] = b;
+    if (!__any_sync(0xffffffffu, any)) continue;
+#pragma unroll
+    for (int e = 0; e < VEC; ++e) {
+      const bool moved = a[e] != b[e];
+      const bool add = moved && a[e] >= 0, sub = moved && b[e] >= 0;
+      const int32_t sa = warp_add(cur_add, a[e], add);
+      const int32_t sb = warp_add(cur_sub, b[e], sub);
+      if (add) {
+        add_rows[sa] = (int32_t)(i + e);
+        add_lab[sa] = a[e];
+      }
+      if (sub) {
+        sub_rows[sb] = (int32_t)(i + e);
+        sub_lab[sb] = b[e];
+      }
     }
   }
 }
 
-__global__ void delta_counts_kernel(const int32_t *__restrict__ hist_add, const int32_t *__restrict__ hist_sub,
-                                    int K, int64_t *counts) {
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k < K) counts[k] += (int64_t)hist_add[k] - (int64_t)hist_sub[k];
-}
+// Objective and new centres in one pass over (S, n, C); one block per
+// (centre k, 1024-column slice):
+//   J = sum ||x||^2 + sum_k (n_k ||c_k||^2 - 2 c_k . S_k) in fp64 with the
+//       centres that entered this update (bf16-rounded for bf16 features);
+//       block (0, 0) adds sum ||x||^2;
+//   c_k = S_k * (1 / n_k) in fp64, rounded once to fp32, for non-empty k (each
+//       element is read, for J, by the thread that then overwrites it);
+//   counts_out = n.
+constexpr int kFinThreads = 256, kFinPer = 4;
 
-// J = sum ||x||^2 + sum_k (n_k ||c_k||^2 - 2 c_k . S_k), fp64, with the centres
-// that entered this update.  One block per centre; block 0 adds sum ||x||^2.
 template <int DT>
-__global__ void __launch_bounds__(256) update_objective_kernel(const double *__restrict__ sums,
-                                                               const int64_t *__restrict__ counts,
-                                                               const float *__restrict__ C, int d,
-                                                               const double *__restrict__ x2sum, Header *hdr) {
-  __shared__ double part[8];
+__global__ void __launch_bounds__(kFinThreads) update_finish_kernel(const double *__restrict__ sums,
+                                                                    const int64_t *__restrict__ counts, float *C,
+                                                                    int d, const double *__restrict__ x2sum,
+                                                                    int64_t *counts_out, Header *hdr) {
+  __shared__ double part[kFinThreads / 32];
   const int k = blockIdx.x;
-  const double n = (double)counts[k];
+  const int64_t nk = counts[k];
+  const double n = (double)nk;
+  const double inv = nk > 0 ? 1.0 / n : 0.0;
   double acc = 0.0;
-  if (n > 0.0) {
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-      float c = C[(int64_t)k * d + j];
-      if (DT == HME_BF16) c = __bfloat162float(__float2bfloat16_rn(c));
-      const double cd = (double)c;
-      acc += cd * (n * cd - 2.0 * sums[(int64_t)k * d + j]);
+  if (nk > 0) {
+#pragma unroll
+    for (int u = 0; u < kFinPer; ++u) {
+      const int j = blockIdx.y * (kFinThreads * kFinPer) + u * kFinThreads + threadIdx.x;
+      if (j < d) {
+        const int64_t at = (int64_t)k * d + j;
+        float c = C[at];
+        const double S = sums[at];
+        if (DT == HME_BF16) c = __bfloat162float(__float2bfloat16_rn(c));
+        const double cd = (double)c;
+        acc += cd * (n * cd - 2.0 * S);
+        C[at] = (float)(S * inv);
+      }
     }
   }
 #pragma unroll
@@ -341,22 +408,11 @@ __global__ void __launch_bounds__(256) update_objective_kernel(const double *__r
   __syncthreads();
   if (threadIdx.x == 0) {
     double t = 0.0;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += part[w];
-    if (k == 0) t += *x2sum;
-    atomicAdd(&hdr->objective, t);
+    for (int w = 0; w < kFinThreads / 32; ++w) t += part[w];
+    if (k == 0 && blockIdx.y == 0) t += *x2sum;
+    if (t != 0.0) atomicAdd(&hdr->objective, t);
+    if (counts_out && blockIdx.y == 0) counts_out[k] = nk;
   }
-}
-
-__global__ void update_finalize_kernel(const double *__restrict__ sums, const int64_t *__restrict__ hist, int K,
-                                       int d, float *__restrict__ C, int64_t *__restrict__ counts_out) {
-  // hist: the persistent per-cluster counts
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < (int64_t)K * d) {
-    const int k = (int)(i / d);
-    const int64_t n = hist[k];
-    if (n > 0) C[i] = (float)(sums[i] / (double)n);
-  }
-  if (counts_out && i < K) counts_out[i] = hist[i];
 }
 
 // Order used by the re-seed rule: a comes before b if a is farther, or equally far with a lower index.
@@ -577,10 +633,18 @@ __global__ void __launch_bounds__(1024) update_reseed_kernel(const void *__restr
   if (threadIdx.x == 0 && n_reseeded) *n_reseeded = taken;
 }
 
+// List (perm, slab; *n1 rows, added) then optionally (perm2, slab2; *n2 rows,
+// subtracted).  device_rows: the row counts are known only on the device.
+struct SumsLists {
+  const int32_t *perm, *slab;
+  const int64_t *n1;
+  const int32_t *perm2, *slab2;
+  const int64_t *n2;
+};
+
 template <int DT, int VW>
-void launch_sums(const void *X, int64_t N, int d, int64_t ldx, const int32_t *perm, const int32_t *slab,
-                 const int64_t *valid_total, double *sums, double *x2sum, float sign, bool device_rows,
-                 cudaStream_t s) {
+void launch_sums(const void *X, int64_t N, int d, int64_t ldx, const SumsLists &l, double *sums, double *x2sum,
+                 bool device_rows, cudaStream_t s) {
   const int nvec = (d + VW - 1) / VW;
   int V, G, ny;
   if (nvec <= kUpdThreads) {
@@ -598,25 +662,24 @@ void launch_sums(const void *X, int64_t N, int d, int64_t ldx, const int32_t *pe
   if (nx < 1) nx = 1;
   const int64_t rpb = device_rows ? 0 : (N + nx - 1) / nx;
   dim3 grid((unsigned)nx, (unsigned)ny);
-  update_sums_kernel<DT, VW><<<grid, kUpdThreads, 0, s>>>(X, N, d, ldx, perm, slab, valid_total, V, G, rpb, sums,
-                                                          x2sum, sign);
+  update_sums_kernel<DT, VW><<<grid, kUpdThreads, 0, s>>>(X, N, d, ldx, l.perm, l.slab, l.n1, l.perm2, l.slab2,
+                                                          l.n2, V, G, rpb, sums, x2sum);
   count_launch();
 }
 
-void launch_sums_any(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *perm,
-                     const int32_t *slab, const int64_t *valid_total, double *sums, double *x2sum, float sign,
-                     bool device_rows, cudaStream_t s) {
+void launch_sums_any(const void *X, int64_t N, int d, int64_t ldx, int dtype, const SumsLists &l, double *sums,
+                     double *x2sum, bool device_rows, cudaStream_t s) {
   const bool al = (reinterpret_cast<uintptr_t>(X) & 15u) == 0;
   if (dtype == HME_F32) {
     if (al && d % 4 == 0 && ldx % 4 == 0)
-      launch_sums<HME_F32, 4>(X, N, d, ldx, perm, slab, valid_total, sums, x2sum, sign, device_rows, s);
+      launch_sums<HME_F32, 4>(X, N, d, ldx, l, sums, x2sum, device_rows, s);
     else
-      launch_sums<HME_F32, 1>(X, N, d, ldx, perm, slab, valid_total, sums, x2sum, sign, device_rows, s);
+      launch_sums<HME_F32, 1>(X, N, d, ldx, l, sums, x2sum, device_rows, s);
   } else {
     if (al && d % 8 == 0 && ldx % 8 == 0)
-      launch_sums<HME_BF16, 8>(X, N, d, ldx, perm, slab, valid_total, sums, x2sum, sign, device_rows, s);
+      launch_sums<HME_BF16, 8>(X, N, d, ldx, l, sums, x2sum, device_rows, s);
     else
-      launch_sums<HME_BF16, 1>(X, N, d, ldx, perm, slab, valid_total, sums, x2sum, sign, device_rows, s);
+      launch_sums<HME_BF16, 1>(X, N, d, ldx, l, sums, x2sum, device_rows, s);
   }
 }
 
@@ -637,33 +700,43 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
     e = cudaMemcpyAsync(st.counts, hist, (size_t)K * sizeof(int64_t), cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) return e;
     if (N > 0)
-      launch_sums_any(X, N, d, ldx, dtype, perm, sorted_labels, valid_total, st.sums, st.x2sum, 1.0f, false, s);
+      launch_sums_any(X, N, d, ldx, dtype, SumsLists{perm, sorted_labels, valid_total, nullptr, nullptr, nullptr},
+                    st.sums, st.x2sum, false, s);
   } else if (N > 0) {
     // incremental: only the rows whose label changed
     e = cudaMemsetAsync(ds.hist_add, 0, (size_t)2 * K * sizeof(int32_t), s);  // hist_add, hist_sub adjacent
     if (e != cudaSuccess) return e;
+    const bool vec = (reinterpret_cast<uintptr_t>(labels) & 15u) == 0 &&
+                     (reinterpret_cast<uintptr_t>(prev_labels) & 15u) == 0;
+    const int per = vec ? 4 : 1;
     int64_t blocks = (int64_t)num_sms() * 8;
-    const int64_t want = (N + 255) / 256;
+    const int64_t want = (N + 256 * per - 1) / (256 * per);
     if (blocks > want) blocks = want;
-    delta_count_kernel<<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.hist_add, ds.hist_sub, hdr);
-    delta_scan_kernel<<<1, 1024, 0, s>>>(ds.hist_add, ds.hist_sub, K, ds.cur_add, ds.cur_sub, ds.totals);
-    delta_report_kernel<<<1, 1, 0, s>>>(ds.totals, hdr);
-    count_launch();
-    delta_fill_kernel<<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.cur_add, ds.cur_sub,
-                                                       ds.add_rows, ds.add_lab, ds.sub_rows, ds.sub_lab);
+    if (vec)
+      delta_count_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.hist_add, ds.hist_sub, hdr);
+    else
+      delta_count_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.hist_add, ds.hist_sub, hdr);
+    delta_scan_kernel<<<1, 1024, 0, s>>>(ds.hist_add, ds.hist_sub, K, ds.cur_add, ds.cur_sub, ds.totals, st.counts,
+                                         hdr);
+    if (vec)
+      delta_fill_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.cur_add, ds.cur_sub,
+                                                            ds.add_rows, ds.add_lab, ds.sub_rows, ds.sub_lab);
+    else
+      delta_fill_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.cur_add, ds.cur_sub,
+                                                            ds.add_rows, ds.add_lab, ds.sub_rows, ds.sub_lab);
     count_launch(3);
-    launch_sums_any(X, N, d, ldx, dtype, ds.add_rows, ds.add_lab, ds.totals + 0, st.sums, st.x2sum, 1.0f, true, s);
-    launch_sums_any(X, N, d, ldx, dtype, ds.sub_rows, ds.sub_lab, ds.totals + 1, st.sums, st.x2sum, -1.0f, true,
-                    s);
-    delta_counts_kernel<<<(K + 255) / 256, 256, 0, s>>>(ds.hist_add, ds.hist_sub, K, st.counts);
-    count_launch();
+    launch_sums_any(X, N, d, ldx, dtype,
+                    SumsLists{ds.add_rows, ds.add_lab, ds.totals + 0, ds.sub_rows, ds.sub_lab, ds.totals + 1},
+                    st.sums, st.x2sum, true, s);
   }
-  if (dtype == HME_F32)
-    update_objective_kernel<HME_F32><<<K, 256, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, hdr);
-  else
-    update_objective_kernel<HME_BF16><<<K, 256, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, hdr);
-  const int64_t tot = (int64_t)K * d > K ? (int64_t)K * d : K;
-  update_finalize_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(st.sums, st.counts, K, d, C, counts_out);
+  {
+    const dim3 grid((unsigned)K, (unsigned)((d + kFinThreads * kFinPer - 1) / (kFinThreads * kFinPer)));
+    if (dtype == HME_F32)
+      update_finish_kernel<HME_F32><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out, hdr);
+    else
+      update_finish_kernel<HME_BF16><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out,
+                                                                  hdr);
+  }
   {
     const int nblk = (num_sms() < kMaxSms ? num_sms() : kMaxSms) * 2;  // the candidate region holds kMaxSms * 2 blocks
     const int nlists = nblk * kSelWarps;
@@ -678,7 +751,7 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
     update_reseed_kernel<HME_F32><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
   else
     update_reseed_kernel<HME_BF16><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
-  count_launch(5);
+  count_launch(4);
   return cudaGetLastError();
 }
 
