@@ -259,7 +259,7 @@ def run_ours(args, w):
         step(X)
     status = hme.hme_sync_status(ws)
     if status != hme.HME_OK:
-        raise RuntimeError(f"device status {status} after warm-up")
+        raise RuntimeError(f"device status {status} after warm-up: {hme.hme_last_error()}")
 
     clocks = Clocks(local)
     if world > 1:
@@ -280,7 +280,25 @@ def run_ours(args, w):
     rescored = {"pair": int(hdr[1]), "all_k": int(hdr[3])}
     moved = int(moved_dev.item())  # rows that changed label in the last update of a warm-up step
     ms = max_over_ranks(e0.elapsed_time(e1), dev)
-    assert hme.hme_sync_status(ws) == hme.HME_OK
+    status = hme.hme_sync_status(ws)
+    if status != hme.HME_OK:
+        raise RuntimeError(f"device status {status} after the timed steps: {hme.hme_last_error()}")
+
+    # outside the timed steps: routing the same rows as a one-off call (no
+    # preparation; fp32 rows with K <= 256 are split inside the kernel) against
+    # the prepared route the step uses
+    route_ms = {}
+    for name, fl in (("route_prepared", hme.HME_ASSIGN_PREPARED), ("route_unprepared", 0)):
+        r0 = torch.cuda.Event(enable_timing=True)
+        r1 = torch.cuda.Event(enable_timing=True)
+        r0.record(stream)
+        hme.hme_route(X, C, expert, offsets, order, ws, flags=fl)
+        r1.record(stream)
+        torch.cuda.synchronize(dev)
+        route_ms[name] = r0.elapsed_time(r1)
+    status = hme.hme_sync_status(ws)
+    if status != hme.HME_OK:
+        raise RuntimeError(f"device status {status} after the route comparison: {hme.hme_last_error()}")
 
     iters_total = T * args.steps * world
     value = iters_total / (ms / 1000.0)
@@ -361,6 +379,7 @@ def run_ours(args, w):
             "vectors_per_s": N * iters_total / (ms / 1000.0),
             "assign_gflops": flops_assign / (t_assign / 1000.0) / 1e9,
             "kernels_ms": {"assign_call": t_assign, "update_call_full": t_update, "update_call_incremental": t_incr,
+                           **route_ms,
                            "assign_gbs": a_gbs, "update_full_gbs": u_gbs},
             "roofline": roofline,
             "cpu_baseline": cpu,

@@ -123,6 +123,11 @@ HME_API int hme_kmeans_init(const void *X, int64_t N, int32_t d, int64_t ldx, in
  * norms are then those of hi + lo).  Writes
  * ws only.  Pass HME_ASSIGN_PREPARED to hme_assign to reuse it for every
  * iteration; the (N, d, K, dtype) of the later calls must be the same.
+ * Without HME_ASSIGN_PREPARED, hme_assign and hme_route on HME_F32 features
+ * with K <= 256 whose rows TMA can read (X on a 16-byte boundary,
+ * ldx % 4 == 0) split each fp32 row inside the kernel as it arrives: one pass
+ * over X instead of three for a one-off call.  With it they read the prepared
+ * split, which streams faster when the same X is assigned many times.
  */
 HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
                          void *ws, size_t ws_bytes, void *stream);

@@ -197,22 +197,44 @@ int do_prepare(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, c
   return HME_OK;
 }
 
+int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, const AssignGeom &g, const Layout &L,
+                           void *ws, int32_t *labels, float *mind, Header *hdr, cudaStream_t s);
+
+// prepared: ws holds this X's preparation (hme_prepare_features).  An
+// unprepared call on fp32 features that TMA can read splits the rows inside
+// the assign kernel (one pass over X); any other unprepared call prepares
+// first.  Prepared calls use the prepared operands, which stream at the
+// full HBM rate.
 int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K, int32_t *labels,
-              float *mind, const Layout &L, void *ws, cudaStream_t s) {
+              float *mind, const Layout &L, void *ws, bool prepared, cudaStream_t s) {
   const AssignGeom g = assign_geom(d, K, dtype);
+  const bool split = !prepared && split_eligible(X, ldx, g);
+  if (!prepared && !split) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s));
   Header *hdr = at<Header>(ws, 0);
   HME_CUDA(launch_prep_centres(C, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
                                at<float>(ws, L.cn), hdr, s),
            "prepare centres");
+  if (split) {
+    HME_TRY(launch_assign_split(static_cast<const float *>(X), N, ldx, g, at<__nv_bfloat16>(ws, L.cb_hi),
+                                at<__nv_bfloat16>(ws, L.cb_lo), at<float>(ws, L.cn), labels, mind, hdr,
+                                at<int32_t>(ws, L.flagged), at<int32_t>(ws, L.full_rows), s));
+  } else {
+    HME_TRY(launch_assign_prepared(X, N, ldx, dtype, g, L, ws, labels, mind, hdr, s));
+  }
+  HME_CUDA(launch_rescore(X, N, d, ldx, dtype, C, K, labels, mind, hdr, at<int32_t>(ws, L.flagged),
+                          at<int32_t>(ws, L.full_rows), s),
+           "re-score");
+  return HME_OK;
+}
+
+int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, const AssignGeom &g, const Layout &L,
+                           void *ws, int32_t *labels, float *mind, Header *hdr, cudaStream_t s) {
   const void *Xa = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xhi) : X;
   const void *Xb = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;
   const int64_t lda = dtype == HME_F32 ? g.ldp : ldx;
   HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
                         at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged),
                         at<int32_t>(ws, L.full_rows), s));
-  HME_CUDA(launch_rescore(X, N, d, ldx, dtype, C, K, labels, mind, hdr, at<int32_t>(ws, L.flagged),
-                          at<int32_t>(ws, L.full_rows), s),
-           "re-score");
   return HME_OK;
 }
 
@@ -309,8 +331,7 @@ int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, 
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  if (!(flags & HME_ASSIGN_PREPARED)) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s));
-  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, s));
+  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s));
   if (objective_out)
     HME_CUDA(cudaMemcpyAsync(objective_out, &at<Header>(ws, 0)->objective, sizeof(double), cudaMemcpyDeviceToDevice,
                              s),
@@ -390,8 +411,7 @@ int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, c
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  if (!(flags & HME_ASSIGN_PREPARED)) HME_TRY(do_prepare(Q, B, d, ldq, dtype, K, L, ws, s));
-  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, s));
+  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s));
   HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
                             offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
            "route: partition");

@@ -51,6 +51,11 @@ struct AssignParams {
   uint32_t acc_stride; // columns between accumulator buffers
   int nbuf;            // accumulator buffers (2: epilogue overlaps the next MMAs)
   uint32_t a_res_bytes;  // resident A region (0 unless the A rows stay resident)
+  // in-kernel split of fp32 features (assign_split_kernel)
+  int sb_stages;          // centre (B) stages
+  int st_stages;          // split A stages in tensor memory
+  uint32_t b_stage_bytes; // one B stage (hi and lo operands)
+  uint32_t a_col0;        // first TMEM column of the A stages
   const float *xn;
   const float *cn;     // Kp entries, +inf past K
   int32_t *labels;
@@ -129,6 +134,45 @@ __device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float 
     }
   }
   i1 = (b1 < before) ? k0 + jl : i1;
+}
+
+// The result of one row's scan: label, distance, and for a near tie a
+// re-score request.  A centre whose tensor-core distance is within E of the
+// best could be the true nearest one.  E bounds the error of a difference of
+// two computed distances: each fp32 accumulation step of x.c errs by at most
+// one ulp of the accumulator (|x.c| <= (||x||^2 + ||c||^2) / 2), the split
+// operands of fp32 features by 2^-16 per element, and the epilogue adds a few
+// roundings; the dropped xl.cl moves each distance by at most
+// 2^-15 (1 + 2^-8)^2 ||x|| ||c||.  Such rows are queued for an exact
+// comparison: of the two candidates, or of all K when a third centre is also
+// within E (or, in the lean scan, whenever the runner-up is).  Returns the
+// row's share of the objective estimate (0 for queued rows: the re-score adds
+// theirs).
+template <bool LEAN>
+__device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row, float xr, float best1, float best2,
+                                             float best3, int idx1, int idx2, float cn_max, float sqrt_cn_max) {
+  const float D1 = xr + best1;
+  const float D2 = xr + best2;
+  const float D3 = xr + best3;
+  const float md = fmaxf(D1, 0.0f);
+  p.labels[row] = idx1;
+  if (p.mind) p.mind[row] = md;
+  const float sqrt_xr = sqrtf(xr);
+  const float E = p.err_acc * (xr + cn_max) + p.err_split * (sqrt_xr + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f)) +
+                  p.err_ll * sqrt_xr * sqrt_cn_max;
+  const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
+  if (!near2) return (double)md;
+  const bool near3 = LEAN || ((best3 < INFINITY) && ((D3 - D1) <= E));
+  if (near3) {
+    const uint32_t slot = atomicAdd(&p.hdr->rescore_full_count, 1u);
+    p.full_rows[slot] = (int32_t)row;
+  } else {
+    const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
+    p.flagged[3 * slot + 0] = (int32_t)row;
+    p.flagged[3 * slot + 1] = idx1;
+    p.flagged[3 * slot + 2] = idx2;
+  }
+  return 0.0;
 }
 
 // The fused assign kernel.
@@ -410,42 +454,315 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         best1 = take_b ? lb1 : best1;
         idx1 = take_b ? li1 : idx1;
       }
-      if (row < p.N) {
-        const float D1 = xr + best1;
-        const float D2 = xr + best2;
-        const float D3 = xr + best3;
-        const float md = fmaxf(D1, 0.0f);
-        p.labels[row] = idx1;
-        if (p.mind) p.mind[row] = md;
-        // Near tie: a centre whose tensor-core distance is within E of the best
-        // could be the true nearest one.  E bounds the error of a difference of
-        // two computed distances: each fp32 accumulation step of x.c errs by at
-        // most one ulp of the accumulator (|x.c| <= (||x||^2 + ||c||^2) / 2),
-        // the split operands of fp32 features by 2^-16 per element, and the
-        // epilogue adds a few roundings; the dropped xl.cl moves each distance by
-        // at most 2^-15 (1 + 2^-8)^2 ||x|| ||c||.  Such rows are queued for an exact
-        // comparison: of the two candidates, or of all K when a third centre is
-        // also within E (or, in the lean scan, whenever the runner-up is).
-        const float sqrt_xr = sqrtf(xr);
-        const float E = p.err_acc * (xr + cn_max) +
-                        p.err_split * (sqrt_xr + sqrt_cn_max) * sqrtf(fmaxf(D2, 0.0f)) +
-                        p.err_ll * sqrt_xr * sqrt_cn_max;
-        const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
-        if (near2) {
-          const bool near3 = LEAN || ((best3 < INFINITY) && ((D3 - D1) <= E));
-          if (near3) {
-            const uint32_t slot = atomicAdd(&p.hdr->rescore_full_count, 1u);
-            p.full_rows[slot] = (int32_t)row;
-          } else {
-            const uint32_t slot = atomicAdd(&p.hdr->rescore_count, 1u);
-            p.flagged[3 * slot + 0] = (int32_t)row;
-            p.flagged[3 * slot + 1] = idx1;
-            p.flagged[3 * slot + 2] = idx2;
+      if (row < p.N) obj += finish_row<LEAN>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
+    if (lane == 0 && obj != 0.0) atomicAdd(&p.hdr->objective, obj);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// fp32 features split on the fly (one N-chunk, K <= 256)
+// ---------------------------------------------------------------------------
+// The same contraction as assign_kernel<3, false, 1, false>, with the bf16
+// hi/lo split of x made inside the kernel instead of by a preparation pass:
+// the fp32 rows arrive by TMA (two 128-row x 32-column boxes per 64-column
+// k-block, 128-byte swizzle), four converter warps split them (x = xh + xl,
+// both rounded to nearest even), sum ||xh + xl||^2 per row, and store xh and
+// xl into tensor memory, where the MMA reads them as its A operand (row m in
+// lane m, bf16 pairs along k per 32-bit column).  B (ch, cl) streams from
+// shared memory as before.  HBM traffic per row is the fp32 row itself, read
+// once per call; no split copy of X exists.
+// Warps: 0 X producer, 1 TMEM allocator + MMA issuer, 2 B producer,
+// 3-10 converters (two per TMEM lane quarter, taking alternate k-blocks, so
+// that one converts while the other waits on its stores), 11-14 epilogue
+// (warp w touches TMEM lanes 32 (w % 4) ..).
+constexpr int kSplitWarps = 15;
+constexpr int kConvFirst = 3, kEpiFirst = 11;
+constexpr int kSplitThreads = 32 * kSplitWarps;
+constexpr uint32_t kXBox = kBM * 32 * 4;  // 128 rows x 32 fp32 = 16 KB
+constexpr uint32_t kXStage = 2 * kXBox;   // one 64-column k-block
+constexpr uint32_t kWhereConv = 5;
+
+// x0, x1 -> packed bf16 pair (x0 in the low half), rounded to nearest even
+__device__ __forceinline__ uint32_t pack_bf16x2(float x0, float x1) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(x1), "f"(x0));
+  return r;
+}
+
+__global__ void __launch_bounds__(kSplitThreads, 1)
+    assign_split_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmB0,
+                        const __grid_constant__ CUtensorMap tmB1, const AssignParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  const uint32_t base = (raw_addr + 1023u) & ~1023u;
+  uint8_t *smem = smem_raw + (base - raw_addr);
+
+  const int SX = p.stages, SB = p.sb_stages, ST = p.st_stages;
+  const uint32_t xring = base;
+  const uint32_t bring = base + (uint32_t)SX * kXStage;
+  uint8_t *ctrl = smem + (size_t)SX * kXStage + (size_t)SB * p.b_stage_bytes;
+  uint64_t *x_full = reinterpret_cast<uint64_t *>(ctrl);
+  uint64_t *x_empty = x_full + SX;
+  uint64_t *b_full = x_empty + SX;
+  uint64_t *b_empty = b_full + SB;
+  uint64_t *a_full = b_empty + SB;
+  uint64_t *a_empty = a_full + ST;
+  uint64_t *tfull = a_empty + ST;
+  uint64_t *tempty = tfull + 2;
+  uint64_t *xn_full = tempty + 2;
+  uint64_t *xn_empty = xn_full + 2;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(xn_empty + 2);
+  float *xn_buf = reinterpret_cast<float *>(ctrl + 512);  // [2 buffers][2 converter halves][128 rows]
+  float *cnbuf = xn_buf + 4 * kBM;                         // [4][kMaxBN]
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int nbuf = p.nbuf;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < SX; ++i) {
+      mbar_init(smem_u32(&x_full[i]), 1);
+      mbar_init(smem_u32(&x_empty[i]), 4);
+    }
+    for (int i = 0; i < SB; ++i) {
+      mbar_init(smem_u32(&b_full[i]), 1);
+      mbar_init(smem_u32(&b_empty[i]), 1);
+    }
+    for (int i = 0; i < ST; ++i) {
+      mbar_init(smem_u32(&a_full[i]), 4);
+      mbar_init(smem_u32(&a_empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&tfull[i]), 1);
+      mbar_init(smem_u32(&tempty[i]), 4);
+      mbar_init(smem_u32(&xn_full[i]), 8);
+      mbar_init(smem_u32(&xn_empty[i]), 4);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) prefetch_tensormap(&tmX);
+  if (warp == 2 && lane == 0) {
+    prefetch_tensormap(&tmB0);
+    prefetch_tensormap(&tmB1);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), p.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    // ---------------- X producer: fp32 k-blocks ----------------
+    if (lane == 0) {
+      const uint64_t pol = l2_policy_evict_first();
+      uint32_t i = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        const int32_t row0 = tile * kBM;
+        for (int kb = 0; kb < p.num_kb; ++kb, ++i) {
+          const int s = i % SX;
+          if (!mbar_wait_bounded(smem_u32(&x_empty[s]), ((i / SX) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereProducer)) {
+            ok = false;
+            break;
           }
-        } else {
-          obj += (double)md;
+          const uint32_t fb = smem_u32(&x_full[s]);
+          mbar_arrive_expect_tx(fb, kXStage);
+          const uint32_t st = xring + (uint32_t)s * kXStage;
+          tma_load_2d(st, &tmX, fb, kb * kBK, row0, pol);
+          tma_load_2d(st + kXBox, &tmX, fb, kb * kBK + 32, row0, pol);
         }
       }
+      if (!ok)  // every copy issued must land before the CTA may end
+        for (uint32_t j = (i > (uint32_t)SX ? i - SX : 0); j < i; ++j)
+          mbar_wait_bounded(smem_u32(&x_full[j % SX]), (j / SX) & 1u, 200000000ull, p.hdr, kWhereProducer);
+    }
+  } else if (warp == 2) {
+    // ---------------- B producer: centre k-blocks (hi, lo) ----------------
+    if (lane == 0) {
+      const uint64_t pol = l2_policy_evict_last();
+      uint32_t i = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+        for (int kb = 0; kb < p.num_kb; ++kb, ++i) {
+          const int s = i % SB;
+          if (!mbar_wait_bounded(smem_u32(&b_empty[s]), ((i / SB) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereProducer)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&b_full[s]);
+          mbar_arrive_expect_tx(fb, p.b_stage_bytes);
+          const uint32_t st = bring + (uint32_t)s * p.b_stage_bytes;
+          tma_load_2d(st, &tmB0, fb, kb * kBK, 0, pol);
+          tma_load_2d(st + p.b_bytes, &tmB1, fb, kb * kBK, 0, pol);
+        }
+      }
+      if (!ok)
+        for (uint32_t j = (i > (uint32_t)SB ? i - SB : 0); j < i; ++j)
+          mbar_wait_bounded(smem_u32(&b_full[j % SB]), (j / SB) & 1u, 200000000ull, p.hdr, kWhereProducer);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kBM, (uint32_t)p.BN);
+      uint32_t i = 0, acc_it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++acc_it) {
+        const uint32_t a = acc_it % (uint32_t)nbuf;
+        if (!mbar_wait_bounded(smem_u32(&tempty[a]), ((acc_it / (uint32_t)nbuf) & 1u) ^ 1u, p.limit_ns, p.hdr,
+                               kWhereMmaAcc)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dt = tmem_base + a * p.acc_stride;
+        for (int kb = 0; kb < p.num_kb; ++kb, ++i) {
+          const int t = i % ST, sb = i % SB;
+          if (!mbar_wait_bounded(smem_u32(&a_full[t]), (i / ST) & 1u, p.limit_ns, p.hdr, kWhereMma) ||
+              !mbar_wait_bounded(smem_u32(&b_full[sb]), (i / SB) & 1u, p.limit_ns, p.hdr, kWhereMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t at = tmem_base + p.a_col0 + (uint32_t)t * 64u;
+          const uint32_t bst = bring + (uint32_t)sb * p.b_stage_bytes;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            const uint64_t bd0 = smem_desc_sw128(bst + k * 32);
+            const uint64_t bd1 = smem_desc_sw128(bst + p.b_bytes + k * 32);
+            tc_mma_bf16_ts(dt, at + 8u * k, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);  // xh . ch
+            tc_mma_bf16_ts(dt, at + 8u * k, bd1, idesc, 1u);                           // xh . cl
+            tc_mma_bf16_ts(dt, at + 32u + 8u * k, bd0, idesc, 1u);                     // xl . ch
+          }
+          tc_commit(smem_u32(&a_empty[t]));
+          tc_commit(smem_u32(&b_empty[sb]));
+        }
+        if (ok) tc_commit(smem_u32(&tfull[a]));
+      }
+    }
+  } else if (warp < kEpiFirst) {
+    // ---------------- converters: fp32 rows -> bf16 hi/lo in TMEM ----------------
+    const int q = warp & 3;
+    const uint32_t half = (uint32_t)((warp - kConvFirst) >> 2);  // k-blocks i with i % 2 == half
+    const int r = q * 32 + lane;  // row within the tile = TMEM lane
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint32_t i = 0, tile_it = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+      float xs = 0.0f;  // ||xh + xl||^2 of this row over this warp's k-blocks
+      for (int kb = 0; kb < p.num_kb; ++kb, ++i) {
+        if ((i & 1u) != half) continue;
+        const int s = i % SX, t = i % ST;
+        if (!mbar_wait_bounded(smem_u32(&x_full[s]), (i / SX) & 1u, p.limit_ns, p.hdr, kWhereConv) ||
+            !mbar_wait_bounded(smem_u32(&a_empty[t]), ((i / ST) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereConv)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        uint32_t hi[32], lo[32];
+        const uint32_t rowaddr = xring + (uint32_t)s * kXStage + (uint32_t)r * 128u;
+#pragma unroll
+        for (int box = 0; box < 2; ++box) {
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const float4 v = ld_shared_f4(rowaddr + (uint32_t)box * kXBox + ((uint32_t)(c ^ (r & 7)) << 4));
+            const float xv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const float x0 = xv[2 * h], x1 = xv[2 * h + 1];
+              const uint32_t hp = pack_bf16x2(x0, x1);
+              const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xFFFF0000u);
+              const uint32_t lp = pack_bf16x2(x0 - h0, x1 - h1);
+              const float l0 = __uint_as_float(lp << 16), l1 = __uint_as_float(lp & 0xFFFF0000u);
+              const float e0 = h0 + l0, e1 = h1 + l1;  // exact in fp32
+              xs = fmaf(e0, e0, xs);
+              xs = fmaf(e1, e1, xs);
+              hi[box * 16 + 2 * c + h] = hp;
+              lo[box * 16 + 2 * c + h] = lp;
+            }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&x_empty[s]));  // the fp32 stage may be refilled
+        const uint32_t at = tmem_base + lane_off + p.a_col0 + (uint32_t)t * 64u;
+        tmem_st16(at, hi);
+        tmem_st16(at + 16u, hi + 16);
+        tmem_st16(at + 32u, lo);
+        tmem_st16(at + 48u, lo + 16);
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&a_full[t]));
+      }
+      if (!ok) break;
+      const uint32_t b = tile_it & 1u;
+      if (!mbar_wait_bounded(smem_u32(&xn_empty[b]), ((tile_it >> 1) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereConv)) {
+        ok = false;
+        break;
+      }
+      xn_buf[(b * 2 + half) * kBM + r] = xs;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&xn_full[b]));
+    }
+  } else {
+    // ---------------- epilogue: argmin over the accumulator rows ----------------
+    const int q = warp & 3;
+    const int e = warp - kEpiFirst;
+    float *cb = cnbuf + e * kMaxBN;
+    for (int t = lane; t < p.BN; t += 32) cb[t] = __ldg(p.cn + t);
+    __syncwarp();
+    const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
+    const float sqrt_cn_max = sqrtf(cn_max);
+    const int r = q * 32 + lane;
+    uint32_t acc_it = 0;
+    bool ok = true;
+    double obj = 0.0;
+    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++acc_it) {
+      const uint32_t a = acc_it % (uint32_t)nbuf;
+      const uint32_t b = acc_it & 1u;
+      if (!mbar_wait_bounded(smem_u32(&tfull[a]), (acc_it / (uint32_t)nbuf) & 1u, p.limit_ns, p.hdr, kWhereEpi) ||
+          !mbar_wait_bounded(smem_u32(&xn_full[b]), (acc_it >> 1) & 1u, p.limit_ns, p.hdr, kWhereEpi)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const float xr = xn_buf[(b * 2) * kBM + r] + xn_buf[(b * 2 + 1) * kBM + r];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&xn_empty[b]));
+      float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
+      int idx1 = 0, idx2 = 0;
+      const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
+      uint32_t ra[16], rb[16];
+      tmem_ld16(taddr, ra);
+      tmem_ld_wait(ra);
+      for (int c = 0; c < p.BN; c += 32) {
+        const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+        if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
+        epilogue_group(ra, cb + c, c, best1, best2, best3, idx1, idx2);
+        if (more1) {
+          tmem_ld_wait(rb);
+          if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
+          epilogue_group(rb, cb + c + 16, c + 16, best1, best2, best3, idx1, idx2);
+          if (more2) tmem_ld_wait(ra);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
+      const int64_t row = (int64_t)tile * kBM + r;
+      if (row < p.N) obj += finish_row<false>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
@@ -799,6 +1116,23 @@ int make_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint
   return HME_OK;
 }
 
+// fp32 matrix rows x cols (row stride ld elements), box = 128 rows x 32 columns, 128-byte swizzle.
+int make_map_f32(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return fail(HME_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 4};
+  cuuint32_t box[2] = {32, (cuuint32_t)kBM};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(HME_ECUDA, "cuTensorMapEncodeTiled (fp32) failed (%d) for %llu x %llu, ld %llu", (int)r,
+                (unsigned long long)rows, (unsigned long long)cols, (unsigned long long)ld);
+  return HME_OK;
+}
+
 }  // namespace
 
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
@@ -871,6 +1205,80 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");
+  return HME_OK;
+}
+
+bool split_eligible(const void *X, int64_t ldx, const AssignGeom &g) {
+  return g.nprod == 3 && g.nchunks == 1 && (reinterpret_cast<uintptr_t>(X) & 15u) == 0 && ldx % 4 == 0;
+}
+
+int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom &g, const __nv_bfloat16 *chi,
+                        const __nv_bfloat16 *clo, const float *cn, int32_t *labels, float *mind, Header *hdr,
+                        int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
+  if (N == 0) return HME_OK;
+  CUtensorMap mX, mB0, mB1;
+  int rc;
+  if ((rc = make_map_f32(&mX, X, (uint64_t)N, (uint64_t)g.d, (uint64_t)ldx)) != HME_OK) return rc;
+  if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
+    return rc;
+  if ((rc = make_map(&mB1, clo, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
+    return rc;
+  AssignParams p{};
+  p.N = N;
+  p.num_kb = (g.d + kBK - 1) / kBK;
+  p.BN = g.BN;
+  p.nchunks = 1;
+  p.num_tiles = (int)((N + kBM - 1) / kBM);
+  p.a_bytes = 0;
+  p.b_bytes = (uint32_t)g.BN * kBK * 2;
+  p.b_stage_bytes = 2 * p.b_bytes;
+  p.a_res_bytes = 0;
+  // TMEM: accumulators (double-buffered when they fit) + 4 split A stages of 64 columns
+  uint32_t stride = 32;
+  while (stride < (uint32_t)g.BN) stride <<= 1;
+  p.acc_stride = stride;
+  p.nbuf = (2 * stride + 64u * 4u <= 512u) ? 2 : 1;
+  p.a_col0 = (uint32_t)p.nbuf * stride;
+  p.st_stages = 4;
+  p.tmem_cols = 512;
+  if (p.a_col0 + 64u * p.st_stages > 512u) return fail(HME_EINTERNAL, "assign (split): TMEM columns");
+  // shared memory: fp32 stages get what the centre stages leave
+  const size_t ctrl_bytes = 512 + (size_t)4 * kBM * sizeof(float) + (size_t)4 * kMaxBN * sizeof(float);
+  const size_t budget = 227 * 1024 - 1024 - ctrl_bytes;
+  // Both rings hide a load latency per k-block (HBM for the rows, L2 for the
+  // centres, which queues behind the same traffic): four fp32 stages, then as
+  // many centre stages as fit (at most five, at least two).
+  int sx = 4;
+  int sb = (int)((budget - (size_t)sx * kXStage) / p.b_stage_bytes);
+  if (sb > 5) sb = 5;
+  while (sb < 2 && sx > 2) {
+    --sx;
+    sb = (int)((budget - (size_t)sx * kXStage) / p.b_stage_bytes);
+    if (sb > 5) sb = 5;
+  }
+  if (sb < 2) return fail(HME_EINTERNAL, "assign (split): a centre stage of %u bytes does not fit", p.b_stage_bytes);
+  p.sb_stages = sb;
+  p.stages = sx;
+  p.xn = nullptr;
+  p.cn = cn;
+  p.labels = labels;
+  p.mind = mind;
+  p.hdr = hdr;
+  p.flagged = flagged;
+  p.full_rows = full_rows;
+  p.limit_ns = wait_limit_ns();
+  p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
+  p.err_split = 0x1p-14f;
+  p.err_ll = 0x1.1p-14f;
+  const size_t smem = 1024 + (size_t)sx * kXStage + (size_t)p.sb_stages * p.b_stage_bytes + ctrl_bytes;
+  int grid = num_sms();
+  if (grid > p.num_tiles) grid = p.num_tiles;
+  cudaError_t e = cudaFuncSetAttribute(assign_split_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "assign (split): set smem");
+  assign_split_kernel<<<grid, kSplitThreads, smem, s>>>(mX, mB0, mB1, p);
+  count_launch();
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "assign (split) kernel launch");
   return HME_OK;
 }
 

@@ -121,6 +121,11 @@ def hme_sync_status(ws: torch.Tensor, stream=None) -> int:
     return int(lib().hme_sync_status(_ptr(ws), _stream(stream)))
 
 
+def hme_last_error() -> str:
+    """The message of the last failed call on this thread."""
+    return lib().hme_last_error().decode(errors="replace")
+
+
 def hme_kmeans_init(X: torch.Tensor, K: int, seed: int, method: int, C_out: torch.Tensor, ws: torch.Tensor,
                     stream=None):
     N, d, ldx, dt = _features(X)

@@ -96,12 +96,35 @@ def test_assign_parity(dev, N, d, K, dtype, ld):
     assert st["mismatches"] <= st["near_ties"]
 
 
-def test_assign_prepared_equals_unprepared(dev):
-    X = _mixture(2000, 256, 32, "f32", seed=5)
-    C = hme_synth.random_centroids(32, 256, seed=9, scale=3.0)
+@pytest.mark.parametrize("dtype,d,K", [("bf16", 256, 32), ("f32", 130, 300)])
+def test_assign_prepared_equals_unprepared(dev, dtype, d, K):
+    """Where both calls run the same kernel (bf16 features; fp32 with several
+    N-chunks), HME_ASSIGN_PREPARED changes nothing: bit-identical results."""
+    X = _mixture(2000, d, 32, dtype, seed=5)
+    C = hme_synth.random_centroids(K, d, seed=9, scale=3.0)
     a = _assign(X, C, dev, prepared=False)
     b = _assign(X, C, dev, prepared=True)
     assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1]) and a[2] == b[2]
+
+
+@pytest.mark.parametrize("N,d,K", [(2000, 256, 32), (1001, 36, 7), (513, 2048, 64), (300, 100, 256)])
+def test_assign_split_in_kernel_and_prepared_agree(dev, N, d, K):
+    """fp32 features, K <= 256: the unprepared call splits rows inside the kernel,
+    the prepared one reads the prepared split.  Both meet the oracle's bar; their
+    labels agree outside near ties."""
+    X = _mixture(N, d, min(K, 32), "f32", seed=N + d)
+    C = hme_synth.random_centroids(K, d, seed=9, scale=3.0)
+    C[: K // 2] = X[: K // 2].float()
+    Xh = _host(X, "f32")
+    ref = oracle.assign(Xh, C.numpy(), "f32")
+    a = _assign(X, C, dev, prepared=False)
+    b = _assign(X, C, dev, prepared=True)
+    sa = parity.check_assign(Xh, "f32", C.numpy(), a[0], a[1], a[2], ref=ref)
+    sb = parity.check_assign(Xh, "f32", C.numpy(), b[0], b[1], b[2], ref=ref)
+    assert sa["mismatches"] <= sa["near_ties"] and sb["mismatches"] <= sb["near_ties"]
+    gap = (ref[2] - ref[1]) / np.maximum(ref[2], 1e-30)
+    differ = np.nonzero(a[0] != b[0])[0]
+    assert np.all(gap[differ] < parity.ASSIGN_GAP)
 
 
 def test_assign_duplicate_centres_and_zero_rows(dev):
