@@ -16,6 +16,7 @@ row sample of the same workload, scaled to the full N.
 from __future__ import annotations
 
 import argparse
+import datetime
 import hashlib
 import json
 import os
@@ -71,15 +72,18 @@ def profiled_traffic(kernel_file: str, key: str):
 
 
 class Clocks:
-    """nvidia-smi sampling of SM clock and throttle reasons during the timed region."""
+    """nvidia-smi sampling of SM clock and throttle reasons.  Sampling starts
+    before the warm-up (the tool takes a moment to come up) and only samples
+    stamped inside the timed region [begin(), end()] are kept."""
 
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
-         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-         "clocks_event_reasons.sw_power_cap")
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, index: int):
         self.index = index
         self.proc = None
+        self.t0 = self.t1 = None
         self.path = os.path.join(ROOT, "gpurun_out", f"clocks_bench_{os.getpid()}.csv")
 
     def start(self):
@@ -87,10 +91,16 @@ class Clocks:
             os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "25"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
+
+    def begin(self):
+        self.t0 = time.time()
+
+    def end(self):
+        self.t1 = time.time()
 
     def stop(self):
         if self.proc is None:
@@ -105,18 +115,22 @@ class Clocks:
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
+            if len(parts) < 10:
                 continue
             try:
-                sm.append(float(parts[1]))
-                smax.append(float(parts[2]))
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                clk, clkmax = float(parts[2]), float(parts[3])
             except ValueError:
                 continue
-            for n, v in zip(names, parts[5:9]):
+            if self.t0 is not None and not (self.t0 - 0.03 <= ts <= (self.t1 or ts) + 0.03):
+                continue
+            sm.append(clk)
+            smax.append(clkmax)
+            for n, v in zip(names, parts[6:10]):
                 if v.lower() == "active":
                     reasons.add(n)
         if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples in the timed region"]}
         sm.sort()
         return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(smax), "reasons": sorted(reasons),
                 "samples": len(sm)}
@@ -255,17 +269,18 @@ def run_ours(args, w):
         # route the training set with the final centres, reusing its prepared features
         hme.hme_route(Xs, C, expert, offsets, order, ws, flags=hme.HME_ASSIGN_PREPARED)
 
+    clocks = Clocks(local)
+    clocks.start()
     for _ in range(max(3, args.warmup)):
         step(X)
     status = hme.hme_sync_status(ws)
     if status != hme.HME_OK:
         raise RuntimeError(f"device status {status} after warm-up: {hme.hme_last_error()}")
 
-    clocks = Clocks(local)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    clocks.start()
+    clocks.begin()
     launches0 = hme.hme_launch_count()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
@@ -274,6 +289,7 @@ def run_ours(args, w):
         step(X, record=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
+    clocks.end()
     launches = hme.hme_launch_count() - launches0
     ck = clocks.stop()
     hdr = ws[:16].view(torch.int32).cpu()  # queues of the last assign (the route's): pairs, all-K
