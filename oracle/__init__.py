@@ -74,6 +74,8 @@ def _load():
         lib.orc_update.argtypes = [p, i64, i64, i64, i32, p, p, i64, p, p, p]
         lib.orc_partition.restype = i32
         lib.orc_partition.argtypes = [p, i64, i64, p, p, p, p, p, p, p, p]
+        lib.orc_tag_cluster_hist.restype = i32
+        lib.orc_tag_cluster_hist.argtypes = [p, i64, i64, p, p, i64, p, p]
         lib.orc_lloyd.restype = i32
         lib.orc_lloyd.argtypes = [p, i64, i64, i64, i32, p, i64, i64, p, p, p, p]
         _lib = lib
@@ -201,6 +203,26 @@ def partition(labels, K: int, tag_off=None, tags=None):
         out["tag_off"] = too
         out["tags"] = tgo[: tg.shape[0]]
     return out
+
+
+def tag_cluster_hist(labels, K: int, tag_off, tags, V: int):
+    """Section 4.5 tag statistics of a clustering: (counts i64[K, V], sparsity f64[V]).
+
+    counts[k, t] = occurrences of tag t among the tags of the points in cluster k;
+    sparsity[t] = ||counts[:, t]||_1 / ||counts[:, t]||_2, 0 for an absent tag.
+    """
+    labels = np.ascontiguousarray(labels, np.int32)
+    N = labels.shape[0]
+    to = np.ascontiguousarray(tag_off, np.int64)
+    tg = np.ascontiguousarray(tags, np.int32)
+    if tg.shape[0] == 0:
+        tg = np.zeros(1, np.int32)
+    counts = np.zeros((K, V), np.int64)
+    sp = np.zeros(V, np.float64)
+    rc = _load().orc_tag_cluster_hist(_ptr(labels), N, K, _ptr(to), _ptr(tg), V, _ptr(counts), _ptr(sp))
+    if rc != 0:
+        raise ValueError("orc_tag_cluster_hist: label or tag out of range")
+    return counts, sp
 
 
 def lloyd(X, C0, T: int, dtype: str = "f32"):

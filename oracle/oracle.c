@@ -409,6 +409,47 @@ int orc_partition(const int32_t *labels, int64_t N, int64_t K,
 }
 
 /* ---------------------------------------------------------------------- */
+/* Tag statistics of a clustering (Section 4.5, "Analysis of YFCC100M       */
+/* clusters"): counts[k * V + t] = number of times tag t occurs among the   */
+/* tags of the points assigned to cluster k (the bars of the tag-over-      */
+/* cluster histograms), and for every tag the sparsity of its distribution  */
+/* over clusters c(t) = counts[., t]: ||c(t)||_1 / ||c(t)||_2 (the x axis of */
+/* the sparsity-versus-accuracy figure); 0 for a tag that never occurs.     */
+/* Straight from the definition: every point, every one of its tags.        */
+/* Returns -1 on a label outside [0, K) or a tag outside [0, V).            */
+/* ---------------------------------------------------------------------- */
+int orc_tag_cluster_hist(const int32_t *labels, int64_t N, int64_t K,
+                         const int64_t *tag_off, const int32_t *tags, int64_t V,
+                         int64_t *counts, double *sparsity)
+{
+    for (int64_t i = 0; i < K * V; ++i)
+        counts[i] = 0;
+    for (int64_t i = 0; i < N; ++i) {
+        int32_t k = labels[i];
+        if (k < 0 || k >= K)
+            return -1;
+        for (int64_t j = tag_off[i]; j < tag_off[i + 1]; ++j) {
+            int32_t t = tags[j];
+            if (t < 0 || t >= V)
+                return -1;
+            counts[(int64_t)k * V + t] += 1;
+        }
+    }
+    if (sparsity) {
+        for (int64_t t = 0; t < V; ++t) {
+            double l1 = 0.0, l2sq = 0.0;
+            for (int64_t k = 0; k < K; ++k) {
+                double c = (double)counts[k * V + t];
+                l1 += c;
+                l2sq += c * c;
+            }
+            sparsity[t] = l1 > 0.0 ? l1 / sqrt(l2sq) : 0.0;
+        }
+    }
+    return 0;
+}
+
+/* ---------------------------------------------------------------------- */
 /* Lloyd's iteration, free running: T times { assign; update }, the gater's */
 /* single round of K-means (Section 3 contrasts it with alternating rounds). */
 /* objectives[t] = J of the assign step of iteration t; changed[t] = labels  */

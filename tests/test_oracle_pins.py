@@ -401,3 +401,85 @@ def test_partition_rejects_bad_labels():
 def test_empty_input():
     out = oracle.partition(np.zeros(0, np.int32), 4)
     assert out["hist"].tolist() == [0, 0, 0, 0] and out["offsets"].tolist() == [0] * 5
+
+
+# ---------------------------------------------------------------------------
+# Tag statistics of a clustering (Section 4.5)
+# ---------------------------------------------------------------------------
+TAG_CASES = json.load(open(os.path.join(GOLDEN, "tag_cluster_hand_examples.json")))["cases"]
+
+
+@pytest.mark.parametrize("case", TAG_CASES, ids=lambda c: c["name"])
+def test_tag_hist_hand_examples(case):
+    counts, sp = oracle.tag_cluster_hist(np.array(case["labels"], np.int32), case["K"],
+                                         np.array(case["tag_off"], np.int64), np.array(case["tags"], np.int32),
+                                         case["V"])
+    assert np.array_equal(counts, np.array(case["counts"], np.int64))
+    assert np.allclose(sp, case["sparsity"], rtol=1e-15, atol=0)
+
+
+def _random_tagged(N, K, V, seed):
+    rng = np.random.default_rng(seed)
+    labels = rng.integers(0, K, N).astype(np.int32)
+    lens = rng.poisson(3.0, N)
+    tag_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    # Zipf-like vocabulary: a few tags very common
+    w = 1.0 / np.arange(1, V + 1)
+    tags = rng.choice(V, int(tag_off[-1]), p=w / w.sum()).astype(np.int32)
+    return labels, tag_off, tags
+
+
+def test_tag_hist_marginals():
+    """Row sums = tags carried by each cluster's points; column sums = occurrences of each tag."""
+    N, K, V = 3000, 17, 200
+    labels, tag_off, tags = _random_tagged(N, K, V, 3)
+    counts, sp = oracle.tag_cluster_hist(labels, K, tag_off, tags, V)
+    lens = np.diff(tag_off)
+    per_cluster = np.array([lens[labels == k].sum() for k in range(K)])
+    assert np.array_equal(counts.sum(1), per_cluster)
+    assert np.array_equal(counts.sum(0), np.bincount(tags, minlength=V))
+    present = counts.sum(0) > 0
+    assert np.all(sp[~present] == 0.0)
+    # ||c||_1 / ||c||_2 lies in [1, sqrt(number of clusters the tag occurs in)]
+    nz = (counts > 0).sum(0)
+    assert np.all(sp[present] >= 1.0 - 1e-12)
+    assert np.all(sp[present] <= np.sqrt(nz[present]) + 1e-12)
+
+
+def test_tag_hist_closed_forms():
+    """A tag confined to one cluster has sparsity 1; equal counts over m clusters give sqrt(m)."""
+    K, V = 9, 4
+    labels, offs, tags = [], [0], []
+    for k in range(K):
+        for _ in range(5):  # five points per cluster
+            labels.append(k)
+            t = [0] if k < 6 else []          # tag 0: once per point in clusters 0..5 -> m = 6
+            t += [1, 1] if k == 4 else []     # tag 1: only in cluster 4
+            t += [3] * (k + 1)                # tag 3: counts 5 (k + 1) per cluster, unequal
+            tags += t
+            offs.append(offs[-1] + len(t))
+    counts, sp = oracle.tag_cluster_hist(np.array(labels, np.int32), K, np.array(offs, np.int64),
+                                         np.array(tags, np.int32), V)
+    assert sp[0] == pytest.approx(np.sqrt(6.0), rel=1e-15)
+    assert sp[1] == 1.0
+    assert sp[2] == 0.0
+    c3 = 5.0 * np.arange(1, K + 1)
+    assert sp[3] == pytest.approx(c3.sum() / np.sqrt((c3 ** 2).sum()), rel=1e-15)
+
+
+def test_tag_hist_invariant_under_point_order():
+    """The statistics depend on (label, tags) pairs only: the partitioned order gives the same result."""
+    N, K, V = 2000, 11, 150
+    labels, tag_off, tags = _random_tagged(N, K, V, 8)
+    counts, sp = oracle.tag_cluster_hist(labels, K, tag_off, tags, V)
+    part = oracle.partition(labels, K, tag_off, tags)
+    counts2, sp2 = oracle.tag_cluster_hist(part["sorted_labels"], K, part["tag_off"], part["tags"], V)
+    assert np.array_equal(counts, counts2)
+    assert np.array_equal(sp, sp2)
+
+
+def test_tag_hist_rejects_out_of_range():
+    with pytest.raises(ValueError):
+        oracle.tag_cluster_hist(np.array([0, 3], np.int32), 3, np.array([0, 1, 2]), np.array([0, 1], np.int32), 2)
+    with pytest.raises(ValueError):
+        oracle.tag_cluster_hist(np.array([0, 1], np.int32), 3, np.array([0, 1, 2]), np.array([0, 2], np.int32), 2)
