@@ -242,6 +242,17 @@ def run_ours(args, w):
     offsets = torch.empty(K + 1, dtype=torch.int64, device=dev)
     order = torch.empty(N, dtype=torch.int32, device=dev)
 
+    # multilabel workloads: the final expert shares carry each point's tag list
+    tag_off = tags = None
+    if w.tags:
+        tag_off, tags = hme_synth.make_tags(w, device=dev)
+        wp = hme.workspace(hme.HME_OP_PARTITION, N, 1, K, dt, device=dev)
+        p_hist = torch.empty(K, dtype=torch.int64, device=dev)
+        p_offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+        p_perm = torch.empty(N, dtype=torch.int32, device=dev)
+        tag_off_out = torch.empty_like(tag_off)
+        tags_out = torch.empty_like(tags)
+
     ev_assign, ev_update = [], []
     moved_dev = torch.zeros(1, dtype=torch.int32, device=dev)
 
@@ -268,6 +279,8 @@ def run_ours(args, w):
                 ev_update.append((t, a1, u1))
         # route the training set with the final centres, reusing its prepared features
         hme.hme_route(Xs, C, expert, offsets, order, ws, flags=hme.HME_ASSIGN_PREPARED)
+        if w.tags:  # the experts' shares with their tag lists
+            hme.hme_partition(expert, K, p_hist, p_offs, p_perm, wp, None, tag_off, tags, tag_off_out, tags_out)
 
     clocks = Clocks(local)
     clocks.start()
@@ -315,6 +328,26 @@ def run_ours(args, w):
     status = hme.hme_sync_status(ws)
     if status != hme.HME_OK:
         raise RuntimeError(f"device status {status} after the route comparison: {hme.hme_last_error()}")
+    tag_stats = None
+    if w.tags:  # Section 4.5 statistics of the final shares, outside the timed steps
+        V = w.tag_vocab
+        wt = hme.workspace(hme.HME_OP_TAG_HIST, N, V, K, dt, device=dev)
+        tcounts = torch.empty(K, V, dtype=torch.int64, device=dev)
+        tsp = torch.empty(V, dtype=torch.float64, device=dev)
+        hme.hme_tag_cluster_hist(p_offs, tag_off_out, tags_out, K, V, tcounts, wt, tsp)  # warm-up
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        hme.hme_tag_cluster_hist(p_offs, tag_off_out, tags_out, K, V, tcounts, wt, tsp)
+        t1.record(stream)
+        torch.cuda.synchronize(dev)
+        if hme.hme_sync_status(wt) != hme.HME_OK:
+            raise RuntimeError(f"tag statistics: {hme.hme_last_error()}")
+        t_ms = t0.elapsed_time(t1)
+        T_tags = tags.numel()
+        nbytes = 4 * T_tags + 8 * (N + 1) + 8 * (K + 1) + 8 * K * V * 2 + 8 * V  # tags, offsets in; counts out, read back
+        tag_stats = {"ms": t_ms, "tags": T_tags, "vocabulary": V, "gbs": nbytes / (t_ms / 1000) / 1e9,
+                     "tags_per_s": T_tags / (t_ms / 1000)}
 
     iters_total = T * args.steps * world
     value = iters_total / (ms / 1000.0)
@@ -389,7 +422,8 @@ def run_ours(args, w):
             "data": "synthetic",
             "config": {"workload": w.name, "N": N, "d": d, "K": K, "feature_dtype": w.dtype, "iterations": T,
                        "step": "prepare + %d x (assign + update; updates after the first read only rows whose label changed)"
-                    " + route of all N rows" % T,
+                    " + route of all N rows" % T + (" + partition of the routed rows with their tag lists"
+                                                      if w.tags else ""),
                        "l2": "inputs larger than L2 (%.1f GB of features)" % (X.numel() * e / 1e9),
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "vectors_per_s": N * iters_total / (ms / 1000.0),
@@ -403,6 +437,7 @@ def run_ours(args, w):
             "gpu_launches": launches,
             "rescored_rows_last_assign": rescored,
             "moved_rows_last_update": moved,
+            "tag_statistics": tag_stats,
             "clocks": ck,
         }
         print(json.dumps(line), flush=True)

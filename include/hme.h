@@ -67,6 +67,7 @@ extern "C" {
 #define HME_OP_ASSIGN 1    /* hme_prepare_features, hme_assign, hme_update_centroids */
 #define HME_OP_PARTITION 2 /* hme_partition (d and dtype ignored) */
 #define HME_OP_ROUTE 3     /* hme_route */
+#define HME_OP_TAG_HIST 4  /* hme_tag_cluster_hist (d = vocabulary size V; dtype ignored) */
 
 /* ---- k-means++ seeding variants -------------------------------------- */
 #define HME_INIT_KMEANSPP 0           /* candidates = all N rows */
@@ -226,6 +227,28 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
 HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
                       int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,
                       size_t ws_bytes, void *stream);
+
+/*
+ * hme_tag_cluster_hist -- the tag statistics of a clustering that Section 4.5
+ * ("Analysis of YFCC100M clusters") reports: for every cluster k and tag t
+ *   counts_out[k * V + t] = the number of times t occurs among the tags of the
+ *                           points of cluster k (int64, K x V row-major: the
+ *                           bars of the tag-over-cluster histograms),
+ * and for every tag, with c(t) = counts[:, t] its distribution over clusters,
+ *   sparsity_out[t] = ||c(t)||_1 / ||c(t)||_2 in fp64 (between 1 and
+ *                     sqrt(K); 0 for a tag that never occurs)    (may be NULL).
+ * Input is the partitioned form that hme_partition writes: offsets: int64[K+1]
+ * point offsets of the clusters (offsets_out); tag_off: int64[N+1] and tags:
+ * int32[tag_off[N]], the tag lists in that point order (tag_off_out,
+ * tags_out), so each cluster's tags are one contiguous range.  Tags outside
+ * [0, V) are skipped and reported by hme_sync_status (HME_EINVAL).  Integer
+ * counts are exact; the ratio is the fp64 one of those counts.
+ * ws: hme_workspace_bytes(HME_OP_TAG_HIST, N, V, K, 0) bytes.  All pointers
+ * are device memory; asynchronous on stream.
+ */
+HME_API int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int64_t N,
+                                 int32_t K, int32_t V, int64_t *counts_out, double *sparsity_out, void *ws,
+                                 size_t ws_bytes, void *stream);
 
 /*
  * hme_partition_noalloc -- the same stable partition as hme_partition (same

@@ -18,7 +18,8 @@ CSRC = os.path.join(PKG, "csrc")
 LIBDIR = os.path.join(PKG, "lib")
 OBJDIR = os.path.join(LIBDIR, "obj")
 LIB = os.path.join(LIBDIR, "libhme.so")
-SOURCES = ["api.cu", "prep.cu", "assign.cu", "update.cu", "partition.cu", "init.cu", "partition_static.cu"]
+SOURCES = ["api.cu", "prep.cu", "assign.cu", "update.cu", "partition.cu", "init.cu", "partition_static.cu",
+           "tags.cu"]
 HEADERS = ["hme_common.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

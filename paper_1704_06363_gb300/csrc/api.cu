@@ -255,6 +255,10 @@ size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t 
     if (N < 0 || N > (int64_t)0x7FFFFFFF || K < 1 || K > kMaxK) return 0;
     return align_up(part_layout(sizeof(Header), N, K).end, 256);
   }
+  if (op == HME_OP_TAG_HIST) {  // d is the vocabulary size V
+    if (N < 0 || K < 1 || K > kMaxK || d < 1) return 0;
+    return align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256);
+  }
   if (check_common(N, d, K, dtype) != HME_OK) return 0;
   switch (op) {
     case HME_OP_INIT:
@@ -281,6 +285,8 @@ int hme_sync_status(void *ws, void *stream) {
   if (h.status & kStatusTimeout)
     return fail(HME_ETIMEOUT, "a bounded device wait expired (site %u)", h.wait_where);
   if (h.status & kStatusBadLabel) return fail(HME_EINVAL, "a label outside [0, K) was skipped");
+  if (h.status & kStatusBadTag)
+    return fail(HME_EINVAL, "a tag outside [0, V) was skipped, or a cluster's tag range was inverted");
   return HME_OK;
 }
 
@@ -415,6 +421,24 @@ int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, c
   HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
                             offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
            "route: partition");
+  return HME_OK;
+}
+
+int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int64_t N, int32_t K,
+                         int32_t V, int64_t *counts_out, double *sparsity_out, void *ws, size_t ws_bytes,
+                         void *stream) {
+  if (N < 0 || N > (int64_t)0x7FFFFFFF) return fail(HME_EINVAL, "N = %lld out of range", (long long)N);
+  if (K < 1 || K > kMaxK) return fail(HME_EINVAL, "K = %d out of range [1, %d]", K, kMaxK);
+  if (V < 1) return fail(HME_EINVAL, "V = %d must be positive", V);
+  if (!offsets || !tag_off || !counts_out) return fail(HME_EINVAL, "offsets / tag_off / counts_out is NULL");
+  if (!tags && N > 0) return fail(HME_EINVAL, "tags is NULL");
+  const size_t need = align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256);
+  HME_TRY(check_ws(ws, ws_bytes, need));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  HME_CUDA(launch_tag_hist(offsets, tag_off, tags, K, V, at<int64_t>(ws, sizeof(Header)), counts_out, sparsity_out,
+                           at<Header>(ws, 0), s),
+           "tag statistics");
   return HME_OK;
 }
 

@@ -18,7 +18,7 @@ import torch
 
 HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6)
 HME_F32, HME_BF16 = 0, 1
-HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE = range(4)
+HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST = range(5)
 HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
 HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED = 0, 1
 
@@ -65,6 +65,8 @@ def lib():
         L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
         L.hme_partition_noalloc.restype = ctypes.c_int
         L.hme_partition_noalloc.argtypes = [p, i64, i32, p, p, p, p, p, p]
+        L.hme_tag_cluster_hist.restype = ctypes.c_int
+        L.hme_tag_cluster_hist.argtypes = [p, p, p, i64, i32, i32, p, p, p, sz, p]
         L.hme_launch_count.restype = i64
         L.hme_launch_count.argtypes = []
         L.hme_debug_bounded_wait.restype = ctypes.c_int
@@ -183,6 +185,16 @@ def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offset
     w, wb = _ws(ws)
     _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, flags, _ptr(expert_out), _ptr(offsets_out),
                            _ptr(order_out), w, wb, _stream(stream)), "hme_route")
+
+
+def hme_tag_cluster_hist(offsets: torch.Tensor, tag_off: torch.Tensor, tags: torch.Tensor, K: int, V: int,
+                         counts_out: torch.Tensor, ws: torch.Tensor, sparsity_out: Optional[torch.Tensor] = None,
+                         stream=None):
+    """Section 4.5 tag statistics from hme_partition's outputs: counts_out[K, V] int64, sparsity_out[V] fp64."""
+    N = tag_off.shape[0] - 1
+    w, wb = _ws(ws)
+    _check(lib().hme_tag_cluster_hist(_ptr(offsets), _ptr(tag_off), _ptr(tags), N, K, V, _ptr(counts_out),
+                                      _ptr(sparsity_out), w, wb, _stream(stream)), "hme_tag_cluster_hist")
 
 
 def hme_partition_noalloc(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_out: torch.Tensor,

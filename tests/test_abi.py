@@ -87,3 +87,20 @@ def test_product_path_has_no_oracle_import():
             if fn.endswith((".py", ".cu", ".cuh", ".h")):
                 text = open(os.path.join(dirpath, fn)).read()
                 assert "import oracle" not in text and "from oracle" not in text and "liboracle" not in text, fn
+
+
+def test_tag_hist_host_validation(lib):
+    f = lib.hme_workspace_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    assert f(4, 16_000_000, 20_000, 1024, 0) >= 256 + 1025 * 8  # op 4: d is the vocabulary size
+    assert f(4, 10, 0, 4, 0) == 0  # V = 0 rejected
+    g = lib.hme_tag_cluster_hist
+    g.restype = ctypes.c_int
+    p, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    g.argtypes = [p, p, p, i64, i32, i32, p, p, p, ctypes.c_size_t, p]
+    ok = [p(256), p(256), p(256), 10, 4, 100, p(256), None, p(256), 1 << 20, None]
+    for i, bad in [(4, 0), (5, 0), (6, None), (0, None), (9, 8)]:  # K = 0, V = 0, no counts, no offsets, tiny ws
+        args = list(ok)
+        args[i] = bad
+        assert g(*args) != 0
