@@ -238,6 +238,13 @@ int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, con
   return HME_OK;
 }
 
+// hme_tag_cluster_hist: header, chunk table int64[K + 1], per-slice column sums double[kTagSlices][2 V]
+size_t tag_ws_bytes(int K, int V) {
+  return align_up(align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256) +
+                      (size_t)kTagSlices * 2 * V * sizeof(double),
+                  256);
+}
+
 int clear_header(void *ws, cudaStream_t s) {
   HME_CUDA(cudaMemsetAsync(ws, 0, sizeof(Header), s), "clear workspace header");
   return HME_OK;
@@ -257,7 +264,7 @@ size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t 
   }
   if (op == HME_OP_TAG_HIST) {  // d is the vocabulary size V
     if (N < 0 || K < 1 || K > kMaxK || d < 1) return 0;
-    return align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256);
+    return tag_ws_bytes(K, d);
   }
   if (check_common(N, d, K, dtype) != HME_OK) return 0;
   switch (op) {
@@ -432,12 +439,12 @@ int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const i
   if (V < 1) return fail(HME_EINVAL, "V = %d must be positive", V);
   if (!offsets || !tag_off || !counts_out) return fail(HME_EINVAL, "offsets / tag_off / counts_out is NULL");
   if (!tags && N > 0) return fail(HME_EINVAL, "tags is NULL");
-  const size_t need = align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256);
-  HME_TRY(check_ws(ws, ws_bytes, need));
+  HME_TRY(check_ws(ws, ws_bytes, tag_ws_bytes(K, V)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_CUDA(launch_tag_hist(offsets, tag_off, tags, K, V, at<int64_t>(ws, sizeof(Header)), counts_out, sparsity_out,
-                           at<Header>(ws, 0), s),
+  const size_t sums_at = align_up(sizeof(Header) + (size_t)(K + 1) * sizeof(int64_t), 256);
+  HME_CUDA(launch_tag_hist(offsets, tag_off, tags, K, V, at<int64_t>(ws, sizeof(Header)), at<double>(ws, sums_at),
+                           counts_out, sparsity_out, at<Header>(ws, 0), s),
            "tag statistics");
   return HME_OK;
 }

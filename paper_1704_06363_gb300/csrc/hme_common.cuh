@@ -154,9 +154,12 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
 cudaError_t launch_kmeanspp(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, uint64_t seed,
                             int64_t m, bool subsample, float *C_out, int32_t *rows, double *d2, double *part,
                             Header *hdr, cudaStream_t s);
-// Tag statistics of a clustering (tags.cu); chunk_start: int64[K + 1] scratch.
+// Tag statistics of a clustering (tags.cu); scratch: chunk_start int64[K + 1],
+// colsums double[kTagSlices * 2 V].
+constexpr int kTagSlices = 16;
 cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int K, int V,
-                            int64_t *chunk_start, int64_t *counts, double *sparsity, Header *hdr, cudaStream_t s);
+                            int64_t *chunk_start, double *colsums, int64_t *counts, double *sparsity, Header *hdr,
+                            cudaStream_t s);
 cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
 int64_t kpp_candidates(int64_t N, int K, int method);
 constexpr int kMaxSms = 256;  // bound used to size the re-seed candidate region

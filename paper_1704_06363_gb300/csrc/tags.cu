@@ -14,16 +14,16 @@
 //   tag_zero      rows of clusters with several chunks start at zero (they are
 //                 accumulated with atomics);
 //   tag_hist      persistent blocks over the chunks: a shared-memory histogram
-//                 of the V tag ids (equal ids of a warp add once, with
-//                 __match_any_sync), then the row of counts goes out with
+//                 of the V tag ids in 16-bit fields (one shared atomic per
+//                 tag), then the row of counts goes out with
 //                 plain stores when the cluster is one chunk, or 64-bit
 //                 atomics of the non-zero bins otherwise.  A vocabulary
 //                 too large for shared memory counts straight into the
-//                 (zeroed) global rows with the same warp aggregation;
-//   tag_sparsity  a block per 32 tags, its warps splitting the clusters
-//                 (reads coalesced over tags): l1 and sum of squares in fp64
-//                 (exact for integer counts below 2^53), ratio; 0 for absent
-//                 tags.
+//                 (zeroed) global rows with 64-bit atomics;
+//   tag_colsum    blocks of 256 tags x one of 16 slices of the clusters write
+//                 each tag's partial l1 and sum of squares (64-bit integers,
+//                 exact);
+//   tag_sparsity  adds the slices and forms the ratio; 0 for absent tags.
 // Tags outside [0, V) are skipped and set kStatusBadTag.
 #include "hme_common.cuh"
 
@@ -31,7 +31,8 @@ namespace hme {
 
 namespace {
 
-constexpr int64_t kTagChunk = 65536;
+// at most 65535 tags per chunk: a tag's count in a chunk fits a 16-bit field
+constexpr int64_t kTagChunk = 65535;
 constexpr int kTagThreads = 512;
 
 __global__ void __launch_bounds__(1024) tag_chunks_kernel(const int64_t *__restrict__ offsets,
@@ -103,21 +104,25 @@ __device__ __forceinline__ int chunk_cluster(const int64_t *chunk_start, int K, 
   return lo;
 }
 
+// Shared-memory counters are 16-bit fields, two per 32-bit word (tag t in
+// word t / 2, bits 16 (t % 2) ..): a chunk holds at most 65535 tags, so no
+// field carries into its neighbour, and twice as many blocks fit an SM.
 template <bool SMEM>
 __global__ void __launch_bounds__(kTagThreads) tag_hist_kernel(const int64_t *__restrict__ offsets,
                                                                const int64_t *__restrict__ tag_off,
                                                                const int32_t *__restrict__ tags, int K, int V,
                                                                const int64_t *__restrict__ chunk_start,
                                                                int64_t *counts, Header *hdr) {
-  extern __shared__ int32_t hist[];  // V counters (SMEM)
+  extern __shared__ uint32_t hist[];  // (V + 1) / 2 words (SMEM)
   __shared__ int k_s;
   const int lane = threadIdx.x & 31;
+  const int words = (V + 1) >> 1;
   const int64_t nchunks = chunk_start[K];
   bool bad = false;
   for (int64_t c = blockIdx.x; c < nchunks; c += gridDim.x) {
     if (threadIdx.x == 0) k_s = chunk_cluster(chunk_start, K, c);
     if (SMEM)
-      for (int t = threadIdx.x; t < V; t += blockDim.x) hist[t] = 0;
+      for (int w = threadIdx.x; w < words; w += blockDim.x) hist[w] = 0u;
     __syncthreads();
     const int k = k_s;
     const int64_t j = c - chunk_start[k];
@@ -126,28 +131,39 @@ __global__ void __launch_bounds__(kTagThreads) tag_hist_kernel(const int64_t *__
     const int64_t lo = a + j * kTagChunk;
     const int64_t hi = b < lo + kTagChunk ? b : lo + kTagChunk;
     int64_t *row = counts + (int64_t)k * V;
-    // whole warps step together so that __match_any_sync sees every lane
-    for (int64_t base = lo + (threadIdx.x & ~31); base < hi; base += blockDim.x) {
-      const int64_t i = base + lane;
-      const int32_t t = i < hi ? __ldg(tags + i) : -1;
-      const bool valid = i < hi && t >= 0 && t < V;
-      if (i < hi && !valid) bad = true;
-      const unsigned act = __ballot_sync(0xffffffffu, valid);
-      const unsigned peers = __match_any_sync(0xffffffffu, valid ? t : -1) & act;
-      if (valid && lane == __ffs(peers) - 1) {
+    // 4 loads per thread in flight, then one shared-memory atomic per tag
+    // (equal tags of a warp are serialised by the hardware; cheaper than
+    // grouping them first)
+    for (int64_t base = lo + threadIdx.x; base < hi; base += (int64_t)blockDim.x * 4) {
+      int32_t tv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int64_t i = base + (int64_t)u * blockDim.x;
+        tv[u] = i < hi ? __ldg(tags + i) : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int64_t i = base + (int64_t)u * blockDim.x;
+        if (i >= hi) continue;
+        const int32_t t = tv[u];
+        if (t < 0 || t >= V) {
+          bad = true;
+          continue;
+        }
         if (SMEM)
-          atomicAdd(&hist[t], (int32_t)__popc(peers));
+          atomicAdd(&hist[t >> 1], 1u << (16 * (t & 1)));
         else
-          atomicAdd(reinterpret_cast<unsigned long long *>(row + t), (unsigned long long)__popc(peers));
+          atomicAdd(reinterpret_cast<unsigned long long *>(row + t), 1ull);
       }
     }
     __syncthreads();
     if (SMEM) {
-      if (nk == 1) {
-        for (int t = threadIdx.x; t < V; t += blockDim.x) row[t] = hist[t];
-      } else {
-        for (int t = threadIdx.x; t < V; t += blockDim.x)
-          if (hist[t] != 0) atomicAdd(reinterpret_cast<unsigned long long *>(row + t), (unsigned long long)hist[t]);
+      for (int t = threadIdx.x; t < V; t += blockDim.x) {
+        const uint32_t v = (hist[t >> 1] >> (16 * (t & 1))) & 0xFFFFu;
+        if (nk == 1)
+          row[t] = v;
+        else if (v != 0)
+          atomicAdd(reinterpret_cast<unsigned long long *>(row + t), (unsigned long long)v);
       }
       __syncthreads();  // hist is cleared for the next chunk
     }
@@ -155,35 +171,42 @@ __global__ void __launch_bounds__(kTagThreads) tag_hist_kernel(const int64_t *__
   if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadTag);
 }
 
-// One block per 32 consecutive tags (lane = tag, coalesced 256-byte reads of a
-// row segment); its 8 warps take every 8th cluster and combine in shared memory.
-constexpr int kSpWarps = 8;
-
-__global__ void __launch_bounds__(32 * kSpWarps) tag_sparsity_kernel(const int64_t *__restrict__ counts, int K, int V,
-                                                                     double *sparsity) {
-  __shared__ double part[2][kSpWarps][32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int t = blockIdx.x * 32 + lane;
-  double l1 = 0.0, l2sq = 0.0;
-  if (t < V) {
+// Per-tag l1 and sum of squares over the clusters: a block takes 256
+// consecutive tags (2 KB of every row it reads, coalesced) and one of
+// kTagSlices slices of the clusters, and writes its partial sums to
+// part[slice][0 .. V) and part[slice][V .. 2V); tag_sparsity adds the slices.
+// The sums are kept in 64-bit integers (exact: a tag's squared counts add up
+// to at most (number of tags)^2 < 2^62), so no per-element fp64 arithmetic is
+// needed and the result does not depend on the order; the ratio is formed
+// once per tag in fp64.
+__global__ void __launch_bounds__(256) tag_colsum_kernel(const int64_t *__restrict__ counts, int K, int V,
+                                                         int rows_per_slice, uint64_t *part) {
+  const int t = blockIdx.x * 256 + threadIdx.x;
+  const int k0 = blockIdx.y * rows_per_slice;
+  const int k1 = min(K, k0 + rows_per_slice);
+  if (t >= V) return;
+  uint64_t l1 = 0, l2sq = 0;
 #pragma unroll 8
-    for (int k = warp; k < K; k += kSpWarps) {
-      const double c = (double)__ldg(counts + (int64_t)k * V + t);
-      l1 += c;
-      l2sq = fma(c, c, l2sq);
-    }
+  for (int k = k0; k < k1; ++k) {
+    const uint64_t c = (uint64_t)__ldg(counts + (int64_t)k * V + t);
+    l1 += c;
+    l2sq += c * c;
   }
-  part[0][warp][lane] = l1;
-  part[1][warp][lane] = l2sq;
-  __syncthreads();
-  if (warp == 0 && t < V) {
-    double a = 0.0, b = 0.0;
-    for (int w = 0; w < kSpWarps; ++w) {  // counts are integers below 2^53: every partial sum is exact
-      a += part[0][w][lane];
-      b += part[1][w][lane];
-    }
-    sparsity[t] = a > 0.0 ? a / sqrt(b) : 0.0;
+  uint64_t *dst = part + (int64_t)blockIdx.y * 2 * V;
+  dst[t] = l1;
+  dst[V + t] = l2sq;
+}
+
+__global__ void __launch_bounds__(256) tag_sparsity_kernel(const uint64_t *__restrict__ part, int V, int slices,
+                                                           double *sparsity) {
+  const int t = blockIdx.x * 256 + threadIdx.x;
+  if (t >= V) return;
+  uint64_t l1 = 0, l2sq = 0;
+  for (int sl = 0; sl < slices; ++sl) {
+    l1 += part[(int64_t)sl * 2 * V + t];
+    l2sq += part[(int64_t)sl * 2 * V + V + t];
   }
+  sparsity[t] = l1 > 0 ? (double)l1 / sqrt((double)l2sq) : 0.0;
 }
 
 }  // namespace
@@ -191,9 +214,10 @@ __global__ void __launch_bounds__(32 * kSpWarps) tag_sparsity_kernel(const int64
 size_t tag_hist_smem_limit() { return (size_t)200 * 1024; }
 
 cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int K, int V,
-                            int64_t *chunk_start, int64_t *counts, double *sparsity, Header *hdr, cudaStream_t s) {
+                            int64_t *chunk_start, double *colsums, int64_t *counts, double *sparsity, Header *hdr,
+                            cudaStream_t s) {
   tag_chunks_kernel<<<1, 1024, 0, s>>>(offsets, tag_off, K, chunk_start, hdr);
-  const size_t smem = (size_t)V * sizeof(int32_t);
+  const size_t smem = (size_t)((V + 1) / 2) * sizeof(uint32_t);
   const bool in_smem = smem <= tag_hist_smem_limit();
   const int zb = K < 1024 ? K : 1024;
   tag_zero_kernel<<<zb, 256, 0, s>>>(chunk_start, K, V, !in_smem, counts);
@@ -203,7 +227,7 @@ cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, cons
     e = cudaFuncSetAttribute(tag_hist_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int per_sm = (int)((size_t)(227 * 1024) / (smem + 1024));
-    grid *= per_sm < 1 ? 1 : (per_sm > 4 ? 4 : per_sm);
+    grid *= per_sm < 1 ? 1 : (per_sm > 8 ? 8 : per_sm);
     tag_hist_kernel<true><<<grid, kTagThreads, smem, s>>>(offsets, tag_off, tags, K, V, chunk_start, counts, hdr);
   } else {
     grid *= 4;
@@ -211,8 +235,13 @@ cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, cons
   }
   count_launch(3);
   if (sparsity) {
-    tag_sparsity_kernel<<<(V + 31) / 32, 32 * kSpWarps, 0, s>>>(counts, K, V, sparsity);
-    count_launch();
+    const int slices = K < kTagSlices ? K : kTagSlices;
+    const int rows = (K + slices - 1) / slices;
+    const dim3 cg((unsigned)((V + 255) / 256), (unsigned)slices);
+    tag_colsum_kernel<<<cg, 256, 0, s>>>(counts, K, V, rows, reinterpret_cast<uint64_t *>(colsums));
+    tag_sparsity_kernel<<<(V + 255) / 256, 256, 0, s>>>(reinterpret_cast<const uint64_t *>(colsums), V, slices,
+                                                          sparsity);
+    count_launch(2);
   }
   return cudaGetLastError();
 }

@@ -79,7 +79,7 @@ def test_tag_hist_parity(dev, N, K, V):
 
 
 def test_tag_hist_multi_chunk_and_empty_clusters(dev):
-    """One cluster carries > 2 * 65536 tags (several chunks, accumulated with atomics);
+    """One cluster carries > 2 * 65535 tags (several chunks, accumulated with atomics);
     clusters 5..9 are empty (rows of zeros)."""
     N, K, V = 4000, 10, 1000
     rng = np.random.default_rng(4)
@@ -90,13 +90,29 @@ def test_tag_hist_multi_chunk_and_empty_clusters(dev):
     assert np.all(counts[5:] == 0)
 
 
-def test_tag_hist_vocabulary_beyond_shared_memory(dev):
-    """V = 60000 counters do not fit in shared memory: global-memory counting path."""
-    N, K, V = 6000, 33, 60_000
+@pytest.mark.parametrize("V", [60_000, 120_000])
+def test_tag_hist_large_vocabularies(dev, V):
+    """V = 60000: one shared-memory histogram per SM; V = 120000 counters do not fit
+    in shared memory: the global-memory counting path."""
+    N, K = 6000, 33
     rng = np.random.default_rng(6)
     labels = rng.integers(0, K, N).astype(np.int32)
     tag_off, tags = _zipf_tags(N, V, 4.0, 6)
     _check(labels, K, tag_off, tags, V, dev)
+
+
+def test_tag_hist_one_tag_fills_a_chunk(dev):
+    """70000 copies of one tag on one point: a full chunk of 65535 equal tags (the 16-bit
+    field at its maximum) and the rest in a second chunk."""
+    N, K, V = 10, 2, 5
+    labels = np.array([0, 1] * 5, np.int32)
+    lens = np.array([1] * N, np.int64)
+    lens[3] = 70_000
+    tag_off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    tags = np.full(int(tag_off[-1]), 3, np.int32)
+    tags[: tag_off[3]] = 1
+    counts = _check(labels, K, tag_off, tags, V, dev)
+    assert counts[1, 3] == 70_000 + 3  # point 3, then points 5, 7 and 9 of cluster 1 with one tag 3 each
 
 
 def test_tag_hist_no_tags(dev):
