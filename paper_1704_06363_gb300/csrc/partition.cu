@@ -4,8 +4,7 @@
 //
 // A stable counting sort of the labels, integer-exact:
 //   1. count    each warp owns a contiguous tile of labels and counts it into
-//               private shared-memory bins (__match_any_sync groups equal
-//               labels of a 32-item round, the lowest lane adds the group);
+//               private shared-memory bins (one shared atomic per label);
 //               tile counts go to an ntiles x K int32 matrix.
 //   2. colscan  exclusive prefix of that matrix down each column (per bucket)
 //               and the bucket totals hist[k].
@@ -14,7 +13,10 @@
 //               is offsets[k] + (items of bucket k in earlier tiles) + (items
 //               of k earlier in this tile), the last part from the running
 //               shared-memory bin plus the rank among equal labels of lower
-//               lanes in the round.  So within a bucket indices ascend.
+//               lanes in the round.  So within a bucket indices ascend.  The
+//               lanes holding the same label are found with one ballot per
+//               label bit (ceil(log2 K) ballots), which is much cheaper than
+//               __match_any_sync on this hardware.
 // Labels are staged 512 at a time through a per-warp shared buffer with
 // 16-byte loads.  Labels outside [0, K) set kStatusBadLabel and are skipped.
 #include "hme_common.cuh"
@@ -45,6 +47,18 @@ __device__ __forceinline__ void stage_labels(const int32_t *__restrict__ labels,
   __syncwarp();
 }
 
+// Lanes of the warp whose key equals this lane's key (valid keys are in
+// [0, 2^nbits)); keys < 0 match no valid lane and get an empty mask.
+__device__ __forceinline__ unsigned same_key_lanes(int key, int nbits) {
+  unsigned peers = __ballot_sync(0xffffffffu, key >= 0);
+  for (int b = 0; b < nbits; ++b) {
+    const bool bit = (key >> b) & 1;
+    const unsigned m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
+  }
+  return key >= 0 ? peers : 0u;
+}
+
 __global__ void part_count_kernel(const int32_t *__restrict__ labels, int64_t N, int K, int64_t tile,
                                   int64_t ntiles, int32_t *__restrict__ tilecnt, Header *hdr, int wpb) {
   extern __shared__ int32_t psm[];
@@ -64,12 +78,9 @@ __global__ void part_count_kernel(const int32_t *__restrict__ labels, int64_t N,
     const int rounds = (int)min((int64_t)kChunk, end - pos + 31) / 32;
     for (int r = 0; r < rounds; ++r) {
       const int64_t i = pos + 32 * r + lane;
-      int key = buf[32 * r + lane];
+      const int key = buf[32 * r + lane];
       if (i < end && (key < 0 || key >= K)) bad = true;
-      if (i >= end || key < 0 || key >= K) key = -1;
-      const unsigned peers = __match_any_sync(0xffffffffu, key);
-      if (key >= 0 && lane == __ffs(peers) - 1) bins[key] += __popc(peers);
-      __syncwarp();
+      if (i < end && key >= 0 && key < K) atomicAdd(&bins[key], 1);
     }
     __syncwarp();
   }
@@ -146,7 +157,7 @@ __global__ void __launch_bounds__(1024) part_offsets_kernel(const int64_t *__res
   if (t == 1023) offsets[K] = run;
 }
 
-__global__ void part_scatter_kernel(const int32_t *__restrict__ labels, int64_t N, int K, int64_t tile,
+__global__ void part_scatter_kernel(const int32_t *__restrict__ labels, int64_t N, int K, int nbits, int64_t tile,
                                     int64_t ntiles, const int32_t *__restrict__ tileoff,
                                     const int64_t *__restrict__ offsets, int32_t *__restrict__ perm,
                                     int32_t *__restrict__ sorted_labels, int wpb) {
@@ -169,7 +180,7 @@ __global__ void part_scatter_kernel(const int32_t *__restrict__ labels, int64_t 
       const int64_t i = pos + 32 * r + lane;
       int key = buf[32 * r + lane];
       if (i >= end || key < 0 || key >= K) key = -1;
-      const unsigned peers = __match_any_sync(0xffffffffu, key);
+      const unsigned peers = same_key_lanes(key, nbits);
       if (key >= 0) {
         const int32_t slot = run[key] + __popc(peers & lt);
         perm[slot] = (int32_t)i;
@@ -333,8 +344,10 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
   part_offsets_kernel<<<1, 1024, 0, s>>>(hist, K, offsets);
   count_launch(2);
   if (pl.ntiles > 0) {
-    part_scatter_kernel<<<blocks, 32 * wpb, smem, s>>>(labels, N, K, pl.tile, pl.ntiles, tilecnt, offsets, perm,
-                                                       sorted_labels, wpb);
+    int nbits = 0;
+    while ((1 << nbits) < K) ++nbits;
+    part_scatter_kernel<<<blocks, 32 * wpb, smem, s>>>(labels, N, K, nbits, pl.tile, pl.ntiles, tilecnt, offsets,
+                                                       perm, sorted_labels, wpb);
     count_launch();
   }
   return cudaGetLastError();

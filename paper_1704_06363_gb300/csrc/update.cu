@@ -213,22 +213,30 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
 
 // Incremental update, in three small kernels over the label vectors:
 //   delta_count  rows whose label changed, counted per new label (to add) and
-//                per old label (to subtract); labels outside [0, K) count as
-//                unassigned on either side;
+//                per old label (to subtract), warp-aggregated (warps with no
+//                change skip); labels outside [0, K) count as unassigned on
+//                either side;
 //   delta_scan   exclusive prefix of both counts -> fill cursors and totals;
 //                also moves n_k by (added - subtracted);
 //   delta_fill   the changed rows grouped by label (order inside a group is
 //                irrelevant for sums), as (row, label) lists;
 // then one sums launch runs over both lists (added, then subtracted).
-// Warp-aggregated increment: lanes with the same key add once, by the lowest
-// lane, and each lane gets its own slot (base + rank among equal keys).
-__device__ __forceinline__ int32_t warp_add(int32_t *ctr, int key, bool active) {
-  const unsigned act = __ballot_sync(0xffffffffu, active);
-  const unsigned peers = __match_any_sync(0xffffffffu, active ? key : -1) & act;
+// Warp-aggregated increment: lanes with the same key (found with one ballot
+// per key bit, keys in [0, 2^nbits)) add once, by the lowest lane, and each
+// lane gets its own slot (base + rank among equal keys).  Aggregation keeps
+// the atomics on K hot counters from serialising when many rows move.
+__device__ __forceinline__ int32_t warp_add(int32_t *ctr, int key, bool active, int nbits) {
+  unsigned peers = __ballot_sync(0xffffffffu, active);
+  for (int b = 0; b < nbits; ++b) {
+    const bool bit = (key >> b) & 1;
+    const unsigned m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
+  }
   const int lane = threadIdx.x & 31;
+  const int leader = active ? __ffs(peers) - 1 : lane;
   int32_t base = 0;
-  if (active && lane == __ffs(peers) - 1) base = atomicAdd(ctr + key, __popc(peers));
-  base = __shfl_sync(0xffffffffu, base, active ? __ffs(peers) - 1 : lane);
+  if (active && lane == leader) base = atomicAdd(ctr + key, __popc(peers));
+  base = __shfl_sync(0xffffffffu, base, leader);
   return base + __popc(peers & ((1u << lane) - 1u));
 }
 
@@ -254,7 +262,8 @@ __device__ __forceinline__ void load_pair(const int32_t *labels, const int32_t *
 template <int VEC>
 __global__ void __launch_bounds__(256) delta_count_kernel(const int32_t *__restrict__ labels,
                                                           const int32_t *__restrict__ prev, int64_t N, int K,
-                                                          int32_t *hist_add, int32_t *hist_sub, Header *hdr) {
+                                                          int nbits, int32_t *hist_add, int32_t *hist_sub,
+                                                          Header *hdr) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
   bool bad = false;
   // whole warps iterate together (the loop bound is rounded up to a warp)
@@ -274,8 +283,8 @@ __global__ void __launch_bounds__(256) delta_count_kernel(const int32_t *__restr
 #pragma unroll
     for (int e = 0; e < VEC; ++e) {
       const bool moved = a[e] != b[e];
-      warp_add(hist_add, a[e], moved && a[e] >= 0);
-      warp_add(hist_sub, b[e], moved && b[e] >= 0);
+      warp_add(hist_add, a[e], moved && a[e] >= 0, nbits);
+      warp_add(hist_sub, b[e], moved && b[e] >= 0, nbits);
     }
   }
   if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadLabel);
@@ -333,7 +342,8 @@ __global__ void __launch_bounds__(1024) delta_scan_kernel(const int32_t *__restr
 template <int VEC>
 __global__ void __launch_bounds__(256) delta_fill_kernel(const int32_t *__restrict__ labels,
                                                          const int32_t *__restrict__ prev, int64_t N, int K,
-                                                         int32_t *cur_add, int32_t *cur_sub, int32_t *add_rows,
+                                                         int nbits, int32_t *cur_add, int32_t *cur_sub,
+                                                         int32_t *add_rows,
                                                          int32_t *add_lab, int32_t *sub_rows, int32_t *sub_lab) {
   const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
   const int64_t Nw = (N + 32 * VEC - 1) / (32 * VEC) * (32 * VEC);
@@ -352,8 +362,8 @@ __global__ void __launch_bounds__(256) delta_fill_kernel(const int32_t *__restri
     for (int e = 0; e < VEC; ++e) {
       const bool moved = a[e] != b[e];
       const bool add = moved && a[e] >= 0, sub = moved && b[e] >= 0;
-      const int32_t sa = warp_add(cur_add, a[e], add);
-      const int32_t sb = warp_add(cur_sub, b[e], sub);
+      const int32_t sa = warp_add(cur_add, a[e], add, nbits);  // order inside a group is irrelevant
+      const int32_t sb = warp_add(cur_sub, b[e], sub, nbits);
       if (add) {
         add_rows[sa] = (int32_t)(i + e);
         add_lab[sa] = a[e];
@@ -712,18 +722,24 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
     int64_t blocks = (int64_t)num_sms() * 8;
     const int64_t want = (N + 256 * per - 1) / (256 * per);
     if (blocks > want) blocks = want;
+    int nbits = 0;
+    while ((1 << nbits) < K) ++nbits;
     if (vec)
-      delta_count_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.hist_add, ds.hist_sub, hdr);
+      delta_count_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.hist_add,
+                                                             ds.hist_sub, hdr);
     else
-      delta_count_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.hist_add, ds.hist_sub, hdr);
+      delta_count_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.hist_add,
+                                                             ds.hist_sub, hdr);
     delta_scan_kernel<<<1, 1024, 0, s>>>(ds.hist_add, ds.hist_sub, K, ds.cur_add, ds.cur_sub, ds.totals, st.counts,
                                          hdr);
     if (vec)
-      delta_fill_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.cur_add, ds.cur_sub,
-                                                            ds.add_rows, ds.add_lab, ds.sub_rows, ds.sub_lab);
+      delta_fill_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.cur_add,
+                                                            ds.cur_sub, ds.add_rows, ds.add_lab, ds.sub_rows,
+                                                            ds.sub_lab);
     else
-      delta_fill_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, ds.cur_add, ds.cur_sub,
-                                                            ds.add_rows, ds.add_lab, ds.sub_rows, ds.sub_lab);
+      delta_fill_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.cur_add,
+                                                            ds.cur_sub, ds.add_rows, ds.add_lab, ds.sub_rows,
+                                                            ds.sub_lab);
     count_launch(3);
     launch_sums_any(X, N, d, ldx, dtype,
                     SumsLists{ds.add_rows, ds.add_lab, ds.totals + 0, ds.sub_rows, ds.sub_lab, ds.totals + 1},
