@@ -68,8 +68,16 @@ extern "C" int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K
   if (!hist_out || !offsets_out) return fail(HME_EINVAL, "hist_out / offsets_out is NULL");
   if (N > 0 && (!labels || !perm_out)) return fail(HME_EINVAL, "labels / perm_out is NULL");
 
-  // Tile counts go right after the 256-byte header; lengthen tiles until they fit.
+  // One counting-sort pass (the two-pass form needs 12 bytes of scratch per
+  // label); tile counts go right after the 256-byte header; lengthen tiles
+  // until they fit.
   PartLayout pl = part_layout(sizeof(Header), N, K);
+  if (pl.two_pass) {
+    pl.two_pass = false;
+    pl.bins = K;
+    if (pl.tile < 4 * (int64_t)K) pl.tile = (4 * (int64_t)K + kStaticTileRound - 1) / kStaticTileRound * kStaticTileRound;
+    pl.ntiles = N > 0 ? (N + pl.tile - 1) / pl.tile : 0;
+  }
   const size_t room = kStaticScratchBytes - sizeof(Header);
   const int64_t max_tiles = (int64_t)(room / ((size_t)K * sizeof(int32_t)));
   if (max_tiles < 1) return fail(HME_EINVAL, "K = %d needs more than %zu bytes of static scratch", K, room);
