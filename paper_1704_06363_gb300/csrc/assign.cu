@@ -56,6 +56,7 @@ struct AssignParams {
   int st_stages;          // split A stages in tensor memory
   uint32_t b_stage_bytes; // one B stage (hi and lo operands)
   uint32_t a_col0;        // first TMEM column of the A stages
+  int wide;               // 2 BN <= 256: xh.[ch; cl] as one N = 2 BN MMA (accumulator columns j and BN + j add up)
   const float *xn;
   const float *cn;     // Kp entries, +inf past K
   int32_t *labels;
@@ -617,6 +618,7 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16_f32(kBM, (uint32_t)p.BN);
+      const uint32_t idesc2 = idesc_bf16_f32(kBM, 2u * (uint32_t)p.BN);
       uint32_t i = 0, acc_it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++acc_it) {
@@ -642,9 +644,16 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
           for (int k = 0; k < kBK / 16; ++k) {
             const uint64_t bd0 = smem_desc_sw128(bst + k * 32);
             const uint64_t bd1 = smem_desc_sw128(bst + p.b_bytes + k * 32);
-            tc_mma_bf16_ts(dt, at + 8u * k, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);  // xh . ch
-            tc_mma_bf16_ts(dt, at + 8u * k, bd1, idesc, 1u);                           // xh . cl
-            tc_mma_bf16_ts(dt, at + 32u + 8u * k, bd0, idesc, 1u);                     // xl . ch
+            if (p.wide) {
+              // ch and cl are adjacent in the stage: one MMA over both (columns
+              // 0..BN-1 get xh.ch, BN..2BN-1 get xh.cl), then xl.ch into 0..BN-1
+              tc_mma_bf16_ts(dt, at + 8u * k, bd0, idesc2, (kb > 0 || k > 0) ? 1u : 0u);  // xh . [ch; cl]
+              tc_mma_bf16_ts(dt, at + 32u + 8u * k, bd0, idesc, 1u);                       // xl . ch
+            } else {
+              tc_mma_bf16_ts(dt, at + 8u * k, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);  // xh . ch
+              tc_mma_bf16_ts(dt, at + 8u * k, bd1, idesc, 1u);                           // xh . cl
+              tc_mma_bf16_ts(dt, at + 32u + 8u * k, bd0, idesc, 1u);                     // xl . ch
+            }
           }
           tc_commit(smem_u32(&a_empty[t]));
           tc_commit(smem_u32(&b_empty[sb]));
@@ -745,17 +754,30 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
       int idx1 = 0, idx2 = 0;
       const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
       uint32_t ra[16], rb[16];
-      tmem_ld16(taddr, ra);
-      tmem_ld_wait(ra);
-      for (int c = 0; c < p.BN; c += 32) {
-        const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
-        if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
-        epilogue_group(ra, cb + c, c, best1, best2, best3, idx1, idx2);
-        if (more1) {
+      if (p.wide) {
+        // x.c = (column j) + (column BN + j)
+        for (int c = 0; c < p.BN; c += 16) {
+          tmem_ld16(taddr + (uint32_t)c, ra);
+          tmem_ld16(taddr + (uint32_t)(p.BN + c), rb);
+          tmem_ld_wait(ra);
           tmem_ld_wait(rb);
-          if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
-          epilogue_group(rb, cb + c + 16, c + 16, best1, best2, best3, idx1, idx2);
-          if (more2) tmem_ld_wait(ra);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) ra[j] = __float_as_uint(__uint_as_float(ra[j]) + __uint_as_float(rb[j]));
+          epilogue_group(ra, cb + c, c, best1, best2, best3, idx1, idx2);
+        }
+      } else {
+        tmem_ld16(taddr, ra);
+        tmem_ld_wait(ra);
+        for (int c = 0; c < p.BN; c += 32) {
+          const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+          if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
+          epilogue_group(ra, cb + c, c, best1, best2, best3, idx1, idx2);
+          if (more1) {
+            tmem_ld_wait(rb);
+            if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
+            epilogue_group(rb, cb + c + 16, c + 16, best1, best2, best3, idx1, idx2);
+            if (more2) tmem_ld_wait(ra);
+          }
         }
       }
       tc_fence_before();
@@ -1234,8 +1256,9 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
   p.b_stage_bytes = 2 * p.b_bytes;
   p.a_res_bytes = 0;
   // TMEM: accumulators (double-buffered when they fit) + 4 split A stages of 64 columns
+  p.wide = 2 * g.BN <= kMaxBN ? 1 : 0;
   uint32_t stride = 32;
-  while (stride < (uint32_t)g.BN) stride <<= 1;
+  while (stride < (uint32_t)(p.wide ? 2 * g.BN : g.BN)) stride <<= 1;
   p.acc_stride = stride;
   p.nbuf = (2 * stride + 64u * 4u <= 512u) ? 2 : 1;
   p.a_col0 = (uint32_t)p.nbuf * stride;
