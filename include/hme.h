@@ -68,6 +68,7 @@ extern "C" {
 #define HME_OP_PARTITION 2 /* hme_partition (d and dtype ignored) */
 #define HME_OP_ROUTE 3     /* hme_route */
 #define HME_OP_TAG_HIST 4  /* hme_tag_cluster_hist (d = vocabulary size V; dtype ignored) */
+#define HME_OP_STREAM 5    /* hme_kmeans_stream (N = chunk_rows) */
 
 /* ---- k-means++ seeding variants -------------------------------------- */
 #define HME_INIT_KMEANSPP 0           /* candidates = all N rows */
@@ -227,6 +228,32 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
 HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
                       int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,
                       size_t ws_bytes, void *stream);
+
+/*
+ * hme_kmeans_stream -- Lloyd's iterations (Section 2, "K-means clustering")
+ * for a feature set that stays outside HBM: X lives in page-locked host
+ * memory (or anywhere device-accessible) and is streamed through two device
+ * buffers of chunk_rows rows, the copy of one chunk overlapping the
+ * clustering of the previous one.  Each of the `iters` iterations assigns
+ * every chunk against the centres C_t (as hme_assign: Eq. 2, near ties
+ * re-scored exactly), adds the chunk's rows to the fp64 per-cluster sums (as
+ * hme_update_centroids' full pass), and then forms, from all N rows:
+ *   objectives_out[t] = J(C_t, labels) in fp64               (may be NULL),
+ *   C_inout = the new centres (S_k / n_k; the re-seed rule for empty
+ *             clusters, whose picked rows are read from X in place),
+ *   counts_out[k], *n_reseeded_out as hme_update_centroids   (may be NULL).
+ * labels_out int32[N] and mind_out float32[N] (device memory) hold the last
+ * iteration's assignment and distances.  The result is Lloyd's iteration
+ * on all N rows; only the fp64 summation order differs from the in-HBM path.
+ * X: N x d (ldx, dtype).  ws: hme_workspace_bytes(HME_OP_STREAM, chunk_rows,
+ * d, K, dtype) bytes of device memory.  The call creates one stream and four
+ * events of its own for the copies (so it cannot be captured into a graph);
+ * the caller's stream is ordered after all of its work.
+ */
+HME_API int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
+                              int32_t iters, int64_t chunk_rows, float *C_inout, int32_t *labels_out, float *mind_out,
+                              double *objectives_out, int64_t *counts_out, int32_t *n_reseeded_out, void *ws,
+                              size_t ws_bytes, void *stream);
 
 /*
  * hme_tag_cluster_hist -- the tag statistics of a clustering that Section 4.5

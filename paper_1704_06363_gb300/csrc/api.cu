@@ -245,6 +245,16 @@ size_t tag_ws_bytes(int K, int V) {
                   256);
 }
 
+// hme_kmeans_stream: a chunk's assign/update workspace, then two device chunk
+// buffers of dense rows (pitch stream_ld(d) elements: 16-byte rows for TMA).
+int64_t stream_ld(int d, int dtype) { return dtype == HME_F32 ? (d + 3) / 4 * 4 : (d + 7) / 8 * 8; }
+size_t stream_buf_bytes(int64_t chunk, int d, int dtype) {
+  return align_up((size_t)chunk * stream_ld(d, dtype) * (dtype == HME_F32 ? 4 : 2), 256);
+}
+size_t stream_ws_bytes(int64_t chunk, int d, int K, int dtype) {
+  return align_up(feature_layout(chunk, d, K, dtype, 0).total, 256) + 2 * stream_buf_bytes(chunk, d, dtype);
+}
+
 int clear_header(void *ws, cudaStream_t s) {
   HME_CUDA(cudaMemsetAsync(ws, 0, sizeof(Header), s), "clear workspace header");
   return HME_OK;
@@ -261,6 +271,10 @@ size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t 
   if (op == HME_OP_PARTITION) {
     if (N < 0 || N > (int64_t)0x7FFFFFFF || K < 1 || K > kMaxK) return 0;
     return align_up(part_layout(sizeof(Header), N, K).end, 256);
+  }
+  if (op == HME_OP_STREAM) {  // N is the chunk length
+    if (check_common(N, d, K, dtype) != HME_OK || N < 1) return 0;
+    return stream_ws_bytes(N, d, K, dtype);
   }
   if (op == HME_OP_TAG_HIST) {  // d is the vocabulary size V
     if (N < 0 || K < 1 || K > kMaxK || d < 1) return 0;
@@ -447,6 +461,111 @@ int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const i
                            counts_out, sparsity_out, at<Header>(ws, 0), s),
            "tag statistics");
   return HME_OK;
+}
+
+int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K, int32_t iters,
+                      int64_t chunk_rows, float *C_inout, int32_t *labels_out, float *mind_out,
+                      double *objectives_out, int64_t *counts_out, int32_t *n_reseeded_out, void *ws, size_t ws_bytes,
+                      void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  if (N < 1) return fail(HME_EINVAL, "N = %lld: nothing to cluster", (long long)N);
+  if (iters < 0) return fail(HME_EINVAL, "iters = %d is negative", iters);
+  if (chunk_rows < 1) return fail(HME_EINVAL, "chunk_rows = %lld must be positive", (long long)chunk_rows);
+  if (!X || !C_inout || !labels_out || !mind_out) return fail(HME_EINVAL, "X / C_inout / labels_out / mind_out is NULL");
+  if (ldx < d) return fail(HME_EINVAL, "ldx = %lld < d = %d", (long long)ldx, d);
+  const int64_t chunk = chunk_rows < N ? chunk_rows : N;
+  // X is read by the copy engine; the re-seed reads its picked rows in place,
+  // so host memory must be page-locked (device-accessible).
+  cudaPointerAttributes attr;
+  HME_CUDA(cudaPointerGetAttributes(&attr, X), "query X");
+  const void *Xdev = nullptr;
+  if (attr.type == cudaMemoryTypeDevice || attr.type == cudaMemoryTypeManaged)
+    Xdev = X;
+  else if (attr.type == cudaMemoryTypeHost)
+    Xdev = attr.devicePointer;
+  if (!Xdev) return fail(HME_EINVAL, "X must be page-locked host memory or device memory");
+  if (ws_bytes < stream_ws_bytes(chunk, d, K, dtype))
+    return fail(HME_ENOMEM, "workspace of %zu bytes is smaller than the %zu bytes needed", ws_bytes,
+                stream_ws_bytes(chunk, d, K, dtype));
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return fail(HME_EINVAL, "workspace is NULL or not 256-byte aligned");
+  const Layout L = feature_layout(chunk, d, K, dtype, 0);
+  const size_t e = dtype == HME_F32 ? 4 : 2;
+  const int64_t ldc = stream_ld(d, dtype);
+  char *buf[2] = {static_cast<char *>(ws) + align_up(L.total, 256),
+                  static_cast<char *>(ws) + align_up(L.total, 256) + stream_buf_bytes(chunk, d, dtype)};
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  Header *hdr = at<Header>(ws, 0);
+  int64_t *hist = at<int64_t>(ws, L.part.hist);
+  int64_t *offs = at<int64_t>(ws, L.part.offs);
+  int32_t *perm = at<int32_t>(ws, L.perm);
+  int32_t *slab = at<int32_t>(ws, L.slab);
+  UpdateState st{at<double>(ws, L.sums), at<int64_t>(ws, L.counts), at<double>(ws, L.x2sum)};
+  int32_t *dk = at<int32_t>(ws, L.delta_k);
+  int32_t *fl = at<int32_t>(ws, L.flagged);
+  DeltaScratch ds{dk, dk + K, dk + 2 * K, dk + 3 * K, reinterpret_cast<int64_t *>(dk + 4 * K),
+                  perm, slab, fl, fl + chunk, at<unsigned long long>(ws, L.reseed)};
+
+  // copies of chunk j + 1 run on their own stream while chunk j is clustered
+  cudaStream_t cs = nullptr;
+  cudaEvent_t ready[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr};
+  int rc = HME_OK;
+  auto cuda_ok = [&](cudaError_t err, const char *what) {
+    if (err != cudaSuccess && rc == HME_OK) rc = cuda_fail(err, what);
+    return rc == HME_OK;
+  };
+  if (cuda_ok(cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking), "stream: copy stream"))
+    for (int b = 0; b < 2 && rc == HME_OK; ++b) {
+      cuda_ok(cudaEventCreateWithFlags(&ready[b], cudaEventDisableTiming), "stream: event");
+      if (rc == HME_OK) cuda_ok(cudaEventCreateWithFlags(&done[b], cudaEventDisableTiming), "stream: event");
+      if (rc == HME_OK) cuda_ok(cudaEventRecord(done[b], s), "stream: event");
+    }
+  const int64_t nchunks = (N + chunk - 1) / chunk;
+  for (int t = 0; t < iters && rc == HME_OK; ++t) {
+    for (int64_t j = 0; j < nchunks && rc == HME_OK; ++j) {
+      const int64_t r0 = j * chunk, n = (N - r0) < chunk ? (N - r0) : chunk;
+      const int b = (int)(j & 1);
+      if (!cuda_ok(cudaStreamWaitEvent(cs, done[b], 0), "stream: wait buffer")) break;
+      if (!cuda_ok(cudaMemcpy2DAsync(buf[b], (size_t)ldc * e, static_cast<const char *>(X) + (size_t)r0 * ldx * e,
+                                     (size_t)ldx * e, (size_t)d * e, (size_t)n, cudaMemcpyDefault, cs),
+                   "stream: copy chunk"))
+        break;
+      if (!cuda_ok(cudaEventRecord(ready[b], cs), "stream: event")) break;
+      if (!cuda_ok(cudaStreamWaitEvent(s, ready[b], 0), "stream: wait chunk")) break;
+      // this chunk's re-score queues and centre-norm maximum start at zero
+      if (!cuda_ok(cudaMemsetAsync(&hdr->rescore_count, 0, 3 * sizeof(uint32_t), s), "stream: clear queues")) break;
+      if (!cuda_ok(cudaMemsetAsync(&hdr->cn_max_bits, 0, sizeof(uint32_t), s), "stream: clear queues")) break;
+      rc = do_assign(buf[b], n, d, ldc, dtype, C_inout, K, labels_out + r0, mind_out + r0, L, ws, false, s);
+      if (rc != HME_OK) break;
+      if (!cuda_ok(launch_partition(labels_out + r0, n, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab,
+                                    hdr, s),
+                   "stream: sort labels"))
+        break;
+      if (!cuda_ok(launch_update_add(buf[b], n, d, ldc, dtype, perm, slab, hist, offs + K, K, st, j == 0, s),
+                   "stream: sums"))
+        break;
+      cuda_ok(cudaEventRecord(done[b], s), "stream: event");
+    }
+    if (rc != HME_OK) break;
+    // objective of (C_t, labels), new centres, re-seeds (picked rows read from X in place)
+    if (!cuda_ok(cudaMemsetAsync(&hdr->objective, 0, sizeof(double), s), "stream: clear objective")) break;
+    if (!cuda_ok(launch_update_finish(Xdev, N, d, ldx, dtype, mind_out, K, st, ds, C_inout, counts_out,
+                                      n_reseeded_out, hdr, s),
+                 "stream: centres"))
+      break;
+    if (objectives_out)
+      cuda_ok(cudaMemcpyAsync(objectives_out + t, &hdr->objective, sizeof(double), cudaMemcpyDeviceToDevice, s),
+              "stream: copy objective");
+  }
+  // the copy stream's last work is ordered before the caller's stream goes on
+  for (int b = 0; b < 2; ++b)
+    if (ready[b]) cudaStreamWaitEvent(s, ready[b], 0);
+  for (int b = 0; b < 2; ++b) {
+    if (ready[b]) cudaEventDestroy(ready[b]);
+    if (done[b]) cudaEventDestroy(done[b]);
+  }
+  if (cs) cudaStreamDestroy(cs);
+  return rc;
 }
 
 int hme_debug_bounded_wait(uint64_t timeout_ns, void *ws, size_t ws_bytes, void *stream) {

@@ -157,6 +157,12 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
                           const int64_t *hist, const int64_t *valid_total, const float *mind, int K,
                           UpdateState st, DeltaScratch ds, float *C, int64_t *counts_out, int32_t *n_reseeded,
                           Header *hdr, cudaStream_t s);
+cudaError_t launch_update_finish(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *mind, int K,
+                                 UpdateState st, DeltaScratch ds, float *C, int64_t *counts_out, int32_t *n_reseeded,
+                                 Header *hdr, cudaStream_t s);
+cudaError_t launch_update_add(const void *X, int64_t n, int d, int64_t ldx, int dtype, const int32_t *perm,
+                              const int32_t *sorted_labels, const int64_t *hist, const int64_t *valid_total, int K,
+                              UpdateState st, bool reset, cudaStream_t s);
 cudaError_t launch_kmeanspp(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, uint64_t seed,
                             int64_t m, bool subsample, float *C_out, int32_t *rows, double *d2, double *part,
                             Header *hdr, cudaStream_t s);

@@ -693,7 +693,66 @@ void launch_sums_any(const void *X, int64_t N, int d, int64_t ldx, int dtype, co
   }
 }
 
+__global__ void counts_add_kernel(const int64_t *__restrict__ hist, int K, int64_t *counts) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k < K) counts[k] += hist[k];
+}
+
 }  // namespace
+
+// After the sums: objective and new centres, then the re-seed of empty
+// clusters from the rows (X may be any device-accessible pointer, e.g.
+// page-locked host memory: only the picked rows are read).
+cudaError_t launch_update_finish(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *mind, int K,
+                                 UpdateState st, DeltaScratch ds, float *C, int64_t *counts_out, int32_t *n_reseeded,
+                                 Header *hdr, cudaStream_t s) {
+  {
+    const dim3 grid((unsigned)K, (unsigned)((d + kFinThreads * kFinPer - 1) / (kFinThreads * kFinPer)));
+    if (dtype == HME_F32)
+      update_finish_kernel<HME_F32><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out, hdr);
+    else
+      update_finish_kernel<HME_BF16><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out,
+                                                                  hdr);
+  }
+  {
+    const int nblk = (num_sms() < kMaxSms ? num_sms() : kMaxSms) * 2;  // the candidate region holds kMaxSms * 2 blocks
+    const int nlists = nblk * kSelWarps;
+    reseed_select_kernel<<<nblk, 32 * kSelWarps, 0, s>>>(mind, N, st.counts, K, ds.cand);
+    const size_t hsm = (size_t)nlists * sizeof(int);
+    if (dtype == HME_F32)
+      reseed_apply_kernel<HME_F32><<<1, 1024, hsm, s>>>(X, d, ldx, st.counts, K, ds.cand, nlists, C, n_reseeded);
+    else
+      reseed_apply_kernel<HME_BF16><<<1, 1024, hsm, s>>>(X, d, ldx, st.counts, K, ds.cand, nlists, C, n_reseeded);
+  }
+  if (dtype == HME_F32)
+    update_reseed_kernel<HME_F32><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
+  else
+    update_reseed_kernel<HME_BF16><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
+  count_launch(4);
+  return cudaGetLastError();
+}
+
+// Streamed full pass: add one chunk's rows (sorted by label: perm / sorted
+// labels / hist of the chunk) to the state; reset first when asked.
+cudaError_t launch_update_add(const void *X, int64_t n, int d, int64_t ldx, int dtype, const int32_t *perm,
+                              const int32_t *sorted_labels, const int64_t *hist, const int64_t *valid_total, int K,
+                              UpdateState st, bool reset, cudaStream_t s) {
+  cudaError_t e;
+  if (reset) {
+    e = cudaMemsetAsync(st.sums, 0, (size_t)K * d * sizeof(double), s);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(st.x2sum, 0, sizeof(double), s);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(st.counts, 0, (size_t)K * sizeof(int64_t), s);
+    if (e != cudaSuccess) return e;
+  }
+  if (n <= 0) return cudaSuccess;
+  counts_add_kernel<<<(K + 255) / 256, 256, 0, s>>>(hist, K, st.counts);
+  count_launch();
+  launch_sums_any(X, n, d, ldx, dtype, SumsLists{perm, sorted_labels, valid_total, nullptr, nullptr, nullptr},
+                  st.sums, st.x2sum, false, s);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *labels,
                           const int32_t *prev_labels, const int32_t *perm, const int32_t *sorted_labels,
@@ -745,30 +804,7 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
                     SumsLists{ds.add_rows, ds.add_lab, ds.totals + 0, ds.sub_rows, ds.sub_lab, ds.totals + 1},
                     st.sums, st.x2sum, true, s);
   }
-  {
-    const dim3 grid((unsigned)K, (unsigned)((d + kFinThreads * kFinPer - 1) / (kFinThreads * kFinPer)));
-    if (dtype == HME_F32)
-      update_finish_kernel<HME_F32><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out, hdr);
-    else
-      update_finish_kernel<HME_BF16><<<grid, kFinThreads, 0, s>>>(st.sums, st.counts, C, d, st.x2sum, counts_out,
-                                                                  hdr);
-  }
-  {
-    const int nblk = (num_sms() < kMaxSms ? num_sms() : kMaxSms) * 2;  // the candidate region holds kMaxSms * 2 blocks
-    const int nlists = nblk * kSelWarps;
-    reseed_select_kernel<<<nblk, 32 * kSelWarps, 0, s>>>(mind, N, st.counts, K, ds.cand);
-    const size_t hsm = (size_t)nlists * sizeof(int);
-    if (dtype == HME_F32)
-      reseed_apply_kernel<HME_F32><<<1, 1024, hsm, s>>>(X, d, ldx, st.counts, K, ds.cand, nlists, C, n_reseeded);
-    else
-      reseed_apply_kernel<HME_BF16><<<1, 1024, hsm, s>>>(X, d, ldx, st.counts, K, ds.cand, nlists, C, n_reseeded);
-  }
-  if (dtype == HME_F32)
-    update_reseed_kernel<HME_F32><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
-  else
-    update_reseed_kernel<HME_BF16><<<1, 1024, 0, s>>>(X, N, d, ldx, mind, st.counts, K, C, n_reseeded);
-  count_launch(4);
-  return cudaGetLastError();
+  return launch_update_finish(X, N, d, ldx, dtype, mind, K, st, ds, C, counts_out, n_reseeded, hdr, s);
 }
 
 }  // namespace hme

@@ -18,7 +18,7 @@ import torch
 
 HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6)
 HME_F32, HME_BF16 = 0, 1
-HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST = range(5)
+HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST, HME_OP_STREAM = range(6)
 HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
 HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED = 0, 1
 
@@ -65,6 +65,8 @@ def lib():
         L.hme_route.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
         L.hme_partition_noalloc.restype = ctypes.c_int
         L.hme_partition_noalloc.argtypes = [p, i64, i32, p, p, p, p, p, p]
+        L.hme_kmeans_stream.restype = ctypes.c_int
+        L.hme_kmeans_stream.argtypes = [p, i64, i32, i64, i32, i32, i32, i64, p, p, p, p, p, p, p, sz, p]
         L.hme_tag_cluster_hist.restype = ctypes.c_int
         L.hme_tag_cluster_hist.argtypes = [p, p, p, i64, i32, i32, p, p, p, sz, p]
         L.hme_launch_count.restype = i64
@@ -185,6 +187,18 @@ def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offset
     w, wb = _ws(ws)
     _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, flags, _ptr(expert_out), _ptr(offsets_out),
                            _ptr(order_out), w, wb, _stream(stream)), "hme_route")
+
+
+def hme_kmeans_stream(X: torch.Tensor, K: int, iters: int, chunk_rows: int, C_inout: torch.Tensor,
+                      labels_out: torch.Tensor, mind_out: torch.Tensor, ws: torch.Tensor,
+                      objectives_out: Optional[torch.Tensor] = None, counts_out: Optional[torch.Tensor] = None,
+                      n_reseeded_out: Optional[torch.Tensor] = None, stream=None):
+    """Lloyd's iterations on X in page-locked host memory (or device memory), streamed in chunks."""
+    N, d, ldx, dt = _features(X)
+    w, wb = _ws(ws)
+    _check(lib().hme_kmeans_stream(_ptr(X), N, d, ldx, dt, K, iters, chunk_rows, _ptr(C_inout), _ptr(labels_out),
+                                   _ptr(mind_out), _ptr(objectives_out), _ptr(counts_out), _ptr(n_reseeded_out), w,
+                                   wb, _stream(stream)), "hme_kmeans_stream")
 
 
 def hme_tag_cluster_hist(offsets: torch.Tensor, tag_off: torch.Tensor, tags: torch.Tensor, K: int, V: int,
