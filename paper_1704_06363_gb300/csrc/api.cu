@@ -526,10 +526,12 @@ int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t 
       const int64_t r0 = j * chunk, n = (N - r0) < chunk ? (N - r0) : chunk;
       const int b = (int)(j & 1);
       if (!cuda_ok(cudaStreamWaitEvent(cs, done[b], 0), "stream: wait buffer")) break;
-      if (!cuda_ok(cudaMemcpy2DAsync(buf[b], (size_t)ldc * e, static_cast<const char *>(X) + (size_t)r0 * ldx * e,
-                                     (size_t)ldx * e, (size_t)d * e, (size_t)n, cudaMemcpyDefault, cs),
-                   "stream: copy chunk"))
-        break;
+      const char *src = static_cast<const char *>(X) + (size_t)r0 * ldx * e;
+      const cudaError_t ce =
+          ldx == ldc ? cudaMemcpyAsync(buf[b], src, (size_t)n * ldc * e, cudaMemcpyDefault, cs)  // contiguous rows
+                     : cudaMemcpy2DAsync(buf[b], (size_t)ldc * e, src, (size_t)ldx * e, (size_t)d * e, (size_t)n,
+                                         cudaMemcpyDefault, cs);
+      if (!cuda_ok(ce, "stream: copy chunk")) break;
       if (!cuda_ok(cudaEventRecord(ready[b], cs), "stream: event")) break;
       if (!cuda_ok(cudaStreamWaitEvent(s, ready[b], 0), "stream: wait chunk")) break;
       // this chunk's re-score queues and centre-norm maximum start at zero
