@@ -17,7 +17,7 @@
  * Section 4.2 fixes K = 50 on 256-dimensional PCA features; Section 4.5 shows
  * unbalanced cluster sizes with every cluster used.
  *
- * Everything the paper leaves open is a stated reading (listed in the design doc):
+ * Everything the paper leaves open is a stated reading:
  *   init = k-means++ (Arthur & Vassilvitskii 2007) driven by splitmix64
  *   (Steele, Lea, Flood 2014); a fixed number of Lloyd iterations; ties in the
  *   argmin go to the lowest centre index; the argmin is taken on the squared
