@@ -3,9 +3,10 @@
 Workload (default): 1,000,000 fp32 feature vectors, d = 2048, K = 64 centres,
 post-ReLU mixture of 64 Gaussians (about half zeros), the shape of pooled
 ResNet-50 features.  One step = one whole job on inputs resident in HBM:
-    prepare the features (row norms, bf16 split), 20 Lloyd iterations
-    (hme_assign + hme_update_centroids), then hme_route of all N rows with the
-    final centres (assign + expert partition), reusing the prepared features.
+    20 Lloyd iterations (hme_assign + hme_update_centroids; the first assign
+    also leaves the prepared features -- row norms, bf16 split -- in the
+    workspace for the later ones), then hme_route of all N rows with the final
+    centres (assign + expert partition), reusing the prepared features.
 The k-means++ seeding is the boundary and is not timed; every step starts
 from the same seeded centres.  value = Lloyd iterations per second of the
 whole job (all ranks); inputs (8.2 GB) are larger than L2 (129 MB).
@@ -260,14 +261,15 @@ def run_ours(args, w):
 
     def step(Xs, record=False):
         C.copy_(C0)
-        hme.hme_prepare_features(Xs, K, ws)
         for t in range(T):
             labels, prev = labels_buf[t % 2], (labels_buf[(t - 1) % 2] if t > 0 else None)
             if record:
                 a0 = torch.cuda.Event(enable_timing=True)
                 a1 = torch.cuda.Event(enable_timing=True)
                 a0.record(stream)
-            hme.hme_assign(Xs, C, labels, ws, mind, obj[t:t + 1], flags=hme.HME_ASSIGN_PREPARED)
+            # the first assign leaves the prepared features (row norms, bf16 split) in ws
+            hme.hme_assign(Xs, C, labels, ws, mind, obj[t:t + 1],
+                           flags=hme.HME_ASSIGN_PREPARED if t > 0 else hme.HME_ASSIGN_PREPARE_OUT)
             if record:
                 a1.record(stream)
                 u1 = torch.cuda.Event(enable_timing=True)
@@ -277,7 +279,7 @@ def run_ours(args, w):
                 moved_dev.copy_(ws[32:36].view(torch.int32))
             if record:
                 u1.record(stream)
-                ev_assign.append((a0, a1))
+                ev_assign.append((t, a0, a1))
                 ev_update.append((t, a1, u1))
         # route the training set with the final centres, reusing its prepared features
         hme.hme_route(Xs, C, expert, offsets, order, ws, flags=hme.HME_ASSIGN_PREPARED)
@@ -380,7 +382,11 @@ def run_ours(args, w):
 
     iters_total = T * args.steps * world
     value = iters_total / (ms / 1000.0)
-    t_assign = sum(a.elapsed_time(b) for a, b in ev_assign) / len(ev_assign)
+    # the assign kernel on prepared features (iterations 1..T-1); the first call also prepares
+    later = [a.elapsed_time(b) for t, a, b in ev_assign if t > 0] or [a.elapsed_time(b) for _, a, b in ev_assign]
+    t_assign = sum(later) / len(later)
+    first = [a.elapsed_time(b) for t, a, b in ev_assign if t == 0]
+    t_assign_first = sum(first) / len(first)
     full = [a.elapsed_time(b) for t, a, b in ev_update if t == 0]
     incr = [a.elapsed_time(b) for t, a, b in ev_update if t > 0]
     t_update = sum(full) / len(full)
@@ -392,7 +398,7 @@ def run_ours(args, w):
     a_gbs = assign_bytes / (t_assign / 1000) / 1e9
     u_gbs = update_bytes / (t_update / 1000) / 1e9
     # the dominant kernel by GPU time per step: T assign calls vs one full and T-1 incremental updates
-    dominant = "assign" if T * t_assign >= t_update + (T - 1) * t_incr else "update"
+    dominant = "assign" if (T - 1) * t_assign + t_assign_first >= t_update + (T - 1) * t_incr else "update"
     if dominant == "assign":
         achieved, traffic = a_gbs, profiled_traffic("assign.cu", "assign_relu_gmm64_n1e6_d2048_k64_f32")
     else:
@@ -450,14 +456,14 @@ def run_ours(args, w):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16x3" if w.dtype == "f32" else "bf16",
             "data": "synthetic",
             "config": {"workload": w.name, "N": N, "d": d, "K": K, "feature_dtype": w.dtype, "iterations": T,
-                       "step": "prepare + %d x (assign + update; updates after the first read only rows whose label changed)"
+                       "step": "%d x (assign + update; the first assign also writes the prepared features, updates after the first read only rows whose label changed)"
                     " + route of all N rows" % T + (" + partition of the routed rows with their tag lists"
                                                       if w.tags else ""),
                        "l2": "inputs larger than L2 (%.1f GB of features)" % (X.numel() * e / 1e9),
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "vectors_per_s": N * iters_total / (ms / 1000.0),
             "assign_gflops": flops_assign / (t_assign / 1000.0) / 1e9,
-            "kernels_ms": {"assign_call": t_assign, "update_call_full": t_update, "update_call_incremental": t_incr,
+            "kernels_ms": {"assign_call": t_assign, "assign_call_prepare_out": t_assign_first, "update_call_full": t_update, "update_call_incremental": t_incr,
                            **route_ms,
                            "assign_gbs": a_gbs, "update_full_gbs": u_gbs},
             "roofline": roofline,

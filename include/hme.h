@@ -77,6 +77,11 @@ extern "C" {
 /* ---- hme_assign flags ------------------------------------------------- */
 #define HME_ASSIGN_DEFAULT 0
 #define HME_ASSIGN_PREPARED 1 /* ws already holds this X, prepared by hme_prepare_features */
+/* Not with HME_ASSIGN_PREPARED: the call also leaves this X prepared in ws, as
+ * hme_prepare_features would, so that later calls can pass HME_ASSIGN_PREPARED.
+ * An in-kernel split (see hme_prepare_features) writes the split rows as it
+ * makes them: the first Lloyd iteration reads X once instead of twice. */
+#define HME_ASSIGN_PREPARE_OUT 2
 
 /*
  * hme_workspace_bytes -- bytes of scratch an operation needs.
@@ -156,8 +161,9 @@ HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ld
  * direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of non-negative
  * terms).  The N x K distance matrix is never written.
  * X: N x d (ldx, dtype); C: K x d float32 (read only); labels_out: int32[N].
- * flags: HME_ASSIGN_DEFAULT, or HME_ASSIGN_PREPARED (skip the per-call
- * hme_prepare_features pass; ws must hold this X's preparation).
+ * flags: HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARE_OUT (also leave X prepared in
+ * ws), or HME_ASSIGN_PREPARED (skip the per-call hme_prepare_features pass; ws
+ * must hold this X's preparation).  Both at once: HME_EINVAL.
  */
 HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *C, int32_t K,
                int32_t flags, int32_t *labels_out, float *mind_out, double *objective_out,
@@ -221,9 +227,10 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
  * receives a contiguous run of rows:
  *   expert_out[b] = label of Q row b (int32[B]), offsets_out (int64[K+1]),
  *   order_out (int32[B]) = rows of Q grouped by expert, ascending within one.
- * flags: HME_ASSIGN_DEFAULT, or HME_ASSIGN_PREPARED when ws already holds Q
- * prepared by hme_prepare_features (e.g. routing the training set with the
- * workspace of the Lloyd loop: HME_OP_ROUTE and HME_OP_ASSIGN sizes agree).
+ * flags: HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARE_OUT, or HME_ASSIGN_PREPARED
+ * when ws already holds Q prepared by hme_prepare_features or a PREPARE_OUT
+ * call (e.g. routing the training set with the workspace of the Lloyd loop:
+ * HME_OP_ROUTE and HME_OP_ASSIGN sizes agree).
  */
 HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
                       int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,

@@ -204,9 +204,10 @@ int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, con
 // unprepared call on fp32 features that TMA can read splits the rows inside
 // the assign kernel (one pass over X); any other unprepared call prepares
 // first.  Prepared calls use the prepared operands, which stream at the
-// full HBM rate.
+// full HBM rate.  prepare_out: an in-kernel split also writes the prepared
+// operands to ws (every other unprepared call leaves them there anyway).
 int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K, int32_t *labels,
-              float *mind, const Layout &L, void *ws, bool prepared, cudaStream_t s) {
+              float *mind, const Layout &L, void *ws, bool prepared, cudaStream_t s, bool prepare_out) {
   const AssignGeom g = assign_geom(d, K, dtype);
   const bool split = !prepared && split_eligible(X, ldx, g);
   if (!prepared && !split) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s));
@@ -217,7 +218,10 @@ int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const flo
   if (split) {
     HME_TRY(launch_assign_split(static_cast<const float *>(X), N, ldx, g, at<__nv_bfloat16>(ws, L.cb_hi),
                                 at<__nv_bfloat16>(ws, L.cb_lo), at<float>(ws, L.cn), labels, mind, hdr,
-                                at<int32_t>(ws, L.flagged), at<int32_t>(ws, L.full_rows), s));
+                                at<int32_t>(ws, L.flagged), at<int32_t>(ws, L.full_rows),
+                                prepare_out ? at<__nv_bfloat16>(ws, L.xhi) : nullptr,
+                                prepare_out ? at<__nv_bfloat16>(ws, L.xlo) : nullptr,
+                                prepare_out ? at<float>(ws, L.xn) : nullptr, s));
   } else {
     HME_TRY(launch_assign_prepared(X, N, ldx, dtype, g, L, ws, labels, mind, hdr, s));
   }
@@ -353,12 +357,15 @@ int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, 
   HME_TRY(check_features(X, N, d, ldx, dtype, true));
   if (!C) return fail(HME_EINVAL, "C is NULL");
   if (N > 0 && !labels_out) return fail(HME_EINVAL, "labels_out is NULL");
-  if (flags & ~HME_ASSIGN_PREPARED) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  if ((flags & ~(HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) ||
+      (flags & (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) == (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT))
+    return fail(HME_EINVAL, "unknown flags 0x%x", flags);
   const Layout L = feature_layout(N, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s));
+  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s,
+                    (flags & HME_ASSIGN_PREPARE_OUT) != 0));
   if (objective_out)
     HME_CUDA(cudaMemcpyAsync(objective_out, &at<Header>(ws, 0)->objective, sizeof(double), cudaMemcpyDeviceToDevice,
                              s),
@@ -433,12 +440,15 @@ int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, c
   if (!C) return fail(HME_EINVAL, "C is NULL");
   if (!offsets_out) return fail(HME_EINVAL, "offsets_out is NULL");
   if (B > 0 && (!expert_out || !order_out)) return fail(HME_EINVAL, "expert_out / order_out is NULL");
-  if (flags & ~HME_ASSIGN_PREPARED) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  if ((flags & ~(HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) ||
+      (flags & (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) == (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT))
+    return fail(HME_EINVAL, "unknown flags 0x%x", flags);
   const Layout L = feature_layout(B, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s));
+  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s,
+                    (flags & HME_ASSIGN_PREPARE_OUT) != 0));
   HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
                             offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
            "route: partition");
@@ -537,7 +547,7 @@ int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t 
       // this chunk's re-score queues and centre-norm maximum start at zero
       if (!cuda_ok(cudaMemsetAsync(&hdr->rescore_count, 0, 3 * sizeof(uint32_t), s), "stream: clear queues")) break;
       if (!cuda_ok(cudaMemsetAsync(&hdr->cn_max_bits, 0, sizeof(uint32_t), s), "stream: clear queues")) break;
-      rc = do_assign(buf[b], n, d, ldc, dtype, C_inout, K, labels_out + r0, mind_out + r0, L, ws, false, s);
+      rc = do_assign(buf[b], n, d, ldc, dtype, C_inout, K, labels_out + r0, mind_out + r0, L, ws, false, s, false);
       if (rc != HME_OK) break;
       if (!cuda_ok(launch_partition(labels_out + r0, n, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab,
                                     hdr, s),

@@ -57,6 +57,8 @@ struct AssignParams {
   uint32_t b_stage_bytes; // one B stage (hi and lo operands)
   uint32_t a_col0;        // first TMEM column of the A stages
   int wide;               // 2 BN <= 256: xh.[ch; cl] as one N = 2 BN MMA (accumulator columns j and BN + j add up)
+  int write_split;  // also store the split rows (tensor maps tmOh, tmOl) and their norms (xn_out)
+  float *xn_out;
   const float *xn;
   const float *cn;     // Kp entries, +inf past K
   int32_t *labels;
@@ -502,7 +504,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float x0, float x1) {
 
 __global__ void __launch_bounds__(kSplitThreads, 1)
     assign_split_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmB0,
-                        const __grid_constant__ CUtensorMap tmB1, const AssignParams p) {
+                        const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmOh,
+                        const __grid_constant__ CUtensorMap tmOl, const AssignParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_u32(smem_raw);
   const uint32_t base = (raw_addr + 1023u) & ~1023u;
@@ -703,13 +706,44 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
             }
           }
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&x_empty[s]));  // the fp32 stage may be refilled
         const uint32_t at = tmem_base + lane_off + p.a_col0 + (uint32_t)t * 64u;
-        tmem_st16(at, hi);
-        tmem_st16(at + 16u, hi + 16);
-        tmem_st16(at + 32u, lo);
-        tmem_st16(at + 48u, lo + 16);
+        if (p.write_split) {
+          // Leave the split behind for later prepared calls: this thread has
+          // read all of its row, so it overwrites the row in place (hi in the
+          // first box, lo in the second, each a 64-column bf16 row in the same
+          // 128-byte swizzle) and lane 0 stores the warp's 32 rows with TMA;
+          // the stage is released once the bulk copies have read it.
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const uint32_t off = (uint32_t)r * 128u + ((uint32_t)(c ^ (r & 7)) << 4);
+            st_shared_u4(xring + (uint32_t)s * kXStage + off, hi[4 * c], hi[4 * c + 1], hi[4 * c + 2], hi[4 * c + 3]);
+            st_shared_u4(xring + (uint32_t)s * kXStage + kXBox + off, lo[4 * c], lo[4 * c + 1], lo[4 * c + 2],
+                         lo[4 * c + 3]);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0 && (int64_t)tile * kBM + q * 32 < p.N) {  // rows past N are clipped by TMA
+            const uint32_t src = xring + (uint32_t)s * kXStage + (uint32_t)q * 32u * 128u;
+            tma_store_2d(&tmOh, src, kb * kBK, tile * kBM + q * 32);
+            tma_store_2d(&tmOl, src + kXBox, kb * kBK, tile * kBM + q * 32);
+            bulk_commit();
+          }
+          tmem_st16(at, hi);
+          tmem_st16(at + 16u, hi + 16);
+          tmem_st16(at + 32u, lo);
+          tmem_st16(at + 48u, lo + 16);
+          if (lane == 0) {
+            bulk_wait_read_all();
+            mbar_arrive(smem_u32(&x_empty[s]));
+          }
+        } else {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&x_empty[s]));  // the fp32 stage may be refilled
+          tmem_st16(at, hi);
+          tmem_st16(at + 16u, hi + 16);
+          tmem_st16(at + 32u, lo);
+          tmem_st16(at + 48u, lo + 16);
+        }
         tmem_st_wait();
         tc_fence_before();
         __syncwarp();
@@ -725,6 +759,7 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&xn_full[b]));
     }
+    if (p.write_split && lane == 0) bulk_wait_all();
   } else {
     // ---------------- epilogue: argmin over the accumulator rows ----------------
     const int q = warp & 3;
@@ -748,6 +783,7 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
       }
       tc_fence_after();
       const float xr = xn_buf[(b * 2) * kBM + r] + xn_buf[(b * 2 + 1) * kBM + r];
+      if (p.xn_out && (int64_t)tile * kBM + r < p.N) p.xn_out[(int64_t)tile * kBM + r] = xr;
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&xn_empty[b]));
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
@@ -1236,11 +1272,16 @@ bool split_eligible(const void *X, int64_t ldx, const AssignGeom &g) {
 
 int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom &g, const __nv_bfloat16 *chi,
                         const __nv_bfloat16 *clo, const float *cn, int32_t *labels, float *mind, Header *hdr,
-                        int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
+                        int32_t *flagged, int32_t *full_rows, __nv_bfloat16 *xhi_out, __nv_bfloat16 *xlo_out,
+                        float *xn_out, cudaStream_t s) {
   if (N == 0) return HME_OK;
-  CUtensorMap mX, mB0, mB1;
+  CUtensorMap mX, mB0, mB1, mOh, mOl;
   int rc;
   if ((rc = make_map_f32(&mX, X, (uint64_t)N, (uint64_t)g.d, (uint64_t)ldx)) != HME_OK) return rc;
+  if (xhi_out) {  // 64 columns x 32 rows: one converter warp's share of a k-block
+    if ((rc = make_map(&mOh, xhi_out, (uint64_t)N, (uint64_t)g.d, (uint64_t)g.ldp, 32)) != HME_OK) return rc;
+    if ((rc = make_map(&mOl, xlo_out, (uint64_t)N, (uint64_t)g.d, (uint64_t)g.ldp, 32)) != HME_OK) return rc;
+  }
   if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
     return rc;
   if ((rc = make_map(&mB1, clo, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
@@ -1250,6 +1291,8 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
   p.num_kb = (g.d + kBK - 1) / kBK;
   p.BN = g.BN;
   p.nchunks = 1;
+  p.write_split = xhi_out ? 1 : 0;
+  p.xn_out = xn_out;
   p.num_tiles = (int)((N + kBM - 1) / kBM);
   p.a_bytes = 0;
   p.b_bytes = (uint32_t)g.BN * kBK * 2;
@@ -1298,7 +1341,7 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
   if (grid > p.num_tiles) grid = p.num_tiles;
   cudaError_t e = cudaFuncSetAttribute(assign_split_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "assign (split): set smem");
-  assign_split_kernel<<<grid, kSplitThreads, smem, s>>>(mX, mB0, mB1, p);
+  assign_split_kernel<<<grid, kSplitThreads, smem, s>>>(mX, mB0, mB1, xhi_out ? mOh : mB0, xhi_out ? mOl : mB1, p);
   count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign (split) kernel launch");

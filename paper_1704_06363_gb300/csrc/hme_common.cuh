@@ -119,10 +119,13 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s);
 // fp32 features with one N-chunk, split to bf16 hi/lo inside the kernel (no
 // preparation pass); eligible when X is 16-byte aligned and ldx % 4 == 0.
+// With xhi_out/xlo_out/xn_out set (all or none) the kernel also writes the
+// split rows (pitch g.ldp) and their norms, the layout of a preparation pass.
 bool split_eligible(const void *X, int64_t ldx, const AssignGeom &g);
 int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom &g, const __nv_bfloat16 *chi,
                         const __nv_bfloat16 *clo, const float *cn, int32_t *labels, float *mind, Header *hdr,
-                        int32_t *flagged, int32_t *full_rows, cudaStream_t s);
+                        int32_t *flagged, int32_t *full_rows, __nv_bfloat16 *xhi_out, __nv_bfloat16 *xlo_out,
+                        float *xn_out, cudaStream_t s);
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);
@@ -247,6 +250,26 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(policy)
       : "memory");
+}
+
+// Shared -> global tiled store (bulk-group completion); the writing threads
+// fence their generic-proxy stores with fence_proxy_async_smem() first.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int32_t c0, int32_t c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(c0), "r"(c1)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// the shared-memory sources of all committed bulk stores have been read
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// all committed bulk stores are complete
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void st_shared_u4(uint32_t saddr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(saddr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {

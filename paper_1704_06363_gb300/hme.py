@@ -20,7 +20,7 @@ HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6
 HME_F32, HME_BF16 = 0, 1
 HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST, HME_OP_STREAM = range(6)
 HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
-HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED = 0, 1
+HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED, HME_ASSIGN_PREPARE_OUT = 0, 1, 2
 
 _NAMES = {0: "HME_OK", 1: "HME_EINVAL", 2: "HME_ENOMEM", 3: "HME_ECUDA", 4: "HME_ETIMEOUT", 5: "HME_EINTERNAL"}
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libhme.so")

@@ -127,6 +127,46 @@ def test_assign_split_in_kernel_and_prepared_agree(dev, N, d, K):
     assert np.all(gap[differ] < parity.ASSIGN_GAP)
 
 
+@pytest.mark.parametrize("N,d,K", [(2000, 256, 32), (1001, 36, 7), (700, 130, 300)])
+def test_assign_prepare_out_leaves_the_prepared_split(dev, N, d, K):
+    """HME_ASSIGN_PREPARE_OUT: the call's own results are those of a default call
+    (bit-identical), and a later HME_ASSIGN_PREPARED call on other centres agrees
+    with one after hme_prepare_features (K = 300: the preparation pass; otherwise
+    the split written by the assign kernel).  The row norms of the two
+    preparations are summed in different orders, so labels may differ only at
+    near ties and both meet the oracle's bar."""
+    X = _mixture(N, d, min(K, 32), "f32", seed=N + d + 1)
+    C1 = hme_synth.random_centroids(K, d, seed=3, scale=3.0)
+    C1[: K // 2] = X[: K // 2].float()
+    C2 = hme_synth.random_centroids(K, d, seed=4, scale=3.0)
+    C2[K // 2:] = X[N - (K - K // 2):].float()
+    Xg, C1g, C2g = X.to(dev), C1.to(dev), C2.to(dev)
+    ws_out = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, hme.HME_F32, device=dev)
+    ws_ref = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, hme.HME_F32, device=dev)
+
+    def run(ws, C, flags):
+        lab = torch.full((N,), -1, dtype=torch.int32, device=dev)
+        md = torch.empty(N, dtype=torch.float32, device=dev)
+        obj = torch.zeros(1, dtype=torch.float64, device=dev)
+        hme.hme_assign(Xg, C, lab, ws, md, obj, flags=flags)
+        assert hme.hme_sync_status(ws) == hme.HME_OK
+        return lab.cpu().numpy(), md.cpu().numpy(), obj.item()
+
+    first = run(ws_out, C1g, hme.HME_ASSIGN_PREPARE_OUT)
+    plain = run(ws_ref, C1g, hme.HME_ASSIGN_DEFAULT)
+    assert all(np.array_equal(a, b) for a, b in zip(first[:2], plain[:2])) and first[2] == plain[2]
+    a = run(ws_out, C2g, hme.HME_ASSIGN_PREPARED)
+    hme.hme_prepare_features(Xg, K, ws_ref)
+    b = run(ws_ref, C2g, hme.HME_ASSIGN_PREPARED)
+    Xh = _host(X, "f32")
+    ref = oracle.assign(Xh, C2.numpy(), "f32")
+    for r in (a, b):
+        st = parity.check_assign(Xh, "f32", C2.numpy(), r[0], r[1], r[2], ref=ref)
+        assert st["mismatches"] <= st["near_ties"]
+    gap = (ref[2] - ref[1]) / np.maximum(ref[2], 1e-30)
+    assert np.all(gap[np.nonzero(a[0] != b[0])[0]] < parity.ASSIGN_GAP)
+
+
 def test_assign_duplicate_centres_and_zero_rows(dev):
     N, d, K = 600, 64, 8
     X = _mixture(N, d, 4, "f32", seed=3, relu=True)
