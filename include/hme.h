@@ -69,6 +69,7 @@ extern "C" {
 #define HME_OP_ROUTE 3     /* hme_route */
 #define HME_OP_TAG_HIST 4  /* hme_tag_cluster_hist (d = vocabulary size V; dtype ignored) */
 #define HME_OP_STREAM 5    /* hme_kmeans_stream (N = chunk_rows) */
+#define HME_OP_PCA 6       /* hme_pca_covariance, hme_pca_fit (K = r components); N = 0: hme_pca_transform only */
 
 /* ---- k-means++ seeding variants -------------------------------------- */
 #define HME_INIT_KMEANSPP 0           /* candidates = all N rows */
@@ -305,6 +306,50 @@ HME_API int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off,
 HME_API int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out,
                                   int64_t *offsets_out, int32_t *perm_out, int32_t *sorted_labels_out,
                                   int32_t *status_out, void *stream);
+
+/*
+ * PCA before the gater (Section 4.2, "Model and training details": the gater
+ * features Z = T^{L-1}(X) are projected onto their first 256 PCA dimensions
+ * before the K-means).  The paper names the method and the dimension only;
+ * readings: centred about the column mean, covariance normalised by N,
+ * unwhitened projection, components in decreasing variance, each signed so
+ * that its entry of largest magnitude (lowest index among equals) is positive.
+ * fp32 features only (dtype HME_F32; anything else is HME_EINVAL).
+ *
+ * hme_pca_covariance -- mean_out[j] = (1/N) sum_i x_ij (fp64, d entries) and
+ *   cov_out = (1/N) sum_i (x_i - mu)(x_i - mu)^T (fp64, d x d row-major, both
+ *   triangles).  The centred values y = x - fp32(mu) are split into bf16
+ *   y = yh + yl (|y - yh - yl| <= 2^-16 |y|) and the products
+ *   yh yh' + yh yl' + yl yh' are summed on the tensor cores in fp32 over 512
+ *   rows at a time (96 accumulation steps), those sums in fp64, so that each
+ *   entry is within (3 * 2^-16 + 98 * 2^-23) (1/N) sum_i (|y_ia| + |mu_a|)
+ *   (|y_ib| + |mu_b|) of the exact value (2^-23 per accumulation step: one
+ *   ulp, whatever the accumulator's rounding).  Requires N >= 1.
+ *
+ * hme_pca_fit -- the covariance as above, then its eigendecomposition by
+ *   cyclic Jacobi in fp32 (until the off-diagonal norm is at most 2^-22 of
+ *   the Frobenius norm, or stagnates below 2^-16 of it), then
+ *   mean_out (fp32, d), components_out (fp32, r x d row-major, orthonormal
+ *   rows), variances_out (fp32, r, the eigenvalues; may be NULL) and
+ *   *sweeps_out (host int32, the Jacobi sweeps made; may be NULL).
+ *   Synchronises `stream` once per sweep.  1 <= r <= d.  A matrix that does
+ *   not converge in 40 sweeps returns HME_EINTERNAL.
+ *
+ * hme_pca_transform -- Z_out[i * ldz + j] = components_j . (x_i - mean)
+ *   (fp32, N x r, ldz >= r): the assign kernel that splits fp32 rows inside
+ *   the kernel, the components as its centres (bf16 hi/lo, three products),
+ *   and mean.components_j (fp64, stored fp32) subtracted in the epilogue.
+ *   1 <= r <= 256; X on a 16-byte boundary with ldx % 4 == 0 (TMA).
+ *   Workspace: hme_workspace_bytes(HME_OP_PCA, 0, d, r, HME_F32) or larger.
+ */
+HME_API int hme_pca_covariance(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, double *mean_out,
+                               double *cov_out, void *ws, size_t ws_bytes, void *stream);
+HME_API int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t r, float *mean_out,
+                        float *components_out, float *variances_out, int32_t *sweeps_out, void *ws, size_t ws_bytes,
+                        void *stream);
+HME_API int hme_pca_transform(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *mean,
+                              const float *components, int32_t r, float *Z_out, int64_t ldz, void *ws,
+                              size_t ws_bytes, void *stream);
 
 /* Number of kernels this library has launched in this process (diagnostic). */
 HME_API int64_t hme_launch_count(void);

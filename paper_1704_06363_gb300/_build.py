@@ -19,7 +19,7 @@ LIBDIR = os.path.join(PKG, "lib")
 OBJDIR = os.path.join(LIBDIR, "obj")
 LIB = os.path.join(LIBDIR, "libhme.so")
 SOURCES = ["api.cu", "prep.cu", "assign.cu", "update.cu", "partition.cu", "init.cu", "partition_static.cu",
-           "tags.cu"]
+           "tags.cu", "pca.cu"]
 HEADERS = ["hme_common.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -216,12 +216,15 @@ int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const flo
                                at<float>(ws, L.cn), hdr, s),
            "prepare centres");
   if (split) {
+    SplitOut out;
+    if (prepare_out) {
+      out.xhi = at<__nv_bfloat16>(ws, L.xhi);
+      out.xlo = at<__nv_bfloat16>(ws, L.xlo);
+      out.xn = at<float>(ws, L.xn);
+    }
     HME_TRY(launch_assign_split(static_cast<const float *>(X), N, ldx, g, at<__nv_bfloat16>(ws, L.cb_hi),
                                 at<__nv_bfloat16>(ws, L.cb_lo), at<float>(ws, L.cn), labels, mind, hdr,
-                                at<int32_t>(ws, L.flagged), at<int32_t>(ws, L.full_rows),
-                                prepare_out ? at<__nv_bfloat16>(ws, L.xhi) : nullptr,
-                                prepare_out ? at<__nv_bfloat16>(ws, L.xlo) : nullptr,
-                                prepare_out ? at<float>(ws, L.xn) : nullptr, s));
+                                at<int32_t>(ws, L.flagged), at<int32_t>(ws, L.full_rows), out, s));
   } else {
     HME_TRY(launch_assign_prepared(X, N, ldx, dtype, g, L, ws, labels, mind, hdr, s));
   }
@@ -264,6 +267,74 @@ int clear_header(void *ws, cudaStream_t s) {
   return HME_OK;
 }
 
+// PCA fit (hme_pca_covariance / hme_pca_fit): slab sums, mean, transposed
+// split, covariance partial tiles, the Jacobi matrices and small scratch.
+struct PcaLayout {
+  size_t slab, mean64, mean32, yh, yl, part, A0, A1, V0, V1, acc, order, total;
+};
+PcaLayout pca_layout(int64_t N, int d, int r) {
+  const PcaGeom g = pca_geom(N, d, r);
+  PcaLayout L;
+  size_t off = sizeof(Header);
+  auto take = [&](size_t bytes) {
+    off = align_up(off, 256);
+    const size_t at = off;
+    off += bytes;
+    return at;
+  };
+  L.slab = take((size_t)g.nslabs * d * 8);
+  L.mean64 = take((size_t)d * 8);
+  L.mean32 = take((size_t)d * 4);
+  L.yh = take((size_t)d * g.ldn * 2);
+  L.yl = take((size_t)d * g.ldn * 2);
+  L.part = take((size_t)g.nchunks * g.ntiles * kBM * kBM * 8);
+  const size_t nn = (size_t)g.n * g.n * 4;
+  L.A0 = take(nn);
+  L.A1 = take(nn);
+  L.V0 = take(nn);
+  L.V1 = take(nn);
+  L.acc = take(16);
+  L.order = take((size_t)r * 4);
+  L.total = align_up(off, 256);
+  return L;
+}
+// hme_pca_transform: the components split to bf16 (hi, lo), their norms and
+// the per-component offsets mu.w_j
+struct PcaTLayout {
+  size_t chi, clo, cn, zoff, total;
+};
+PcaTLayout pca_t_layout(int d, int r) {
+  const AssignGeom g = assign_geom(d, r, HME_F32);
+  PcaTLayout L;
+  size_t off = sizeof(Header);
+  auto take = [&](size_t bytes) {
+    off = align_up(off, 256);
+    const size_t at = off;
+    off += bytes;
+    return at;
+  };
+  L.chi = take((size_t)g.Kp * g.ldp * 2);
+  L.clo = take((size_t)g.Kp * g.ldp * 2);
+  L.cn = take((size_t)g.Kp * 4);
+  L.zoff = take((size_t)g.Kp * 4);
+  L.total = align_up(off, 256);
+  return L;
+}
+int check_pca_sizes(int64_t N, int d, int dtype, int r, int64_t min_n) {
+  if (dtype != HME_F32) return fail(HME_EINVAL, "PCA takes fp32 features (dtype HME_F32)");
+  if (N < min_n || N > (int64_t)0x7FFFFFFF)
+    return fail(HME_EINVAL, "N = %lld out of range [%lld, 2^31)", (long long)N, (long long)min_n);
+  if (d < 1 || d > kMaxD) return fail(HME_EINVAL, "d = %d out of range [1, %d]", d, kMaxD);
+  if (r < 1 || r > d) return fail(HME_EINVAL, "r = %d out of range [1, d = %d]", r, d);
+  return HME_OK;
+}
+int check_pca(const void *X, int64_t N, int d, int64_t ldx, int dtype, int r, int64_t min_n) {
+  HME_TRY(check_pca_sizes(N, d, dtype, r, min_n));
+  if (N > 0 && !X) return fail(HME_EINVAL, "feature pointer is NULL");
+  if (ldx < d) return fail(HME_EINVAL, "ldx = %lld < d = %d", (long long)ldx, d);
+  return HME_OK;
+}
+
 }  // namespace
 }  // namespace hme
 
@@ -279,6 +350,13 @@ size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t 
   if (op == HME_OP_STREAM) {  // N is the chunk length
     if (check_common(N, d, K, dtype) != HME_OK || N < 1) return 0;
     return stream_ws_bytes(N, d, K, dtype);
+  }
+  if (op == HME_OP_PCA) {  // K is the number of components r; N = 0: hme_pca_transform only
+    if (check_pca_sizes(N, d, dtype, K, 0) != HME_OK) return 0;
+    const size_t t = pca_t_layout(d, K > kMaxBN ? kMaxBN : K).total;
+    if (N == 0) return t;
+    const size_t f = pca_layout(N, d, K).total;
+    return f > t ? f : t;
   }
   if (op == HME_OP_TAG_HIST) {  // d is the vocabulary size V
     if (N < 0 || K < 1 || K > kMaxK || d < 1) return 0;
@@ -470,6 +548,84 @@ int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const i
   HME_CUDA(launch_tag_hist(offsets, tag_off, tags, K, V, at<int64_t>(ws, sizeof(Header)), at<double>(ws, sums_at),
                            counts_out, sparsity_out, at<Header>(ws, 0), s),
            "tag statistics");
+  return HME_OK;
+}
+
+int hme_pca_covariance(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, double *mean_out,
+                       double *cov_out, void *ws, size_t ws_bytes, void *stream) {
+  HME_TRY(check_pca(X, N, d, ldx, dtype, 1, 1));
+  if (!mean_out || !cov_out) return fail(HME_EINVAL, "mean_out / cov_out is NULL");
+  const PcaLayout L = pca_layout(N, d, 1);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  const PcaGeom g = pca_geom(N, d, 1);
+  const float *Xf = static_cast<const float *>(X);
+  HME_CUDA(launch_pca_mean(Xf, g, ldx, at<double>(ws, L.slab), at<double>(ws, L.mean64), at<float>(ws, L.mean32), s),
+           "pca: mean");
+  HME_TRY(launch_pca_cov(Xf, g, ldx, at<float>(ws, L.mean32), at<__nv_bfloat16>(ws, L.yh),
+                         at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), cov_out, at<float>(ws, L.A0),
+                         at<Header>(ws, 0), s));
+  HME_CUDA(cudaMemcpyAsync(mean_out, at<double>(ws, L.mean64), (size_t)d * 8, cudaMemcpyDeviceToDevice, s),
+           "pca: copy mean");
+  return HME_OK;
+}
+
+int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t r, float *mean_out,
+                float *components_out, float *variances_out, int32_t *sweeps_out, void *ws, size_t ws_bytes,
+                void *stream) {
+  HME_TRY(check_pca(X, N, d, ldx, dtype, r, 1));
+  if (!mean_out || !components_out) return fail(HME_EINVAL, "mean_out / components_out is NULL");
+  const PcaLayout L = pca_layout(N, d, r);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  const PcaGeom g = pca_geom(N, d, r);
+  const float *Xf = static_cast<const float *>(X);
+  HME_CUDA(launch_pca_mean(Xf, g, ldx, at<double>(ws, L.slab), at<double>(ws, L.mean64), at<float>(ws, L.mean32), s),
+           "pca: mean");
+  HME_TRY(launch_pca_cov(Xf, g, ldx, at<float>(ws, L.mean32), at<__nv_bfloat16>(ws, L.yh),
+                         at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), nullptr, at<float>(ws, L.A0),
+                         at<Header>(ws, 0), s));
+  int sweeps = 0;
+  const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.A1), at<float>(ws, L.V0), at<float>(ws, L.V1),
+                                at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,
+                                &sweeps, s);
+  if (sweeps_out) *sweeps_out = sweeps;
+  if (rc != HME_OK) return rc;
+  HME_CUDA(cudaMemcpyAsync(mean_out, at<float>(ws, L.mean32), (size_t)d * 4, cudaMemcpyDeviceToDevice, s),
+           "pca: copy mean");
+  return HME_OK;
+}
+
+int hme_pca_transform(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *mean,
+                      const float *components, int32_t r, float *Z_out, int64_t ldz, void *ws, size_t ws_bytes,
+                      void *stream) {
+  HME_TRY(check_pca(X, N, d, ldx, dtype, r, 0));
+  if (r > kMaxBN) return fail(HME_EINVAL, "r = %d: hme_pca_transform takes at most %d components", r, kMaxBN);
+  if (!mean || !components) return fail(HME_EINVAL, "mean / components is NULL");
+  if (N > 0 && !Z_out) return fail(HME_EINVAL, "Z_out is NULL");
+  if (ldz < r) return fail(HME_EINVAL, "ldz = %lld < r = %d", (long long)ldz, r);
+  const AssignGeom g = assign_geom(d, r, HME_F32);
+  if (N > 0 && !split_eligible(X, ldx, g))
+    return fail(HME_EINVAL, "X must start on a 16-byte boundary with ldx %% 4 == 0 (TMA)");
+  const PcaTLayout L = pca_t_layout(d, r);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  if (N == 0) return HME_OK;
+  Header *hdr = at<Header>(ws, 0);
+  HME_CUDA(launch_prep_centres(components, g, at<__nv_bfloat16>(ws, L.chi), at<__nv_bfloat16>(ws, L.clo),
+                               at<float>(ws, L.cn), hdr, s),
+           "pca: prepare components");
+  HME_CUDA(launch_pca_zoff(mean, components, d, r, g.Kp, at<float>(ws, L.zoff), s), "pca: offsets");
+  SplitOut out;
+  out.z = Z_out;
+  out.ldz = ldz;
+  out.zcols = r;
+  HME_TRY(launch_assign_split(static_cast<const float *>(X), N, ldx, g, at<__nv_bfloat16>(ws, L.chi),
+                              at<__nv_bfloat16>(ws, L.clo), at<float>(ws, L.zoff), nullptr, nullptr, hdr, nullptr,
+                              nullptr, out, s));
   return HME_OK;
 }
 

@@ -59,6 +59,10 @@ struct AssignParams {
   int wide;               // 2 BN <= 256: xh.[ch; cl] as one N = 2 BN MMA (accumulator columns j and BN + j add up)
   int write_split;  // also store the split rows (tensor maps tmOh, tmOl) and their norms (xn_out)
   float *xn_out;
+  float *z_out;     // projection mode: z_ij = x_i.c_j - cn_j for j < zcols, rows of pitch ldz (no argmin)
+  int64_t ldz;
+  int zcols;
+  int zvec;         // z_out 16-byte aligned and ldz % 4 == 0: float4 stores
   const float *xn;
   const float *cn;     // Kp entries, +inf past K
   int32_t *labels;
@@ -790,6 +794,39 @@ __global__ void __launch_bounds__(kSplitThreads, 1)
       int idx1 = 0, idx2 = 0;
       const uint32_t taddr = tmem_base + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
       uint32_t ra[16], rb[16];
+      if (p.z_out) {
+        // projection: write x.c_j - cn_j (cn holds the per-column offsets)
+        const int64_t row = (int64_t)tile * kBM + r;
+        float *zr = p.z_out + row * p.ldz;
+        for (int c = 0; c < p.BN; c += 16) {
+          tmem_ld16(taddr + (uint32_t)c, ra);
+          if (p.wide) tmem_ld16(taddr + (uint32_t)(p.BN + c), rb);
+          tmem_ld_wait(ra);
+          if (p.wide) {
+            tmem_ld_wait(rb);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) ra[j] = __float_as_uint(__uint_as_float(ra[j]) + __uint_as_float(rb[j]));
+          }
+          float z[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) z[j] = __uint_as_float(ra[j]) - cb[c + j];
+          if (row < p.N) {
+            if (p.zvec && c + 16 <= p.zcols) {
+#pragma unroll
+              for (int j = 0; j < 16; j += 4)
+                *reinterpret_cast<float4 *>(zr + c + j) = make_float4(z[j], z[j + 1], z[j + 2], z[j + 3]);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j)
+                if (c + j < p.zcols) zr[c + j] = z[j];
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
+        continue;
+      }
       if (p.wide) {
         // x.c = (column j) + (column BN + j)
         for (int c = 0; c < p.BN; c += 16) {
@@ -1193,6 +1230,10 @@ int make_map_f32(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, 
 
 }  // namespace
 
+int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows) {
+  return make_map(m, ptr, rows, cols, ld, box_rows);
+}
+
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
@@ -1272,8 +1313,9 @@ bool split_eligible(const void *X, int64_t ldx, const AssignGeom &g) {
 
 int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom &g, const __nv_bfloat16 *chi,
                         const __nv_bfloat16 *clo, const float *cn, int32_t *labels, float *mind, Header *hdr,
-                        int32_t *flagged, int32_t *full_rows, __nv_bfloat16 *xhi_out, __nv_bfloat16 *xlo_out,
-                        float *xn_out, cudaStream_t s) {
+                        int32_t *flagged, int32_t *full_rows, const SplitOut &out, cudaStream_t s) {
+  __nv_bfloat16 *xhi_out = out.xhi, *xlo_out = out.xlo;
+  float *xn_out = out.xn;
   if (N == 0) return HME_OK;
   CUtensorMap mX, mB0, mB1, mOh, mOl;
   int rc;
@@ -1293,6 +1335,10 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
   p.nchunks = 1;
   p.write_split = xhi_out ? 1 : 0;
   p.xn_out = xn_out;
+  p.z_out = out.z;
+  p.ldz = out.ldz;
+  p.zcols = out.zcols;
+  p.zvec = out.z && (reinterpret_cast<uintptr_t>(out.z) & 15u) == 0 && out.ldz % 4 == 0;
   p.num_tiles = (int)((N + kBM - 1) / kBM);
   p.a_bytes = 0;
   p.b_bytes = (uint32_t)g.BN * kBK * 2;

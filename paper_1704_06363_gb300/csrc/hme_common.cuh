@@ -119,13 +119,25 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s);
 // fp32 features with one N-chunk, split to bf16 hi/lo inside the kernel (no
 // preparation pass); eligible when X is 16-byte aligned and ldx % 4 == 0.
-// With xhi_out/xlo_out/xn_out set (all or none) the kernel also writes the
-// split rows (pitch g.ldp) and their norms, the layout of a preparation pass.
+// Optional outputs: with xhi/xlo/xn set (all or none) the kernel also writes
+// the split rows (pitch g.ldp) and their norms, the layout of a preparation
+// pass.  With z set it is a projection instead of an assign: it writes
+// z[i * ldz + j] = x_i.c_j - cn[j] for j < zcols and touches no label, mind
+// or queue.
+struct SplitOut {
+  __nv_bfloat16 *xhi = nullptr, *xlo = nullptr;
+  float *xn = nullptr;
+  float *z = nullptr;
+  int64_t ldz = 0;
+  int zcols = 0;
+};
 bool split_eligible(const void *X, int64_t ldx, const AssignGeom &g);
 int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom &g, const __nv_bfloat16 *chi,
                         const __nv_bfloat16 *clo, const float *cn, int32_t *labels, float *mind, Header *hdr,
-                        int32_t *flagged, int32_t *full_rows, __nv_bfloat16 *xhi_out, __nv_bfloat16 *xlo_out,
-                        float *xn_out, cudaStream_t s);
+                        int32_t *flagged, int32_t *full_rows, const SplitOut &out, cudaStream_t s);
+// bf16 matrix rows x cols (row stride ld elements), box = box_rows x 64
+// columns, 128-byte swizzle (the operand layout of the tcgen05 kernels).
+int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows);
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);
@@ -175,6 +187,29 @@ constexpr int kTagSlices = 16;
 cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int K, int V,
                             int64_t *chunk_start, double *colsums, int64_t *counts, double *sparsity, Header *hdr,
                             cudaStream_t s);
+// PCA (pca.cu): see the file header for the steps.
+constexpr int64_t kCovSub = 512;  // rows per fp32 (TMEM) accumulation of the covariance
+constexpr int kJacobiMaxSweeps = 40;
+struct PcaGeom {
+  int64_t N;
+  int d, r;
+  int n;           // Jacobi order: d rounded up to even
+  int64_t ldn;     // row pitch (elements) of the transposed split: N rounded up to 8
+  int mi, ntiles;  // 128-feature tiles along d; upper-triangle tiles
+  int64_t R, nchunks, nslabs;  // rows per covariance work unit, units per tile, column-sum slabs
+};
+PcaGeom pca_geom(int64_t N, int d, int r);
+cudaError_t launch_pca_mean(const float *X, const PcaGeom &g, int64_t ldx, double *slab_sums, double *mean64,
+                            float *mean32, cudaStream_t s);
+// centred transposed split, tcgen05 covariance partials, fp64 reduction into
+// cov (d x d, may be null) and A (fp32, order g.n)
+int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *mean32, __nv_bfloat16 *yh,
+                   __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s);
+// Jacobi sweeps on A0 (synchronises s once per sweep), then the r leading
+// components (rows of W, r x d) and their variances (may be null)
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1, double *acc, int32_t *order,
+                   float *W, float *variances, int *sweeps_out, cudaStream_t s);
+cudaError_t launch_pca_zoff(const float *mean, const float *W, int d, int r, int Kp, float *zoff, cudaStream_t s);
 cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
 int64_t kpp_candidates(int64_t N, int K, int method);
 constexpr int kMaxSms = 256;  // bound used to size the re-seed candidate region

@@ -1,0 +1,747 @@
+// pca.cu -- principal components of the gater features (Section 4.2, "Model
+// and training details": before the K-means, Z = T^{L-1}(X) is projected onto
+// its first 256 principal directions).  Readings: centred about the column
+// mean, covariance normalised by N, unwhitened projection, components in
+// decreasing variance with the entry of largest magnitude positive.
+//
+// Fit:
+//   pca_colsum      per-slab column sums of X (fp32 over 32 rows, fp64 across);
+//   pca_mean        the slab sums added in slab order / N -> mu (fp64, fp32);
+//   pca_split_t     y = x - mu (fp32) split into bf16 y = yh + yl + O(2^-16 |y|),
+//                   written transposed (YT_hi, YT_lo: d x ldn, one row per
+//                   feature), so that the covariance is a K-major contraction
+//                   over the rows for the tensor cores;
+//   pca_cov         tcgen05 (kind::f16, fp32 accumulate in TMEM): work units
+//                   are (row range, 128 x 128 tile (i <= j) of the upper
+//                   triangle); a unit accumulates yh.yh' + yh.yl' + yl.yh' in
+//                   TMEM over kCovSub rows at a time (short fp32 sums), and its
+//                   epilogue adds each such sub-result into the unit's fp64
+//                   partial tile (read-modify-write, L2-resident) while the
+//                   MMAs of the next sub-range run in the other accumulator;
+//   pca_cov_reduce  the partial tiles added in range order in fp64, / N: the
+//                   covariance (fp64, both triangles) and A (fp32, order n = d
+//                   rounded up to even, padding row and column zero);
+//   Jacobi          cyclic two-sided Jacobi on A, n/2 disjoint rotations per
+//                   round (circle-method ordering: n - 1 rounds meet every pair
+//                   once).  One kernel per round reads A and V (the eigenvector
+//                   estimate, V <- V J) and writes them with the rotations
+//                   applied and the rows/columns moved to the next round's
+//                   slots, so that every pair is two adjacent slots and every
+//                   access is row-contiguous; the matrices (4 n^2 floats, 64 MB
+//                   at d = 2048) stay in L2.  After a sweep the slots are back
+//                   in their original order; sweeps repeat until
+//                   off(A) <= 2^-22 ||A||_F;
+//   pca_rank        eigenvalues diag(A) ranked (decreasing, ties to the lower
+//                   index), the padding slot excluded;
+//   pca_components  the leading r columns of V, normalised, with the sign rule.
+// Transform: hme_pca_transform runs the assign kernel that splits fp32 rows in
+// the kernel, with the components as its centres, in projection mode.
+#include "hme_common.cuh"
+
+namespace hme {
+
+namespace {
+
+constexpr int kColThreads = 256;
+constexpr int kColSlab = 2048;  // rows per column-sum block
+constexpr int kCovThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kCovStages = 3;
+constexpr uint32_t kCovOpBytes = kBM * kBK * 2;  // 128 rows x 64 bf16 = 16 KB
+constexpr uint32_t kCovStageBytes = 4 * kCovOpBytes;  // A hi, A lo, B hi, B lo
+constexpr uint32_t kCovTmemCols = 256;  // two 128-column accumulators
+constexpr int kJacSide = 16;  // pair-blocks per side of an A tile (32 x 32 elements)
+constexpr uint32_t kWhereCovProducer = 11, kWhereCovMma = 12, kWhereCovEpi = 13;
+
+// ---------------------------------------------------------------------------
+// mean and centred transposed split
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kColThreads) pca_colsum_kernel(const float *__restrict__ X, int64_t N, int d,
+                                                                 int64_t ldx, double *__restrict__ part) {
+  const int f = blockIdx.x * kColThreads + threadIdx.x;
+  if (f >= d) return;
+  const int64_t r0 = (int64_t)blockIdx.y * kColSlab;
+  const int64_t r1 = N < r0 + kColSlab ? N : r0 + kColSlab;
+  double acc = 0.0;
+  for (int64_t i = r0; i < r1; i += 32) {
+    const int64_t e = r1 < i + 32 ? r1 : i + 32;
+    float s = 0.0f;
+#pragma unroll 8
+    for (int64_t k = i; k < e; ++k) s += __ldg(X + k * ldx + f);
+    acc += (double)s;
+  }
+  part[(int64_t)blockIdx.y * d + f] = acc;
+}
+
+__global__ void pca_mean_kernel(const double *__restrict__ part, int64_t nslabs, int64_t N, int d,
+                                double *__restrict__ mean64, float *__restrict__ mean32) {
+  const int f = blockIdx.x * blockDim.x + threadIdx.x;
+  if (f >= d) return;
+  double s = 0.0;
+  for (int64_t b = 0; b < nslabs; ++b) s += part[b * d + f];
+  const double m = s / (double)N;
+  mean64[f] = m;
+  mean32[f] = (float)m;
+}
+
+__device__ __forceinline__ void split_bf16(float y, uint16_t &h, uint16_t &l) {
+  const __nv_bfloat16 hb = __float2bfloat16_rn(y);
+  const __nv_bfloat16 lb = __float2bfloat16_rn(y - __bfloat162float(hb));
+  h = __bfloat16_as_ushort(hb);
+  l = __bfloat16_as_ushort(lb);
+}
+
+// A block moves 64 rows x 64 features: loads coalesced along the features,
+// stores coalesced along the rows (128 bytes per feature row).  Rows past N
+// are zero (the columns N .. ldn-1 of YT are written as zeros).
+constexpr int kTPad = 66;  // shared row pitch in 16-bit elements (33 words: few bank conflicts)
+template <bool VEC>
+__global__ void __launch_bounds__(256) pca_split_t_kernel(const float *__restrict__ X, int64_t N, int d, int64_t ldx,
+                                                          const float *__restrict__ mu, int64_t ldn,
+                                                          __nv_bfloat16 *__restrict__ yh,
+                                                          __nv_bfloat16 *__restrict__ yl) {
+  __shared__ __align__(16) uint16_t sh[64 * kTPad];
+  __shared__ __align__(16) uint16_t sl[64 * kTPad];
+  const int64_t n0 = (int64_t)blockIdx.x * 64;
+  const int f0 = blockIdx.y * 64;
+  const int t = threadIdx.x;
+  const int c4 = (t & 15) * 4;
+  float m[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) m[e] = f0 + c4 + e < d ? __ldg(mu + f0 + c4 + e) : 0.0f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int rr = (t >> 4) + 16 * k;
+    const int64_t n = n0 + rr;
+    float v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if (n < N) {
+      const float *src = X + n * ldx + f0 + c4;
+      if (VEC && f0 + c4 + 3 < d) {
+        const float4 q = __ldg(reinterpret_cast<const float4 *>(src));
+        v[0] = q.x - m[0], v[1] = q.y - m[1], v[2] = q.z - m[2], v[3] = q.w - m[3];
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (f0 + c4 + e < d) v[e] = __ldg(src + e) - m[e];
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      uint16_t h, l;
+      split_bf16(v[e], h, l);
+      sh[(c4 + e) * kTPad + rr] = h;
+      sl[(c4 + e) * kTPad + rr] = l;
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < 2; ++k) {
+    const int idx = t + 256 * k;  // 64 features x 8 chunks of 8 rows
+    const int ff = idx >> 3, ch = idx & 7;
+    const int f = f0 + ff;
+    const int64_t n = n0 + ch * 8;
+    if (f < d && n < N) {
+      const uint32_t *ph = reinterpret_cast<const uint32_t *>(sh + ff * kTPad + ch * 8);
+      const uint32_t *pl = reinterpret_cast<const uint32_t *>(sl + ff * kTPad + ch * 8);
+      *reinterpret_cast<uint4 *>(yh + (int64_t)f * ldn + n) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+      *reinterpret_cast<uint4 *>(yl + (int64_t)f * ldn + n) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// covariance: tcgen05 over chunks of rows, upper-triangle tiles
+// ---------------------------------------------------------------------------
+struct CovParams {
+  int64_t N;
+  int64_t R;       // rows per unit range (multiple of kCovSub)
+  int mi;          // 128-feature tiles along d
+  int ntiles;      // mi (mi + 1) / 2
+  int64_t nunits;  // ranges x tiles
+  double *part;    // [nunits][128][128]
+  Header *hdr;
+  uint64_t limit_ns;
+};
+constexpr int kSubKb = (int)(kCovSub / kBK);  // k-blocks per TMEM accumulation
+
+// tile t of the upper triangle, enumerated row by row: (i, j), i <= j
+__device__ __forceinline__ void cov_tile(int t, int mi, int &i, int &j) {
+  int a = 0;
+  while (t >= mi - a) {
+    t -= mi - a;
+    ++a;
+  }
+  i = a;
+  j = a + t;
+}
+
+__global__ void __launch_bounds__(kCovThreads, 1)
+    pca_cov_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmL,
+                   const CovParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  const uint32_t base = (raw_addr + 1023u) & ~1023u;
+  uint8_t *smem = smem_raw + (base - raw_addr);
+  constexpr int S = kCovStages;
+  const uint32_t ring = base;
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + S * kCovStageBytes);
+  uint64_t *empty = full + S;
+  uint64_t *tfull = empty + S;
+  uint64_t *tempty = tfull + 2;
+  uint64_t *drain = tempty + 2;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmH);
+    prefetch_tensormap(&tmL);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), kCovTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  auto kblocks = [&](int64_t c) -> int {
+    const int64_t rows = p.N - c * p.R < p.R ? p.N - c * p.R : p.R;
+    return (int)((rows + kBK - 1) / kBK);
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const uint64_t pol = l2_policy_evict_last();  // a chunk is read by every tile of the triangle
+      uint32_t it = 0;
+      bool ok = true;
+      for (int64_t u = blockIdx.x; u < p.nunits && ok; u += gridDim.x) {
+        const int64_t c = u / p.ntiles;
+        int i, j;
+        cov_tile((int)(u - c * p.ntiles), p.mi, i, j);
+        const int nkb = kblocks(c);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait_bounded(smem_u32(&empty[s]), ((it / S) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereCovProducer)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[s]);
+          mbar_arrive_expect_tx(fb, kCovStageBytes);
+          const uint32_t st = ring + (uint32_t)s * kCovStageBytes;
+          const int32_t x = (int32_t)(c * p.R) + kb * kBK;
+          tma_load_2d(st, &tmH, fb, x, i * kBM, pol);
+          tma_load_2d(st + kCovOpBytes, &tmL, fb, x, i * kBM, pol);
+          tma_load_2d(st + 2 * kCovOpBytes, &tmH, fb, x, j * kBM, pol);
+          tma_load_2d(st + 3 * kCovOpBytes, &tmL, fb, x, j * kBM, pol);
+        }
+      }
+      if (!ok) {  // every copy issued must land before the CTA ends
+        for (uint32_t q = (it > (uint32_t)S ? it - S : 0); q < it; ++q)
+          mbar_wait_bounded(smem_u32(&full[q % S]), (q / S) & 1u, 200000000ull, p.hdr, kWhereCovProducer);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kBM, kBM);
+      uint32_t it = 0, acc_it = 0;
+      bool ok = true;
+      for (int64_t u = blockIdx.x; u < p.nunits && ok; u += gridDim.x) {
+        const int nkb = kblocks(u / p.ntiles);
+        for (int kb0 = 0; kb0 < nkb && ok; kb0 += kSubKb, ++acc_it) {
+          const uint32_t a = acc_it & 1u;
+          if (!mbar_wait_bounded(smem_u32(&tempty[a]), ((acc_it >> 1) & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereCovMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dt = tmem_base + a * (uint32_t)kBM;
+          const int kb1 = nkb < kb0 + kSubKb ? nkb : kb0 + kSubKb;
+          for (int kb = kb0; kb < kb1; ++kb, ++it) {
+            const int s = it % S;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (it / S) & 1u, p.limit_ns, p.hdr, kWhereCovMma)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = ring + (uint32_t)s * kCovStageBytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t ah = smem_desc_sw128(st + k * 32);
+              const uint64_t al = smem_desc_sw128(st + kCovOpBytes + k * 32);
+              const uint64_t bh = smem_desc_sw128(st + 2 * kCovOpBytes + k * 32);
+              const uint64_t bl = smem_desc_sw128(st + 3 * kCovOpBytes + k * 32);
+              tc_mma_bf16(dt, ah, bh, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+              tc_mma_bf16(dt, ah, bl, idesc, 1u);  // yh . yl'
+              tc_mma_bf16(dt, al, bh, idesc, 1u);  // yl . yh'
+            }
+            tc_commit(smem_u32(&empty[s]));
+          }
+          if (ok) tc_commit(smem_u32(&tfull[a]));
+        }
+      }
+      if (!ok) {
+        tc_commit(smem_u32(drain));
+        mbar_wait_bounded(smem_u32(drain), 0, 200000000ull, p.hdr, kWhereCovMma);
+      }
+    }
+  } else {
+    // epilogue: accumulator row (TMEM lane) -> one row of the partial tile
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    uint32_t acc_it = 0;
+    bool ok = true;
+    for (int64_t u = blockIdx.x; u < p.nunits && ok; u += gridDim.x) {
+      const int nkb = kblocks(u / p.ntiles);
+      double *dst = p.part + u * (int64_t)(kBM * kBM) + (int64_t)row * kBM;
+      for (int kb0 = 0; kb0 < nkb; kb0 += kSubKb, ++acc_it) {
+        const uint32_t a = acc_it & 1u;
+        if (!mbar_wait_bounded(smem_u32(&tfull[a]), (acc_it >> 1) & 1u, p.limit_ns, p.hdr, kWhereCovEpi)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + a * (uint32_t)kBM + ((uint32_t)(q * 32) << 16);
+        uint32_t r[16];
+        for (int c = 0; c < kBM; c += 16) {
+          tmem_ld16(taddr + (uint32_t)c, r);
+          tmem_ld_wait(r);
+          double2 *d2 = reinterpret_cast<double2 *>(dst + c);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const double x0 = (double)__uint_as_float(r[2 * e]), x1 = (double)__uint_as_float(r[2 * e + 1]);
+            if (kb0 == 0) {
+              d2[e] = make_double2(x0, x1);
+            } else {
+              const double2 o = d2[e];
+              d2[e] = make_double2(o.x + x0, o.y + x1);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kCovTmemCols);
+  }
+}
+
+// cov[a][b] = cov[b][a] = (sum over chunks of the partial entries, fp64, in
+// chunk order) / N for a <= b; A (order n) gets the same values in fp32.
+__global__ void __launch_bounds__(256) pca_cov_reduce_kernel(const double *__restrict__ part, int64_t nchunks,
+                                                             int ntiles, int mi, int d, int n, int64_t N,
+                                                             double *__restrict__ cov, float *__restrict__ A) {
+  if (blockIdx.x < blockIdx.y) return;  // 32 x 32 blocks wholly below the diagonal
+  const int b = blockIdx.x * 32 + (threadIdx.x & 31);
+  const int a0 = blockIdx.y * 32;
+  for (int aa = threadIdx.x >> 5; aa < 32; aa += 8) {
+    const int a = a0 + aa;
+    if (a >= d || b >= d || b < a) continue;
+    const int i = a >> 7, j = b >> 7;
+    const int t = i * mi - i * (i - 1) / 2 + (j - i);
+    const int64_t off = (int64_t)t * (kBM * kBM) + (int64_t)(a & 127) * kBM + (b & 127);
+    const int64_t stride = (int64_t)ntiles * (kBM * kBM);
+    double s = 0.0;
+    for (int64_t c = 0; c < nchunks; ++c) s += part[c * stride + off];
+    const double v = s / (double)N;
+    if (cov) {
+      cov[(int64_t)a * d + b] = v;
+      cov[(int64_t)b * d + a] = v;
+    }
+    A[(int64_t)a * n + b] = (float)v;
+    A[(int64_t)b * n + a] = (float)v;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Jacobi
+// ---------------------------------------------------------------------------
+// Circle-method ordering: slot 0 holds a fixed index; the other n - 1 indices
+// sit on a list whose position 0 is slot 1, positions 1 .. n/2-1 the even
+// slots 2, 4, .. and positions n/2 .. n-2 the odd slots n-1, n-3, .. 3.  Each
+// round pairs slots (2P, 2P + 1); between rounds every listed index moves one
+// position down the list (cyclically), so after n - 1 rounds each pair has met
+// once and every index is back in its slot.
+__device__ __forceinline__ int jac_next(int slot, int n) {
+  if (slot == 0) return 0;
+  const int pos = slot == 1 ? 0 : ((slot & 1) == 0 ? (slot >> 1) : n - 1 - ((slot - 1) >> 1));
+  int np = pos + n - 2;
+  if (np >= n - 1) np -= n - 1;
+  return np == 0 ? 1 : (np <= (n >> 1) - 1 ? 2 * np : 2 * (n - 1 - np) + 1);
+}
+
+// The rotation of one pair (Rutishauser's form): t = tan(phi) is the smaller
+// root of t^2 + 2 theta t - 1 = 0, theta = (a_qq - a_pp) / (2 a_pq), which
+// zeroes a_pq; the update of a pair of entries (u, v) of rows (or columns) p
+// and q is u - s (v + tau u), v + s (u - tau v) with s = sin(phi), tau =
+// tan(phi / 2), which keeps the norm of (u, v) to second order in s even when
+// cos(phi) rounds to 1.  Entries with |a_pq| <= 2^-23 sqrt(|a_pp| |a_qq|) are
+// left alone.  Not inlined: every block that needs a pair's rotation gets the
+// same bits from the same instructions.
+struct JacRot {
+  float s, tau, dp, dq;  // dp, dq: the new diagonal entries
+};
+__device__ __noinline__ JacRot jac_rot(float app, float aqq, float apq) {
+  JacRot r{0.0f, 0.0f, app, aqq};
+  if (apq != 0.0f && fabsf(apq) > 0x1p-23f * sqrtf(fabsf(app)) * sqrtf(fabsf(aqq))) {
+    const float theta = (aqq - app) / (2.0f * apq);
+    const float at = fabsf(theta);
+    float t = at > 0x1p20f ? 0.5f / at : 1.0f / (at + sqrtf(at * at + 1.0f));
+    t = copysignf(t, theta);
+    const float c = 1.0f / sqrtf(t * t + 1.0f);
+    r.s = t * c;
+    r.tau = r.s / (1.0f + c);
+    r.dp = app - t * apq;
+    r.dq = aqq + t * apq;
+  }
+  return r;
+}
+
+__device__ __forceinline__ JacRot jac_pair(const float *A, int n, int P) {
+  const int64_t p = 2 * P;
+  return jac_rot(A[p * n + p], A[(p + 1) * n + p + 1], A[p * n + p + 1]);
+}
+
+// Blocks [0, a_blocks): 32 x 32 tiles of A (a thread per 2 x 2 pair block);
+// the rest: 8 rows x 32 column pairs of V.
+__global__ void __launch_bounds__(256) jacobi_round_kernel(const float *__restrict__ A, const float *__restrict__ V,
+                                                           float *__restrict__ An, float *__restrict__ Vn, int n,
+                                                           int a_side, int v_side) {
+  __shared__ float rs[2][32][2];  // (s, tau) of the tile's row pairs [0] and column pairs [1]
+  __shared__ float rd[kJacSide][2];
+  const int np = n >> 1;
+  const int a_blocks = a_side * a_side;
+  if ((int)blockIdx.x < a_blocks) {
+    const int P0 = (blockIdx.x / a_side) * kJacSide, Q0 = (blockIdx.x % a_side) * kJacSide;
+    if (threadIdx.x < 2 * kJacSide) {
+      const int w = threadIdx.x / kJacSide, k = threadIdx.x % kJacSide;
+      const int P = (w ? Q0 : P0) + k;
+      if (P < np) {
+        const JacRot r = jac_pair(A, n, P);
+        rs[w][k][0] = r.s;
+        rs[w][k][1] = r.tau;
+        if (w == 0) {
+          rd[k][0] = r.dp;
+          rd[k][1] = r.dq;
+        }
+      }
+    }
+    __syncthreads();
+    const int ty = threadIdx.x / kJacSide, tx = threadIdx.x % kJacSide;
+    const int P = P0 + ty, Q = Q0 + tx;
+    if (P >= np || Q >= np) return;
+    const float2 u = *reinterpret_cast<const float2 *>(A + (int64_t)(2 * P) * n + 2 * Q);
+    const float2 v = *reinterpret_cast<const float2 *>(A + (int64_t)(2 * P + 1) * n + 2 * Q);
+    float b00, b01, b10, b11;
+    if (P == Q) {
+      b00 = rd[ty][0];
+      b11 = rd[ty][1];
+      b01 = b10 = 0.0f;
+    } else {
+      const float s1 = rs[0][ty][0], t1 = rs[0][ty][1], s2 = rs[1][tx][0], t2 = rs[1][tx][1];
+      const float m00 = u.x - s1 * (v.x + t1 * u.x), m10 = v.x + s1 * (u.x - t1 * v.x);
+      const float m01 = u.y - s1 * (v.y + t1 * u.y), m11 = v.y + s1 * (u.y - t1 * v.y);
+      b00 = m00 - s2 * (m01 + t2 * m00);
+      b01 = m01 + s2 * (m00 - t2 * m01);
+      b10 = m10 - s2 * (m11 + t2 * m10);
+      b11 = m11 + s2 * (m10 - t2 * m11);
+    }
+    const int64_t p0 = jac_next(2 * P, n), p1 = jac_next(2 * P + 1, n);
+    const int q0 = jac_next(2 * Q, n), q1 = jac_next(2 * Q + 1, n);
+    An[p0 * n + q0] = b00;
+    An[p0 * n + q1] = b01;
+    An[p1 * n + q0] = b10;
+    An[p1 * n + q1] = b11;
+  } else {
+    const int b = blockIdx.x - a_blocks;
+    const int k0 = (b / v_side) * 8, Q0 = (b % v_side) * 32;
+    if (threadIdx.x < 32 && Q0 + (int)threadIdx.x < np) {
+      const JacRot r = jac_pair(A, n, Q0 + threadIdx.x);
+      rs[1][threadIdx.x][0] = r.s;
+      rs[1][threadIdx.x][1] = r.tau;
+    }
+    __syncthreads();
+    const int64_t k = k0 + (threadIdx.x >> 5);
+    const int Q = Q0 + (threadIdx.x & 31);
+    if (k >= n || Q >= np) return;
+    const float s = rs[1][threadIdx.x & 31][0], tau = rs[1][threadIdx.x & 31][1];
+    const float2 w = *reinterpret_cast<const float2 *>(V + k * n + 2 * Q);
+    Vn[k * n + jac_next(2 * Q, n)] = w.x - s * (w.y + tau * w.x);
+    Vn[k * n + jac_next(2 * Q + 1, n)] = w.y + s * (w.x - tau * w.y);
+  }
+}
+
+__global__ void pca_identity_kernel(float *V, int n) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < (int64_t)n * n) V[i] = (i / n == i % n) ? 1.0f : 0.0f;
+}
+
+// acc[0] += sum of squared off-diagonal entries, acc[1] += sum of squared
+// diagonal entries (fp64).
+__global__ void __launch_bounds__(256) jacobi_offnorm_kernel(const float *__restrict__ A, int n, double *acc) {
+  double off = 0.0, dia = 0.0;
+  const int64_t total = (int64_t)n * n;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const double v = (double)A[i];
+    if (i / n == i % n)
+      dia += v * v;
+    else
+      off += v * v;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    off += __shfl_xor_sync(0xffffffffu, off, o);
+    dia += __shfl_xor_sync(0xffffffffu, dia, o);
+  }
+  __shared__ double so[8], sd[8];
+  if ((threadIdx.x & 31) == 0) {
+    so[threadIdx.x >> 5] = off;
+    sd[threadIdx.x >> 5] = dia;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double a = 0.0, b = 0.0;
+    for (int w = 0; w < 8; ++w) a += so[w], b += sd[w];
+    atomicAdd(acc, a);
+    atomicAdd(acc + 1, b);
+  }
+}
+
+// One block: rank of every eigenvalue among the d real ones (decreasing, ties
+// to the lower index); the r leading ones go to order[] and variances[].
+__global__ void __launch_bounds__(1024) pca_rank_kernel(const float *__restrict__ A, int n, int d, int r,
+                                                        int32_t *__restrict__ order, float *__restrict__ variances) {
+  extern __shared__ float lam[];
+  for (int j = threadIdx.x; j < d; j += blockDim.x) lam[j] = A[(int64_t)j * n + j];
+  __syncthreads();
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float v = lam[j];
+    int rank = 0;
+    for (int i = 0; i < d; ++i) rank += (lam[i] > v || (lam[i] == v && i < j)) ? 1 : 0;
+    if (rank < r) {
+      order[rank] = j;
+      if (variances) variances[rank] = v;
+    }
+  }
+}
+
+// Block k: column order[k] of V, normalised (fp64 norm), sign so that the
+// entry of largest magnitude (lowest index among equals) is positive.
+__global__ void __launch_bounds__(256) pca_components_kernel(const float *__restrict__ V, int n, int d,
+                                                             const int32_t *__restrict__ order,
+                                                             float *__restrict__ W) {
+  const int k = blockIdx.x;
+  const int j = order[k];
+  double ss = 0.0;
+  unsigned long long best = 0;  // |v| bits << 32 | (~index): max = largest magnitude, then lowest index
+  for (int m = threadIdx.x; m < d; m += blockDim.x) {
+    const float v = V[(int64_t)m * n + j];
+    ss += (double)v * (double)v;
+    const unsigned long long key =
+        ((unsigned long long)__float_as_uint(fabsf(v)) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)m);
+    best = key > best ? key : best;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    const unsigned long long ob = __shfl_xor_sync(0xffffffffu, best, o);
+    best = ob > best ? ob : best;
+  }
+  __shared__ double sss[8];
+  __shared__ unsigned long long sb[8];
+  __shared__ float scale;
+  if ((threadIdx.x & 31) == 0) {
+    sss[threadIdx.x >> 5] = ss;
+    sb[threadIdx.x >> 5] = best;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    unsigned long long bb = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      t += sss[w];
+      bb = sb[w] > bb ? sb[w] : bb;
+    }
+    const int mbest = (int)(0xFFFFFFFFu - (uint32_t)(bb & 0xFFFFFFFFull));
+    const float vb = V[(int64_t)mbest * n + j];
+    const double inv = t > 0.0 ? 1.0 / sqrt(t) : 1.0;
+    scale = (float)(vb < 0.0f ? -inv : inv);
+  }
+  __syncthreads();
+  const float sc = scale;
+  for (int m = threadIdx.x; m < d; m += blockDim.x) W[(int64_t)k * d + m] = V[(int64_t)m * n + j] * sc;
+}
+
+// zoff[j] = mu . w_j (fp64 sum, stored fp32) for j < r, 0 for r <= j < Kp.
+__global__ void __launch_bounds__(256) pca_zoff_kernel(const float *__restrict__ mu, const float *__restrict__ W,
+                                                       int d, int r, float *__restrict__ zoff) {
+  const int j = blockIdx.x;
+  double s = 0.0;
+  if (j < r)
+    for (int m = threadIdx.x; m < d; m += blockDim.x) s += (double)mu[m] * (double)W[(int64_t)j * d + m];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ double ps[8];
+  if ((threadIdx.x & 31) == 0) ps[threadIdx.x >> 5] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 8; ++w) t += ps[w];
+    zoff[j] = (float)t;
+  }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+PcaGeom pca_geom(int64_t N, int d, int r) {
+  PcaGeom g;
+  g.N = N;
+  g.d = d;
+  g.r = r;
+  g.n = d + (d & 1);
+  g.ldn = (N + 7) / 8 * 8;
+  g.mi = (d + kBM - 1) / kBM;
+  g.ntiles = g.mi * (g.mi + 1) / 2;
+  // row ranges: about 8 units per SM over all tiles (152 SMs assumed for
+  // the sizing only), each range a multiple of kCovSub rows
+  int64_t ranges = (8 * 152 + g.ntiles - 1) / g.ntiles;
+  const int64_t subs = (N + kCovSub - 1) / kCovSub;
+  if (ranges > subs) ranges = subs > 0 ? subs : 1;
+  g.R = (subs + ranges - 1) / ranges * kCovSub;
+  g.nchunks = (N + g.R - 1) / g.R;
+  g.nslabs = (N + kColSlab - 1) / kColSlab;
+  return g;
+}
+
+cudaError_t launch_pca_mean(const float *X, const PcaGeom &g, int64_t ldx, double *slab_sums, double *mean64,
+                            float *mean32, cudaStream_t s) {
+  const dim3 grid((unsigned)((g.d + kColThreads - 1) / kColThreads), (unsigned)g.nslabs);
+  pca_colsum_kernel<<<grid, kColThreads, 0, s>>>(X, g.N, g.d, ldx, slab_sums);
+  pca_mean_kernel<<<(g.d + 255) / 256, 256, 0, s>>>(slab_sums, g.nslabs, g.N, g.d, mean64, mean32);
+  count_launch(2);
+  return cudaGetLastError();
+}
+
+int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *mean32, __nv_bfloat16 *yh,
+                   __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s) {
+  const bool vec = (reinterpret_cast<uintptr_t>(X) & 15u) == 0 && ldx % 4 == 0;
+  const dim3 tg((unsigned)((g.N + 63) / 64), (unsigned)((g.d + 63) / 64));
+  if (vec)
+    pca_split_t_kernel<true><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.ldn, yh, yl);
+  else
+    pca_split_t_kernel<false><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.ldn, yh, yl);
+  count_launch();
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pca: split");
+  CUtensorMap mH, mL;
+  int rc;
+  if ((rc = make_bf16_map(&mH, yh, (uint64_t)g.d, (uint64_t)g.N, (uint64_t)g.ldn, kBM)) != HME_OK) return rc;
+  if ((rc = make_bf16_map(&mL, yl, (uint64_t)g.d, (uint64_t)g.N, (uint64_t)g.ldn, kBM)) != HME_OK) return rc;
+  CovParams p;
+  p.N = g.N;
+  p.R = g.R;
+  p.mi = g.mi;
+  p.ntiles = g.ntiles;
+  p.nunits = g.nchunks * g.ntiles;
+  p.part = part;
+  p.hdr = hdr;
+  p.limit_ns = wait_limit_ns();
+  const size_t smem = 1024 + (size_t)kCovStages * kCovStageBytes + 256;
+  e = cudaFuncSetAttribute(pca_cov_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return cuda_fail(e, "pca: covariance smem");
+  int grid = num_sms();
+  if (grid > p.nunits) grid = (int)p.nunits;
+  pca_cov_kernel<<<grid, kCovThreads, smem, s>>>(mH, mL, p);
+  count_launch();
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pca: covariance kernel launch");
+  e = cudaMemsetAsync(A, 0, (size_t)g.n * g.n * sizeof(float), s);
+  if (e != cudaSuccess) return cuda_fail(e, "pca: clear A");
+  const dim3 rg((unsigned)((g.d + 31) / 32), (unsigned)((g.d + 31) / 32));
+  pca_cov_reduce_kernel<<<rg, 256, 0, s>>>(part, g.nchunks, g.ntiles, g.mi, g.d, g.n, g.N, cov, A);
+  count_launch();
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pca: reduce");
+  return HME_OK;
+}
+
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1, double *acc, int32_t *order,
+                   float *W, float *variances, int *sweeps_out, cudaStream_t s) {
+  const int n = g.n;
+  pca_identity_kernel<<<(unsigned)(((int64_t)n * n + 255) / 256), 256, 0, s>>>(V0, n);
+  count_launch();
+  const int np = n / 2;
+  const int a_side = (np + kJacSide - 1) / kJacSide;
+  const int v_side = (np + 31) / 32;
+  const int blocks = a_side * a_side + v_side * ((n + 7) / 8);
+  float *A[2] = {A0, A1}, *V[2] = {V0, V1};
+  int cur = 0, sweep = 0;
+  bool converged = false;
+  const double tol2 = 0x1p-44;  // (2^-22)^2
+  double prev_off = -1.0;
+  for (sweep = 1; sweep <= kJacobiMaxSweeps && !converged; ++sweep) {
+    for (int t = 0; t < n - 1; ++t) {
+      jacobi_round_kernel<<<blocks, 256, 0, s>>>(A[cur], V[cur], A[cur ^ 1], V[cur ^ 1], n, a_side, v_side);
+      cur ^= 1;
+    }
+    count_launch(n - 1);
+    cudaError_t e = cudaMemsetAsync(acc, 0, 2 * sizeof(double), s);
+    if (e != cudaSuccess) return cuda_fail(e, "pca: clear norms");
+    int nb = (int)(((int64_t)n * n + 255) / 256);
+    if (nb > 4 * num_sms()) nb = 4 * num_sms();
+    jacobi_offnorm_kernel<<<nb, 256, 0, s>>>(A[cur], n, acc);
+    count_launch();
+    double h[2];
+    e = cudaMemcpyAsync(h, acc, sizeof(h), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "pca: Jacobi sweep");
+    // converged: off(A) <= 2^-22 ||A||_F, or off(A) already below 2^-16 ||A||_F
+    // and no longer halving from one sweep to the next (the fp32 floor)
+    converged = h[0] <= tol2 * (h[0] + h[1]) ||
+                (prev_off >= 0.0 && h[0] >= 0.25 * prev_off && h[0] <= 0x1p-32 * (h[0] + h[1]));
+    prev_off = h[0];
+  }
+  if (sweeps_out) *sweeps_out = sweep - 1;
+  if (!converged) return fail(HME_EINTERNAL, "pca: Jacobi did not converge in %d sweeps", kJacobiMaxSweeps);
+  // n - 1 rounds per sweep restore the slot order, so slot j holds index j
+  const size_t rank_smem = (size_t)g.d * sizeof(float);
+  if (rank_smem > 48 * 1024) {
+    cudaError_t ea = cudaFuncSetAttribute(pca_rank_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rank_smem);
+    if (ea != cudaSuccess) return cuda_fail(ea, "pca: rank smem");
+  }
+  pca_rank_kernel<<<1, 1024, rank_smem, s>>>(A[cur], n, g.d, g.r, order, variances);
+  pca_components_kernel<<<g.r, 256, 0, s>>>(V[cur], n, g.d, order, W);
+  count_launch(2);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "pca: components");
+  return HME_OK;
+}
+
+cudaError_t launch_pca_zoff(const float *mean, const float *W, int d, int r, int Kp, float *zoff, cudaStream_t s) {
+  pca_zoff_kernel<<<Kp, 256, 0, s>>>(mean, W, d, r, zoff);
+  count_launch();
+  return cudaGetLastError();
+}
+
+}  // namespace hme

@@ -18,7 +18,7 @@ import torch
 
 HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6)
 HME_F32, HME_BF16 = 0, 1
-HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST, HME_OP_STREAM = range(6)
+HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST, HME_OP_STREAM, HME_OP_PCA = range(7)
 HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
 HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED, HME_ASSIGN_PREPARE_OUT = 0, 1, 2
 
@@ -69,6 +69,12 @@ def lib():
         L.hme_kmeans_stream.argtypes = [p, i64, i32, i64, i32, i32, i32, i64, p, p, p, p, p, p, p, sz, p]
         L.hme_tag_cluster_hist.restype = ctypes.c_int
         L.hme_tag_cluster_hist.argtypes = [p, p, p, i64, i32, i32, p, p, p, sz, p]
+        L.hme_pca_covariance.restype = ctypes.c_int
+        L.hme_pca_covariance.argtypes = [p, i64, i32, i64, i32, p, p, p, sz, p]
+        L.hme_pca_fit.restype = ctypes.c_int
+        L.hme_pca_fit.argtypes = [p, i64, i32, i64, i32, i32, p, p, p, p, p, sz, p]
+        L.hme_pca_transform.restype = ctypes.c_int
+        L.hme_pca_transform.argtypes = [p, i64, i32, i64, i32, p, p, i32, p, i64, p, sz, p]
         L.hme_launch_count.restype = i64
         L.hme_launch_count.argtypes = []
         L.hme_debug_bounded_wait.restype = ctypes.c_int
@@ -209,6 +215,45 @@ def hme_tag_cluster_hist(offsets: torch.Tensor, tag_off: torch.Tensor, tags: tor
     w, wb = _ws(ws)
     _check(lib().hme_tag_cluster_hist(_ptr(offsets), _ptr(tag_off), _ptr(tags), N, K, V, _ptr(counts_out),
                                       _ptr(sparsity_out), w, wb, _stream(stream)), "hme_tag_cluster_hist")
+
+
+def hme_pca_covariance(X: torch.Tensor, mean_out: torch.Tensor, cov_out: torch.Tensor, ws: torch.Tensor,
+                       stream=None):
+    """Section 4.2 PCA: column mean (fp64, d) and covariance (fp64, d x d) of fp32 features."""
+    N, d, ldx, dt = _features(X)
+    if not (mean_out.is_contiguous() and cov_out.is_contiguous()):
+        raise ValueError("mean_out and cov_out must be contiguous")
+    w, wb = _ws(ws)
+    _check(lib().hme_pca_covariance(_ptr(X), N, d, ldx, dt, _ptr(mean_out), _ptr(cov_out), w, wb, _stream(stream)),
+           "hme_pca_covariance")
+
+
+def hme_pca_fit(X: torch.Tensor, r: int, mean_out: torch.Tensor, components_out: torch.Tensor, ws: torch.Tensor,
+                variances_out: Optional[torch.Tensor] = None, stream=None) -> int:
+    """Section 4.2 PCA: mean (fp32, d), r leading components (fp32, r x d) and their variances; returns the
+    Jacobi sweeps made (the call synchronises the stream once per sweep)."""
+    N, d, ldx, dt = _features(X)
+    if not (mean_out.is_contiguous() and components_out.is_contiguous()):
+        raise ValueError("mean_out and components_out must be contiguous")
+    w, wb = _ws(ws)
+    sweeps = ctypes.c_int32(0)
+    _check(lib().hme_pca_fit(_ptr(X), N, d, ldx, dt, r, _ptr(mean_out), _ptr(components_out), _ptr(variances_out),
+                             ctypes.byref(sweeps), w, wb, _stream(stream)), "hme_pca_fit")
+    return int(sweeps.value)
+
+
+def hme_pca_transform(X: torch.Tensor, mean: torch.Tensor, components: torch.Tensor, Z_out: torch.Tensor,
+                      ws: torch.Tensor, stream=None):
+    """Z_out[i, j] = components[j] . (x_i - mean), fp32 (N x r)."""
+    N, d, ldx, dt = _features(X)
+    r = components.shape[0]
+    if Z_out.dim() != 2 or Z_out.stride(1) != 1:
+        raise ValueError("Z_out must be a 2-D tensor with unit column stride")
+    if not (components.is_contiguous() and mean.is_contiguous()):
+        raise ValueError("components (r x d) and mean (d) must be contiguous")
+    w, wb = _ws(ws)
+    _check(lib().hme_pca_transform(_ptr(X), N, d, ldx, dt, _ptr(mean), _ptr(components), r, _ptr(Z_out),
+                                   max(Z_out.stride(0), r), w, wb, _stream(stream)), "hme_pca_transform")
 
 
 def hme_partition_noalloc(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_out: torch.Tensor,

@@ -108,3 +108,39 @@ def test_tag_hist_host_validation(lib):
         args = list(ok)
         args[i] = bad
         assert g(*args) != 0
+
+
+def test_pca_host_validation(lib):
+    f = lib.hme_workspace_bytes
+    f.restype = ctypes.c_size_t
+    f.argtypes = [ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32]
+    full = f(6, 1_000_000, 2048, 256, 0)
+    assert full >= 2 * 1_000_000 * 2048 * 2  # the transposed bf16 split of the centred rows
+    assert 0 < f(6, 0, 2048, 256, 0) < full  # N = 0: transform only
+    assert f(6, 100, 16, 17, 0) == 0  # r > d
+    assert f(6, 100, 16, 4, 1) == 0  # bf16 features are not taken
+    p, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    g = lib.hme_pca_fit
+    g.restype = ctypes.c_int
+    g.argtypes = [p, i64, i32, i64, i32, i32, p, p, p, p, p, ctypes.c_size_t, p]
+    ok = [p(256), 100, 16, 16, 0, 4, p(256), p(256), None, None, p(256), 1 << 30, None]
+    for i, bad in [(1, 0), (4, 1), (5, 0), (5, 17), (3, 8), (6, None), (7, None), (10, None), (10, p(300))]:
+        args = list(ok)
+        args[i] = bad
+        assert g(*args) == 1, (i, bad)  # HME_EINVAL before any CUDA call
+    args = list(ok)
+    args[11] = 64
+    assert g(*args) == 2  # workspace too small
+    t = lib.hme_pca_transform
+    t.restype = ctypes.c_int
+    t.argtypes = [p, i64, i32, i64, i32, p, p, i32, p, i64, p, ctypes.c_size_t, p]
+    tok = [p(256), 100, 300, 300, 0, p(256), p(256), 16, p(256), 16, p(256), 1 << 30, None]
+    for i, bad in [(7, 257), (9, 8), (0, p(260)), (3, 302), (8, None)]:  # r > 256, ldz < r, misaligned X / ldx
+        args = list(tok)
+        args[i] = bad
+        assert t(*args) == 1, (i, bad)
+    c = lib.hme_pca_covariance
+    c.restype = ctypes.c_int
+    c.argtypes = [p, i64, i32, i64, i32, p, p, p, ctypes.c_size_t, p]
+    assert c(p(256), 0, 4, 4, 0, p(256), p(256), p(256), 1 << 20, None) == 1  # N = 0
+    assert c(p(256), 10, 4, 4, 0, None, p(256), p(256), 1 << 20, None) == 1
