@@ -45,6 +45,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-stream", action="store_true", help="skip the streamed-from-host diagnostic")
+    ap.add_argument("--no-pca", action="store_true", help="skip the PCA diagnostic")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
     return ap.parse_args()
 
@@ -359,6 +360,47 @@ def run_ours(args, w):
                         "chunk_rows": chunk, "host_to_device_gbs": its * X.numel() * w.elem_bytes / (st_ms / 1000) / 1e9}
         del Xpin, wst
 
+    # outside the timed steps: the Section 4.2 PCA of the same features (fp32
+    # workloads): covariance on the tensor cores, Jacobi eigensolver, projection
+    pca_stats = None
+    if not args.no_pca and w.dtype == "f32":
+        r = min(256, d)
+        wsp = hme.workspace(hme.HME_OP_PCA, N, d, r, dt, device=dev)
+        mu64 = torch.empty(d, dtype=torch.float64, device=dev)
+        cov = torch.empty(d, d, dtype=torch.float64, device=dev)
+        mu = torch.empty(d, dtype=torch.float32, device=dev)
+        comps = torch.empty(r, d, dtype=torch.float32, device=dev)
+        var = torch.empty(r, dtype=torch.float32, device=dev)
+        Z = torch.empty(N, r, dtype=torch.float32, device=dev)
+
+        def timed(fn, reps):
+            fn()  # warm-up
+            q0 = torch.cuda.Event(enable_timing=True)
+            q1 = torch.cuda.Event(enable_timing=True)
+            q0.record(stream)
+            for _ in range(reps):
+                out = fn()
+            q1.record(stream)
+            torch.cuda.synchronize(dev)
+            return q0.elapsed_time(q1) / reps, out
+
+        cov_ms, _ = timed(lambda: hme.hme_pca_covariance(X, mu64, cov, wsp), 3)
+        fit_ms, sweeps = timed(lambda: hme.hme_pca_fit(X, r, mu, comps, wsp, var), 1)
+        tr_ms, _ = timed(lambda: hme.hme_pca_transform(X, mu, comps, Z, wsp), 5)
+        if hme.hme_sync_status(wsp) != hme.HME_OK:
+            raise RuntimeError(f"pca: {hme.hme_last_error()}")
+        mi = (d + 127) // 128
+        issued = 3 * 2.0 * N * 128 * 128 * mi * (mi + 1) // 2  # three split products on the upper-triangle tiles
+        pca_stats = {"components": r, "fit_ms": fit_ms, "covariance_ms": cov_ms, "jacobi_ms_approx": fit_ms - cov_ms,
+                     "jacobi_sweeps": sweeps,
+                     "covariance_tflops_gram": 2.0 * N * d * d / (cov_ms / 1000) / 1e12,
+                     "covariance_tflops_tensor_issued": issued / (cov_ms / 1000) / 1e12,
+                     "transform_ms": tr_ms,
+                     "transform_tflops": 2.0 * N * d * r / (tr_ms / 1000) / 1e12,
+                     "transform_gbs": (N * d * 4 + N * r * 4) / (tr_ms / 1000) / 1e9,
+                     "variance_captured": float(var.sum().item()) / float(torch.diagonal(cov).sum().item())}
+        del wsp, cov, Z
+
     tag_stats = None
     if w.tags:  # Section 4.5 statistics of the final shares, outside the timed steps
         V = w.tag_vocab
@@ -473,6 +515,7 @@ def run_ours(args, w):
             "rescored_rows_last_assign": rescored,
             "moved_rows_last_update": moved,
             "tag_statistics": tag_stats,
+            "pca": pca_stats,
             "streamed_from_host": stream_stats,
             "clocks": ck,
         }

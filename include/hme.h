@@ -321,9 +321,10 @@ HME_API int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, i
  *   triangles).  The centred values y = x - fp32(mu) are split into bf16
  *   y = yh + yl (|y - yh - yl| <= 2^-16 |y|) and the products
  *   yh yh' + yh yl' + yl yh' are summed on the tensor cores in fp32 over 512
- *   rows at a time (96 accumulation steps), those sums in fp64, so that each
- *   entry is within (3 * 2^-16 + 98 * 2^-23) (1/N) sum_i (|y_ia| + |mu_a|)
- *   (|y_ib| + |mu_b|) of the exact value (2^-23 per accumulation step: one
+ *   rows at a time (96 accumulation steps), up to 16 of those sums in fp32
+ *   (round to nearest), and those in fp64, so that each entry is within
+ *   (3 * 2^-16 + 98 * 2^-23 + 18 * 2^-24) (1/N) sum_i (|y_ia| + |mu_a|)
+ *   (|y_ib| + |mu_b|) of the exact value (2^-23 per tensor-core step: one
  *   ulp, whatever the accumulator's rounding).  Requires N >= 1.
  *
  * hme_pca_fit -- the covariance as above, then its eigendecomposition by

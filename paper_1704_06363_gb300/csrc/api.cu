@@ -270,7 +270,7 @@ int clear_header(void *ws, cudaStream_t s) {
 // PCA fit (hme_pca_covariance / hme_pca_fit): slab sums, mean, transposed
 // split, covariance partial tiles, the Jacobi matrices and small scratch.
 struct PcaLayout {
-  size_t slab, mean64, mean32, yh, yl, part, A0, A1, V0, V1, acc, order, total;
+  size_t slab, mean64, mean32, yh, yl, part, A0, V0, rot0, rot1, acc, order, total;
 };
 PcaLayout pca_layout(int64_t N, int d, int r) {
   const PcaGeom g = pca_geom(N, d, r);
@@ -290,9 +290,9 @@ PcaLayout pca_layout(int64_t N, int d, int r) {
   L.part = take((size_t)g.nchunks * g.ntiles * kBM * kBM * 8);
   const size_t nn = (size_t)g.n * g.n * 4;
   L.A0 = take(nn);
-  L.A1 = take(nn);
   L.V0 = take(nn);
-  L.V1 = take(nn);
+  L.rot0 = take((size_t)(g.n / 2) * 16);
+  L.rot1 = take((size_t)(g.n / 2) * 16);
   L.acc = take(16);
   L.order = take((size_t)r * 4);
   L.total = align_up(off, 256);
@@ -575,6 +575,7 @@ int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
                 float *components_out, float *variances_out, int32_t *sweeps_out, void *ws, size_t ws_bytes,
                 void *stream) {
   HME_TRY(check_pca(X, N, d, ldx, dtype, r, 1));
+  if (d > kPcaMaxFitD) return fail(HME_EINVAL, "d = %d: hme_pca_fit takes d <= %d", d, kPcaMaxFitD);
   if (!mean_out || !components_out) return fail(HME_EINVAL, "mean_out / components_out is NULL");
   const PcaLayout L = pca_layout(N, d, r);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
@@ -588,8 +589,8 @@ int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
                          at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), nullptr, at<float>(ws, L.A0),
                          at<Header>(ws, 0), s));
   int sweeps = 0;
-  const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.A1), at<float>(ws, L.V0), at<float>(ws, L.V1),
-                                at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,
+  JacRotBuf rb{at<void>(ws, L.rot0), at<void>(ws, L.rot1)};
+  const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.V0), rb, at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,
                                 &sweeps, s);
   if (sweeps_out) *sweeps_out = sweeps;
   if (rc != HME_OK) return rc;

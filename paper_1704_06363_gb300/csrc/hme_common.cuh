@@ -207,8 +207,12 @@ int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *m
                    __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s);
 // Jacobi sweeps on A0 (synchronises s once per sweep), then the r leading
 // components (rows of W, r x d) and their variances (may be null)
-int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1, double *acc, int32_t *order,
-                   float *W, float *variances, int *sweeps_out, cudaStream_t s);
+struct JacRotBuf {
+  void *r0, *r1;  // two rotation tables of 16 * (n / 2) bytes (this round's, the next round's)
+};
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, JacRotBuf rotbuf, double *acc, int32_t *order, float *W,
+                   float *variances, int *sweeps_out, cudaStream_t s);
+constexpr int kPcaMaxFitD = 8192;  // int32 item indices of a Jacobi round: (n/2)^2 + n (n/2) < 2^31
 cudaError_t launch_pca_zoff(const float *mean, const float *W, int d, int r, int Kp, float *zoff, cudaStream_t s);
 cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
 int64_t kpp_candidates(int64_t N, int K, int method);

@@ -14,23 +14,22 @@
 //   pca_cov         tcgen05 (kind::f16, fp32 accumulate in TMEM): work units
 //                   are (row range, 128 x 128 tile (i <= j) of the upper
 //                   triangle); a unit accumulates yh.yh' + yh.yl' + yl.yh' in
-//                   TMEM over kCovSub rows at a time (short fp32 sums), and its
-//                   epilogue adds each such sub-result into the unit's fp64
-//                   partial tile (read-modify-write, L2-resident) while the
-//                   MMAs of the next sub-range run in the other accumulator;
+//                   TMEM over kCovSub rows at a time (short fp32 sums), its
+//                   epilogue adds each such sub-result into fp32 registers
+//                   (round to nearest) while the MMAs of the next sub-range run
+//                   in the other accumulator, and every kCovFlush sub-ranges
+//                   adds the registers into the unit's fp64 partial tile;
 //   pca_cov_reduce  the partial tiles added in range order in fp64, / N: the
 //                   covariance (fp64, both triangles) and A (fp32, order n = d
 //                   rounded up to even, padding row and column zero);
 //   Jacobi          cyclic two-sided Jacobi on A, n/2 disjoint rotations per
 //                   round (circle-method ordering: n - 1 rounds meet every pair
-//                   once).  One kernel per round reads A and V (the eigenvector
-//                   estimate, V <- V J) and writes them with the rotations
-//                   applied and the rows/columns moved to the next round's
-//                   slots, so that every pair is two adjacent slots and every
-//                   access is row-contiguous; the matrices (4 n^2 floats, 64 MB
-//                   at d = 2048) stay in L2.  After a sweep the slots are back
-//                   in their original order; sweeps repeat until
-//                   off(A) <= 2^-22 ||A||_F;
+//                   once).  One kernel per round updates A and V (the
+//                   eigenvector estimate, V <- V J) in place, each 2 x 2 block
+//                   by one thread; the two matrices (2 n^2 floats, 32 MB at
+//                   d = 2048) stay in L2, and the next round's rotations are
+//                   formed by the threads that produce its pivots.  Sweeps
+//                   repeat until off(A) <= 2^-22 ||A||_F;
 //   pca_rank        eigenvalues diag(A) ranked (decreasing, ties to the lower
 //                   index), the padding slot excluded;
 //   pca_components  the leading r columns of V, normalised, with the sign rule.
@@ -44,12 +43,12 @@ namespace {
 
 constexpr int kColThreads = 256;
 constexpr int kColSlab = 2048;  // rows per column-sum block
-constexpr int kCovThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kCovThreads = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue (two per TMEM lane quarter)
+constexpr int kCovHalf = kBM / 2;  // accumulator columns per epilogue warp
 constexpr int kCovStages = 3;
 constexpr uint32_t kCovOpBytes = kBM * kBK * 2;  // 128 rows x 64 bf16 = 16 KB
 constexpr uint32_t kCovStageBytes = 4 * kCovOpBytes;  // A hi, A lo, B hi, B lo
 constexpr uint32_t kCovTmemCols = 256;  // two 128-column accumulators
-constexpr int kJacSide = 16;  // pair-blocks per side of an A tile (32 x 32 elements)
 constexpr uint32_t kWhereCovProducer = 11, kWhereCovMma = 12, kWhereCovEpi = 13;
 
 // ---------------------------------------------------------------------------
@@ -162,6 +161,7 @@ struct CovParams {
   uint64_t limit_ns;
 };
 constexpr int kSubKb = (int)(kCovSub / kBK);  // k-blocks per TMEM accumulation
+constexpr int kCovFlush = 16;                   // sub-range sums per fp32 register accumulation
 
 // tile t of the upper triangle, enumerated row by row: (i, j), i <= j
 __device__ __forceinline__ void cov_tile(int t, int mi, int &i, int &j) {
@@ -199,7 +199,7 @@ __global__ void __launch_bounds__(kCovThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&tempty[a]), 8);
     }
     mbar_init(smem_u32(drain), 1);
     fence_mbar_init();
@@ -298,14 +298,23 @@ __global__ void __launch_bounds__(kCovThreads, 1)
       }
     }
   } else {
-    // epilogue: accumulator row (TMEM lane) -> one row of the partial tile
+    // epilogue: accumulator row (TMEM lane), half of its columns -> the partial tile
     const int q = warp & 3;
     const int row = q * 32 + lane;
+    const int col0 = ((warp - 2) >> 2) * kCovHalf;
+    // Each sub-range sum (one TMEM accumulation) is added into fp32 registers
+    // (round to nearest); every kCovFlush sub-ranges, and at the end of the
+    // unit, the registers go to the unit's fp64 partial row.
     uint32_t acc_it = 0;
     bool ok = true;
+    float acc[kCovHalf];
     for (int64_t u = blockIdx.x; u < p.nunits && ok; u += gridDim.x) {
       const int nkb = kblocks(u / p.ntiles);
-      double *dst = p.part + u * (int64_t)(kBM * kBM) + (int64_t)row * kBM;
+      double *dst = p.part + u * (int64_t)(kBM * kBM) + (int64_t)row * kBM + col0;
+      bool first_flush = true;
+      int since = 0;
+#pragma unroll
+      for (int c = 0; c < kCovHalf; ++c) acc[c] = 0.0f;
       for (int kb0 = 0; kb0 < nkb; kb0 += kSubKb, ++acc_it) {
         const uint32_t a = acc_it & 1u;
         if (!mbar_wait_bounded(smem_u32(&tfull[a]), (acc_it >> 1) & 1u, p.limit_ns, p.hdr, kWhereCovEpi)) {
@@ -313,26 +322,39 @@ __global__ void __launch_bounds__(kCovThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t taddr = tmem_base + a * (uint32_t)kBM + ((uint32_t)(q * 32) << 16);
-        uint32_t r[16];
-        for (int c = 0; c < kBM; c += 16) {
-          tmem_ld16(taddr + (uint32_t)c, r);
-          tmem_ld_wait(r);
-          double2 *d2 = reinterpret_cast<double2 *>(dst + c);
+        const uint32_t taddr = tmem_base + a * (uint32_t)kBM + (uint32_t)col0 + ((uint32_t)(q * 32) << 16);
+        uint32_t r0[16], r1[16];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const double x0 = (double)__uint_as_float(r[2 * e]), x1 = (double)__uint_as_float(r[2 * e + 1]);
-            if (kb0 == 0) {
-              d2[e] = make_double2(x0, x1);
-            } else {
-              const double2 o = d2[e];
-              d2[e] = make_double2(o.x + x0, o.y + x1);
-            }
+        for (int c = 0; c < kCovHalf; c += 32) {
+          tmem_ld16(taddr + (uint32_t)c, r0);
+          tmem_ld16(taddr + (uint32_t)(c + 16), r1);
+          tmem_ld_wait(r0);
+          tmem_ld_wait(r1);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            acc[c + e] += __uint_as_float(r0[e]);
+            acc[c + 16 + e] += __uint_as_float(r1[e]);
           }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
+        if (++since == kCovFlush || kb0 + kSubKb >= nkb) {
+#pragma unroll
+          for (int c = 0; c < kCovHalf; c += 2) {
+            double2 *d2 = reinterpret_cast<double2 *>(dst + c);
+            const double x0 = (double)acc[c], x1 = (double)acc[c + 1];
+            if (first_flush) {
+              *d2 = make_double2(x0, x1);
+            } else {
+              const double2 o = *d2;
+              *d2 = make_double2(o.x + x0, o.y + x1);
+            }
+            acc[c] = acc[c + 1] = 0.0f;
+          }
+          first_flush = false;
+          since = 0;
+        }
       }
     }
   }
@@ -374,18 +396,40 @@ __global__ void __launch_bounds__(256) pca_cov_reduce_kernel(const double *__res
 // ---------------------------------------------------------------------------
 // Jacobi
 // ---------------------------------------------------------------------------
-// Circle-method ordering: slot 0 holds a fixed index; the other n - 1 indices
-// sit on a list whose position 0 is slot 1, positions 1 .. n/2-1 the even
-// slots 2, 4, .. and positions n/2 .. n-2 the odd slots n-1, n-3, .. 3.  Each
-// round pairs slots (2P, 2P + 1); between rounds every listed index moves one
-// position down the list (cyclically), so after n - 1 rounds each pair has met
-// once and every index is back in its slot.
-__device__ __forceinline__ int jac_next(int slot, int n) {
-  if (slot == 0) return 0;
-  const int pos = slot == 1 ? 0 : ((slot & 1) == 0 ? (slot >> 1) : n - 1 - ((slot - 1) >> 1));
-  int np = pos + n - 2;
-  if (np >= n - 1) np -= n - 1;
-  return np == 0 ? 1 : (np <= (n >> 1) - 1 ? 2 * np : 2 * (n - 1 - np) + 1);
+// Circle-method ordering on fixed positions (no data movement): with
+// m = n - 1, round t in [0, m) pairs index 0 with 1 + t (pair 0) and, for
+// k = 1 .. n/2 - 1, p_k = 1 + (t + k) mod m with q_k = 1 + (t - k) mod m; over
+// m rounds every two indices meet once.  Consecutive pairs k touch ascending
+// (p) and descending (q) consecutive indices, so a warp's accesses to a row
+// stay contiguous.
+__device__ __forceinline__ int jac_p(int k, int t, int m) {
+  if (k == 0) return 0;
+  const int x = t + k;
+  return 1 + (x >= m ? x - m : x);
+}
+__device__ __forceinline__ int jac_q(int k, int t, int m) {
+  if (k == 0) return 1 + t;
+  const int x = t - k;
+  return 1 + (x < 0 ? x + m : x);
+}
+// pair of index x in round t, and whether x is its p member
+__device__ __forceinline__ int jac_pair_of(int x, int t, int m, bool &is_p) {
+  if (x == 0) {
+    is_p = true;
+    return 0;
+  }
+  int kk = x - 1 - t;
+  if (kk < 0) kk += m;
+  if (kk == 0) {
+    is_p = false;
+    return 0;
+  }
+  if (kk <= (m - 1) / 2) {
+    is_p = true;
+    return kk;
+  }
+  is_p = false;
+  return m - kk;
 }
 
 // The rotation of one pair (Rutishauser's form): t = tan(phi) is the smaller
@@ -394,98 +438,141 @@ __device__ __forceinline__ int jac_next(int slot, int n) {
 // and q is u - s (v + tau u), v + s (u - tau v) with s = sin(phi), tau =
 // tan(phi / 2), which keeps the norm of (u, v) to second order in s even when
 // cos(phi) rounds to 1.  Entries with |a_pq| <= 2^-23 sqrt(|a_pp| |a_qq|) are
-// left alone.  Not inlined: every block that needs a pair's rotation gets the
-// same bits from the same instructions.
-struct JacRot {
-  float s, tau, dp, dq;  // dp, dq: the new diagonal entries
-};
-__device__ __noinline__ JacRot jac_rot(float app, float aqq, float apq) {
-  JacRot r{0.0f, 0.0f, app, aqq};
+// left alone.  Returns (s, tau, dp, dq), dp and dq the new diagonal entries.
+// Each rotation is computed once per round, by one thread.
+__device__ float4 jac_rot4(float app, float aqq, float apq) {
+  float4 r = make_float4(0.0f, 0.0f, app, aqq);
   if (apq != 0.0f && fabsf(apq) > 0x1p-23f * sqrtf(fabsf(app)) * sqrtf(fabsf(aqq))) {
     const float theta = (aqq - app) / (2.0f * apq);
     const float at = fabsf(theta);
     float t = at > 0x1p20f ? 0.5f / at : 1.0f / (at + sqrtf(at * at + 1.0f));
     t = copysignf(t, theta);
     const float c = 1.0f / sqrtf(t * t + 1.0f);
-    r.s = t * c;
-    r.tau = r.s / (1.0f + c);
-    r.dp = app - t * apq;
-    r.dq = aqq + t * apq;
+    r.x = t * c;
+    r.y = r.x / (1.0f + c);
+    r.z = app - t * apq;
+    r.w = aqq + t * apq;
   }
   return r;
 }
 
-__device__ __forceinline__ JacRot jac_pair(const float *A, int n, int P) {
-  const int64_t p = 2 * P;
-  return jac_rot(A[p * n + p], A[(p + 1) * n + p + 1], A[p * n + p + 1]);
+__global__ void jacobi_rot_init_kernel(const float *__restrict__ A, int n, float4 *__restrict__ rot) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  const int m = n - 1;
+  if (k >= (n >> 1)) return;
+  const int64_t p = jac_p(k, 0, m), q = jac_q(k, 0, m);
+  rot[k] = jac_rot4(A[p * n + p], A[q * n + q], A[p * n + q]);
 }
 
-// Blocks [0, a_blocks): 32 x 32 tiles of A (a thread per 2 x 2 pair block);
-// the rest: 8 rows x 32 column pairs of V.
-__global__ void __launch_bounds__(256) jacobi_round_kernel(const float *__restrict__ A, const float *__restrict__ V,
-                                                           float *__restrict__ An, float *__restrict__ Vn, int n,
-                                                           int a_side, int v_side) {
-  __shared__ float rs[2][32][2];  // (s, tau) of the tile's row pairs [0] and column pairs [1]
-  __shared__ float rd[kJacSide][2];
-  const int np = n >> 1;
-  const int a_blocks = a_side * a_side;
-  if ((int)blockIdx.x < a_blocks) {
-    const int P0 = (blockIdx.x / a_side) * kJacSide, Q0 = (blockIdx.x % a_side) * kJacSide;
-    if (threadIdx.x < 2 * kJacSide) {
-      const int w = threadIdx.x / kJacSide, k = threadIdx.x % kJacSide;
-      const int P = (w ? Q0 : P0) + k;
-      if (P < np) {
-        const JacRot r = jac_pair(A, n, P);
-        rs[w][k][0] = r.s;
-        rs[w][k][1] = r.tau;
-        if (w == 0) {
-          rd[k][0] = r.dp;
-          rd[k][1] = r.dq;
+// One round t, in place.  A warp owns one row pair of A (rows rotated by
+// that pair) or one row pair of V, and 32 x kJacLPT column pairs (lane j takes
+// column pairs L0 + j + 32 l, so every access of the warp is a contiguous run
+// of a row); each 2 x 2 block of A gets both rotations (the diagonal block
+// K = L becomes diag(dp, dq)), V gets the column rotations (V <- V J).  Every
+// entry is read and written by one thread, so no two blocks conflict.  The
+// rotation table of the round comes in (read through L1); the next round's is
+// written by the owners of its pivots: the entry (a, b) with a the p member
+// and b the q member of a next-round pair lies in one off-diagonal block of
+// this round, whose thread forms the rotation from the new entry and the new
+// diagonal entries dp / dq of a's and b's pairs.
+constexpr int kJacThreads = 256;
+constexpr int kJacLPT = 4;  // column pairs per thread
+__global__ void __launch_bounds__(kJacThreads) jacobi_round_kernel(float *__restrict__ A, float *__restrict__ V,
+                                                                   const float4 *__restrict__ rot,
+                                                                   float4 *__restrict__ rot_next, int n, int t) {
+  const int np = n >> 1, m = n - 1;
+  const int tn = t + 1 == m ? 0 : t + 1;
+  const int chunks = (np + 32 * kJacLPT - 1) / (32 * kJacLPT);
+  const int warps_a = np * chunks, warps_total = warps_a + n * chunks;
+  const int lane = threadIdx.x & 31;
+  const int wstride = (int)((gridDim.x * blockDim.x) >> 5);
+  for (int w = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); w < warps_total; w += wstride) {
+    if (w < warps_a) {
+      const int K = w / chunks;
+      const int L0 = (w - K * chunks) * 32 * kJacLPT + lane;
+      const int pK = jac_p(K, t, m), qK = jac_q(K, t, m);
+      const float4 rk = __ldg(rot + K);
+      // next-round partner of each row index that is a p member next round (else -1)
+      bool ap0, ap1;
+      const int ka0 = jac_pair_of(pK, tn, m, ap0), ka1 = jac_pair_of(qK, tn, m, ap1);
+      const int part0 = ap0 ? jac_q(ka0, tn, m) : -1, part1 = ap1 ? jac_q(ka1, tn, m) : -1;
+      float *rp = A + (int64_t)pK * n, *rq = A + (int64_t)qK * n;
+      // all loads of the thread's blocks first (they are in flight together),
+      // then the rotations and stores
+      float a[kJacLPT][4];
+      float4 rl[kJacLPT];
+      int pl[kJacLPT], ql[kJacLPT];
+#pragma unroll
+      for (int l = 0; l < kJacLPT; ++l) {
+        const int L = L0 + 32 * l;
+        pl[l] = jac_p(L, t, m);
+        ql[l] = jac_q(L, t, m);
+        if (L < np) {
+          rl[l] = __ldg(rot + L);
+          a[l][0] = rp[pl[l]];
+          a[l][1] = rp[ql[l]];
+          a[l][2] = rq[pl[l]];
+          a[l][3] = rq[ql[l]];
         }
       }
-    }
-    __syncthreads();
-    const int ty = threadIdx.x / kJacSide, tx = threadIdx.x % kJacSide;
-    const int P = P0 + ty, Q = Q0 + tx;
-    if (P >= np || Q >= np) return;
-    const float2 u = *reinterpret_cast<const float2 *>(A + (int64_t)(2 * P) * n + 2 * Q);
-    const float2 v = *reinterpret_cast<const float2 *>(A + (int64_t)(2 * P + 1) * n + 2 * Q);
-    float b00, b01, b10, b11;
-    if (P == Q) {
-      b00 = rd[ty][0];
-      b11 = rd[ty][1];
-      b01 = b10 = 0.0f;
+#pragma unroll
+      for (int l = 0; l < kJacLPT; ++l) {
+        const int L = L0 + 32 * l;
+        if (L >= np) continue;
+        const int pL = pl[l], qL = ql[l];
+        float b00, b01, b10, b11;
+        if (L == K) {
+          b00 = rk.z;
+          b11 = rk.w;
+          b01 = b10 = 0.0f;
+          if (m == 1) rot_next[0] = make_float4(0.0f, 0.0f, b00, b11);  // n = 2: the one pair stays diagonal
+        } else {
+          const float s1 = rk.x, t1 = rk.y, s2 = rl[l].x, t2 = rl[l].y;
+          const float a00 = a[l][0], a01 = a[l][1], a10 = a[l][2], a11 = a[l][3];
+          const float m00 = a00 - s1 * (a10 + t1 * a00), m10 = a10 + s1 * (a00 - t1 * a10);
+          const float m01 = a01 - s1 * (a11 + t1 * a01), m11 = a11 + s1 * (a01 - t1 * a11);
+          b00 = m00 - s2 * (m01 + t2 * m00);
+          b01 = m01 + s2 * (m00 - t2 * m01);
+          b10 = m10 - s2 * (m11 + t2 * m10);
+          b11 = m11 + s2 * (m10 - t2 * m11);
+          if (part0 == pL) rot_next[ka0] = jac_rot4(rk.z, rl[l].z, b00);
+          if (part0 == qL) rot_next[ka0] = jac_rot4(rk.z, rl[l].w, b01);
+          if (part1 == pL) rot_next[ka1] = jac_rot4(rk.w, rl[l].z, b10);
+          if (part1 == qL) rot_next[ka1] = jac_rot4(rk.w, rl[l].w, b11);
+        }
+        rp[pL] = b00;
+        rp[qL] = b01;
+        rq[pL] = b10;
+        rq[qL] = b11;
+      }
     } else {
-      const float s1 = rs[0][ty][0], t1 = rs[0][ty][1], s2 = rs[1][tx][0], t2 = rs[1][tx][1];
-      const float m00 = u.x - s1 * (v.x + t1 * u.x), m10 = v.x + s1 * (u.x - t1 * v.x);
-      const float m01 = u.y - s1 * (v.y + t1 * u.y), m11 = v.y + s1 * (u.y - t1 * v.y);
-      b00 = m00 - s2 * (m01 + t2 * m00);
-      b01 = m01 + s2 * (m00 - t2 * m01);
-      b10 = m10 - s2 * (m11 + t2 * m10);
-      b11 = m11 + s2 * (m10 - t2 * m11);
+      const int wv = w - warps_a;
+      const int k = wv / chunks;
+      const int L0 = (wv - k * chunks) * 32 * kJacLPT + lane;
+      float *vr = V + (int64_t)k * n;
+      float v[kJacLPT][2];
+      float2 rl[kJacLPT];
+      int pl[kJacLPT], ql[kJacLPT];
+#pragma unroll
+      for (int l = 0; l < kJacLPT; ++l) {
+        const int L = L0 + 32 * l;
+        pl[l] = jac_p(L, t, m);
+        ql[l] = jac_q(L, t, m);
+        if (L < np) {
+          const float4 r4 = __ldg(rot + L);
+          rl[l] = make_float2(r4.x, r4.y);
+          v[l][0] = vr[pl[l]];
+          v[l][1] = vr[ql[l]];
+        }
+      }
+#pragma unroll
+      for (int l = 0; l < kJacLPT; ++l) {
+        if (L0 + 32 * l >= np) continue;
+        const float v0 = v[l][0], v1 = v[l][1];
+        vr[pl[l]] = v0 - rl[l].x * (v1 + rl[l].y * v0);
+        vr[ql[l]] = v1 + rl[l].x * (v0 - rl[l].y * v1);
+      }
     }
-    const int64_t p0 = jac_next(2 * P, n), p1 = jac_next(2 * P + 1, n);
-    const int q0 = jac_next(2 * Q, n), q1 = jac_next(2 * Q + 1, n);
-    An[p0 * n + q0] = b00;
-    An[p0 * n + q1] = b01;
-    An[p1 * n + q0] = b10;
-    An[p1 * n + q1] = b11;
-  } else {
-    const int b = blockIdx.x - a_blocks;
-    const int k0 = (b / v_side) * 8, Q0 = (b % v_side) * 32;
-    if (threadIdx.x < 32 && Q0 + (int)threadIdx.x < np) {
-      const JacRot r = jac_pair(A, n, Q0 + threadIdx.x);
-      rs[1][threadIdx.x][0] = r.s;
-      rs[1][threadIdx.x][1] = r.tau;
-    }
-    __syncthreads();
-    const int64_t k = k0 + (threadIdx.x >> 5);
-    const int Q = Q0 + (threadIdx.x & 31);
-    if (k >= n || Q >= np) return;
-    const float s = rs[1][threadIdx.x & 31][0], tau = rs[1][threadIdx.x & 31][1];
-    const float2 w = *reinterpret_cast<const float2 *>(V + k * n + 2 * Q);
-    Vn[k * n + jac_next(2 * Q, n)] = w.x - s * (w.y + tau * w.x);
-    Vn[k * n + jac_next(2 * Q + 1, n)] = w.y + s * (w.x - tau * w.y);
   }
 }
 
@@ -686,23 +773,30 @@ int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *m
   return HME_OK;
 }
 
-int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1, double *acc, int32_t *order,
-                   float *W, float *variances, int *sweeps_out, cudaStream_t s) {
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, JacRotBuf rotbuf, double *acc, int32_t *order, float *W,
+                   float *variances, int *sweeps_out, cudaStream_t s) {
   const int n = g.n;
-  pca_identity_kernel<<<(unsigned)(((int64_t)n * n + 255) / 256), 256, 0, s>>>(V0, n);
-  count_launch();
   const int np = n / 2;
-  const int a_side = (np + kJacSide - 1) / kJacSide;
-  const int v_side = (np + 31) / 32;
-  const int blocks = a_side * a_side + v_side * ((n + 7) / 8);
-  float *A[2] = {A0, A1}, *V[2] = {V0, V1};
+  pca_identity_kernel<<<(unsigned)(((int64_t)n * n + 255) / 256), 256, 0, s>>>(V0, n);
+  float4 *rot[2] = {reinterpret_cast<float4 *>(rotbuf.r0), reinterpret_cast<float4 *>(rotbuf.r1)};
+  jacobi_rot_init_kernel<<<(np + 255) / 256, 256, 0, s>>>(A0, n, rot[0]);
+  count_launch(2);
+  int per_sm = 0;
+  cudaError_t ea = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, jacobi_round_kernel, kJacThreads, 0);
+  if (ea != cudaSuccess) return cuda_fail(ea, "pca: Jacobi occupancy");
+  if (per_sm < 1) per_sm = 1;
+  const int64_t chunks = (np + 32 * kJacLPT - 1) / (32 * kJacLPT);
+  const int64_t warps = ((int64_t)np + n) * chunks;
+  int64_t blocks = (int64_t)num_sms() * per_sm;  // one wave
+  const int64_t need = (warps * 32 + kJacThreads - 1) / kJacThreads;
+  if (blocks > need) blocks = need;
   int cur = 0, sweep = 0;
   bool converged = false;
   const double tol2 = 0x1p-44;  // (2^-22)^2
   double prev_off = -1.0;
   for (sweep = 1; sweep <= kJacobiMaxSweeps && !converged; ++sweep) {
     for (int t = 0; t < n - 1; ++t) {
-      jacobi_round_kernel<<<blocks, 256, 0, s>>>(A[cur], V[cur], A[cur ^ 1], V[cur ^ 1], n, a_side, v_side);
+      jacobi_round_kernel<<<(unsigned)blocks, kJacThreads, 0, s>>>(A0, V0, rot[cur], rot[cur ^ 1], n, t);
       cur ^= 1;
     }
     count_launch(n - 1);
@@ -710,7 +804,7 @@ int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1,
     if (e != cudaSuccess) return cuda_fail(e, "pca: clear norms");
     int nb = (int)(((int64_t)n * n + 255) / 256);
     if (nb > 4 * num_sms()) nb = 4 * num_sms();
-    jacobi_offnorm_kernel<<<nb, 256, 0, s>>>(A[cur], n, acc);
+    jacobi_offnorm_kernel<<<nb, 256, 0, s>>>(A0, n, acc);
     count_launch();
     double h[2];
     e = cudaMemcpyAsync(h, acc, sizeof(h), cudaMemcpyDeviceToHost, s);
@@ -724,14 +818,13 @@ int run_pca_jacobi(const PcaGeom &g, float *A0, float *A1, float *V0, float *V1,
   }
   if (sweeps_out) *sweeps_out = sweep - 1;
   if (!converged) return fail(HME_EINTERNAL, "pca: Jacobi did not converge in %d sweeps", kJacobiMaxSweeps);
-  // n - 1 rounds per sweep restore the slot order, so slot j holds index j
   const size_t rank_smem = (size_t)g.d * sizeof(float);
   if (rank_smem > 48 * 1024) {
     cudaError_t ea = cudaFuncSetAttribute(pca_rank_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rank_smem);
     if (ea != cudaSuccess) return cuda_fail(ea, "pca: rank smem");
   }
-  pca_rank_kernel<<<1, 1024, rank_smem, s>>>(A[cur], n, g.d, g.r, order, variances);
-  pca_components_kernel<<<g.r, 256, 0, s>>>(V[cur], n, g.d, order, W);
+  pca_rank_kernel<<<1, 1024, rank_smem, s>>>(A0, n, g.d, g.r, order, variances);
+  pca_components_kernel<<<g.r, 256, 0, s>>>(V0, n, g.d, order, W);
   count_launch(2);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pca: components");

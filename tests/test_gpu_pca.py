@@ -7,7 +7,8 @@ Tolerances, from the arithmetic (each stated where it is used):
               error give at most 3 * 2^-16 |y_a||y_b| per product; the tensor
               cores accumulate 512 rows at a time in fp32: 3 x 512/16 = 96
               steps of at most one ulp (2^-23, whatever the rounding), +2 for
-              the conversions; those sums are added in fp64.  So |dC_ab| <= TAU_C * B_ab with
+              the conversions; up to 16 such sums are added in fp32 registers
+              (round to nearest, 2^-24 each, +2), then in fp64.  So |dC_ab| <= TAU_C * B_ab with
               B = (1/N) sum_i (|y_ia| + |mu_a|)(|y_ib| + |mu_b|) (the |mu| terms
               cover the rounding of x - fp32(mu)).
   eigen       Weyl: |d lambda| <= ||dC||_2 <= ||TAU_C B||_F, plus the backward
@@ -29,7 +30,7 @@ pytestmark = pytest.mark.gpu
 
 hme = pytest.importorskip("paper_1704_06363_gb300.hme")
 
-TAU_C = 3 * 2.0 ** -16 + 98 * 2.0 ** -23
+TAU_C = 3 * 2.0 ** -16 + 98 * 2.0 ** -23 + 18 * 2.0 ** -24
 JACOBI = 2.0 ** -13
 
 
@@ -202,3 +203,57 @@ def test_fit_then_transform_then_assign(dev):
     assert np.allclose(np.diag(cz), lam, rtol=1e-3, atol=1e-4 * lam[0])
     off = cz - np.diag(np.diag(cz))
     assert np.max(np.abs(off)) <= 1e-3 * lam[0]
+
+
+def test_pca_benchmark_features_full_size(dev):
+    """The 1e6 x 2048 fp32 benchmark features at full size, r = 256, in the
+    launch configuration the benchmark times: covariance entries and means on
+    sampled index pairs against fp64 sums over the full columns; the fit's
+    components orthonormal with eigen-residuals within the bound against the
+    (sample-checked) covariance, variances against its fp64 eigenvalues;
+    projections of sampled rows against fp64 dot products."""
+    import hme_synth
+    w = hme_synth.WORKLOADS[2]
+    X, _ = hme_synth.make_features(w, device=dev)
+    N, d = X.shape
+    r = 256
+    ws = hme.workspace(hme.HME_OP_PCA, N, d, r, hme.HME_F32, device=dev)
+    mu64 = torch.empty(d, dtype=torch.float64, device=dev)
+    C = torch.empty(d, d, dtype=torch.float64, device=dev)
+    hme.hme_pca_covariance(X, mu64, C, ws)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    rng = np.random.default_rng(0)
+    cols = sorted(set([0, 1, 127, 128, 1000, 2047] + rng.integers(0, d, 10).tolist()))
+    colv = {j: X[:, j].double().cpu().numpy() for j in cols}
+    mu_ref = {j: colv[j].mean() for j in cols}
+    Cg, mug = C.cpu().numpy(), mu64.cpu().numpy()
+    for a in cols:
+        assert abs(mug[a] - mu_ref[a]) <= 2.0 ** -20 * (np.abs(colv[a]).mean() + 1e-30)
+        for b in cols:
+            ya, yb = colv[a] - mu_ref[a], colv[b] - mu_ref[b]
+            ref = np.mean(ya * yb)
+            bnd = np.mean((np.abs(ya) + abs(mu_ref[a])) * (np.abs(yb) + abs(mu_ref[b])))
+            assert abs(Cg[a, b] - ref) <= TAU_C * bnd, (a, b, Cg[a, b], ref)
+    mu = torch.empty(d, dtype=torch.float32, device=dev)
+    W = torch.empty(r, d, dtype=torch.float32, device=dev)
+    lam = torch.empty(r, dtype=torch.float32, device=dev)
+    sweeps = hme.hme_pca_fit(X, r, mu, W, ws, lam)
+    assert hme.hme_sync_status(ws) == hme.HME_OK and 1 <= sweeps <= 40
+    Wd, lamd = W.double(), lam.double()
+    normC = torch.linalg.norm(C).item()
+    tol = JACOBI * normC
+    assert (Wd @ Wd.T - torch.eye(r, dtype=torch.float64, device=dev)).abs().max().item() <= 2.0 ** -14
+    res = torch.linalg.norm(C @ Wd.T - Wd.T * lamd, dim=0).max().item()
+    assert res <= 2 * tol, res / normC
+    ev = np.sort(np.linalg.eigvalsh(Cg))[::-1][:r]
+    assert np.all(np.abs(lam.cpu().numpy() - ev) <= tol), np.max(np.abs(lam.cpu().numpy() - ev)) / normC
+    Z = torch.empty(N, r, dtype=torch.float32, device=dev)
+    wt = hme.workspace(hme.HME_OP_PCA, 0, d, r, hme.HME_F32, device=dev)
+    hme.hme_pca_transform(X, mu, W, Z, wt)
+    assert hme.hme_sync_status(wt) == hme.HME_OK
+    rows = torch.tensor(sorted(set([0, N - 1] + rng.integers(0, N, 62).tolist())), device=dev)
+    Xs = X[rows].double().cpu().numpy()
+    Wn, mun = W.double().cpu().numpy(), mu.double().cpu().numpy()
+    ref = (Xs - mun) @ Wn.T
+    bound = _tau_z(d) * (np.abs(Xs) @ np.abs(Wn).T) + 2.0 ** -22 * (np.abs(ref) + np.abs(mun @ Wn.T))
+    assert np.all(np.abs(Z[rows].double().cpu().numpy() - ref) <= bound)
