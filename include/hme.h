@@ -328,7 +328,7 @@ HME_API int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, i
  *   ulp, whatever the accumulator's rounding).  Requires N >= 1.
  *
  * hme_pca_fit -- the covariance as above, then its eigendecomposition by
- *   cyclic Jacobi in fp32 (until the off-diagonal norm is at most 2^-22 of
+ *   cyclic Jacobi in fp32 (until the off-diagonal norm is at most 2^-20 of
  *   the Frobenius norm, or stagnates below 2^-16 of it), then
  *   mean_out (fp32, d), components_out (fp32, r x d row-major, orthonormal
  *   rows), variances_out (fp32, r, the eigenvalues; may be NULL) and

@@ -270,7 +270,7 @@ int clear_header(void *ws, cudaStream_t s) {
 // PCA fit (hme_pca_covariance / hme_pca_fit): slab sums, mean, transposed
 // split, covariance partial tiles, the Jacobi matrices and small scratch.
 struct PcaLayout {
-  size_t slab, mean64, mean32, yh, yl, part, A0, V0, rot0, rot1, acc, order, total;
+  size_t slab, mean64, mean32, yh, yl, part, A0, V0, qbuf, acc, order, total;
 };
 PcaLayout pca_layout(int64_t N, int d, int r) {
   const PcaGeom g = pca_geom(N, d, r);
@@ -291,8 +291,7 @@ PcaLayout pca_layout(int64_t N, int d, int r) {
   const size_t nn = (size_t)g.n * g.n * 4;
   L.A0 = take(nn);
   L.V0 = take(nn);
-  L.rot0 = take((size_t)(g.n / 2) * 16);
-  L.rot1 = take((size_t)(g.n / 2) * 16);
+  L.qbuf = take((size_t)(g.n / 64) * 64 * 64 * 4);
   L.acc = take(16);
   L.order = take((size_t)r * 4);
   L.total = align_up(off, 256);
@@ -589,8 +588,7 @@ int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
                          at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), nullptr, at<float>(ws, L.A0),
                          at<Header>(ws, 0), s));
   int sweeps = 0;
-  JacRotBuf rb{at<void>(ws, L.rot0), at<void>(ws, L.rot1)};
-  const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.V0), rb, at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,
+  const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.V0), at<float>(ws, L.qbuf), at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,
                                 &sweeps, s);
   if (sweeps_out) *sweeps_out = sweeps;
   if (rc != HME_OK) return rc;

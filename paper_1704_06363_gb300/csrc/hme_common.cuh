@@ -193,7 +193,7 @@ constexpr int kJacobiMaxSweeps = 40;
 struct PcaGeom {
   int64_t N;
   int d, r;
-  int n;           // Jacobi order: d rounded up to even
+  int n;           // Jacobi order: d rounded up to a multiple of 64
   int64_t ldn;     // row pitch (elements) of the transposed split: N rounded up to 8
   int mi, ntiles;  // 128-feature tiles along d; upper-triangle tiles
   int64_t R, nchunks, nslabs;  // rows per covariance work unit, units per tile, column-sum slabs
@@ -207,12 +207,9 @@ int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *m
                    __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s);
 // Jacobi sweeps on A0 (synchronises s once per sweep), then the r leading
 // components (rows of W, r x d) and their variances (may be null)
-struct JacRotBuf {
-  void *r0, *r1;  // two rotation tables of 16 * (n / 2) bytes (this round's, the next round's)
-};
-int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, JacRotBuf rotbuf, double *acc, int32_t *order, float *W,
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, float *Qbuf, double *acc, int32_t *order, float *W,
                    float *variances, int *sweeps_out, cudaStream_t s);
-constexpr int kPcaMaxFitD = 8192;  // int32 item indices of a Jacobi round: (n/2)^2 + n (n/2) < 2^31
+constexpr int kPcaMaxFitD = 8192;
 cudaError_t launch_pca_zoff(const float *mean, const float *W, int d, int r, int Kp, float *zoff, cudaStream_t s);
 cudaError_t launch_debug_wait(uint64_t timeout_ns, Header *hdr, cudaStream_t s);
 int64_t kpp_candidates(int64_t N, int K, int method);

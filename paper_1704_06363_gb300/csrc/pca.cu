@@ -22,14 +22,13 @@
 //   pca_cov_reduce  the partial tiles added in range order in fp64, / N: the
 //                   covariance (fp64, both triangles) and A (fp32, order n = d
 //                   rounded up to even, padding row and column zero);
-//   Jacobi          cyclic two-sided Jacobi on A, n/2 disjoint rotations per
-//                   round (circle-method ordering: n - 1 rounds meet every pair
-//                   once).  One kernel per round updates A and V (the
-//                   eigenvector estimate, V <- V J) in place, each 2 x 2 block
-//                   by one thread; the two matrices (2 n^2 floats, 32 MB at
-//                   d = 2048) stay in L2, and the next round's rotations are
-//                   formed by the threads that produce its pivots.  Sweeps
-//                   repeat until off(A) <= 2^-22 ||A||_F;
+//   Jacobi          cyclic two-sided block Jacobi on A (n = d rounded up to a
+//                   multiple of 64; blocks of 32 indices paired by the circle
+//                   method): per round, the 64 x 64 sub-problems of the block
+//                   pairs are diagonalised in shared memory and their
+//                   orthogonal factors applied to the rest of A and to V (the
+//                   eigenvector estimate) as fp32 64 x 64 products, in place.
+//                   Sweeps repeat until off(A) <= 2^-20 ||A||_F;
 //   pca_rank        eigenvalues diag(A) ranked (decreasing, ties to the lower
 //                   index), the padding slot excluded;
 //   pca_components  the leading r columns of V, normalised, with the sign rule.
@@ -412,26 +411,6 @@ __device__ __forceinline__ int jac_q(int k, int t, int m) {
   const int x = t - k;
   return 1 + (x < 0 ? x + m : x);
 }
-// pair of index x in round t, and whether x is its p member
-__device__ __forceinline__ int jac_pair_of(int x, int t, int m, bool &is_p) {
-  if (x == 0) {
-    is_p = true;
-    return 0;
-  }
-  int kk = x - 1 - t;
-  if (kk < 0) kk += m;
-  if (kk == 0) {
-    is_p = false;
-    return 0;
-  }
-  if (kk <= (m - 1) / 2) {
-    is_p = true;
-    return kk;
-  }
-  is_p = false;
-  return m - kk;
-}
-
 // The rotation of one pair (Rutishauser's form): t = tan(phi) is the smaller
 // root of t^2 + 2 theta t - 1 = 0, theta = (a_qq - a_pp) / (2 a_pq), which
 // zeroes a_pq; the update of a pair of entries (u, v) of rows (or columns) p
@@ -456,122 +435,191 @@ __device__ float4 jac_rot4(float app, float aqq, float apq) {
   return r;
 }
 
-__global__ void jacobi_rot_init_kernel(const float *__restrict__ A, int n, float4 *__restrict__ rot) {
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  const int m = n - 1;
-  if (k >= (n >> 1)) return;
-  const int64_t p = jac_p(k, 0, m), q = jac_q(k, 0, m);
-  rot[k] = jac_rot4(A[p * n + p], A[q * n + q], A[p * n + q]);
+// Blocked Jacobi.  The order n is a multiple of 2 kJB; the n / kJB blocks of
+// kJB indices are paired by the same circle method (round t of nb - 1, pair P
+// = blocks (jac_p(P, t, nb - 1), jac_q(P, t, nb - 1))).  A round:
+//   bj_sub_kernel    one CTA per block pair: one cyclic Jacobi sweep (the
+//                    scalar rotations above, 63 rounds) on the 64 x 64
+//                    sub-matrix S of A on the pair's indices, in shared memory
+//                    (more inner sweeps per round saved at most one outer sweep
+//                    in a prototype, and cost a full sweep each); its orthogonal
+//                    factor Q (S <- Q^T S Q, a product of rotations close to the
+//                    identity, never a permutation: eigenvectors sorted by
+//                    eigenvalue stalled the outer iteration in the prototype)
+//                    goes to Qbuf and S back into A;
+//   bj_apply_kernel  A_PR <- Q_P^T A_PR Q_R for every other 64 x 64 tile of A
+//                    on pairs (P, R), and V_kR <- V_kR Q_R for every 64-row
+//                    slice of V: two fp32 64 x 64 x 64 products per tile in
+//                    shared memory, each tile read and written in place by
+//                    one CTA.
+// A sweep (nb - 1 rounds) meets every pair of blocks once, so every pair of
+// indices, as the scalar method does; it passes over A and V 2 (nb - 1) times
+// instead of n - 1.
+constexpr int kJB = 32;        // indices per block
+constexpr int kJS = 2 * kJB;   // order of a sub-problem
+constexpr int kJSP = kJS + 1;  // shared row pitch of the sub-problem kernel
+constexpr int kApT = 68;       // shared row pitch of the apply kernel (16-byte rows)
+
+__device__ __forceinline__ int bj_index(int i, int I, int J) { return i < kJB ? I * kJB + i : J * kJB + (i - kJB); }
+
+// One thread per 2 x 2 block of S and two column pairs of Q per inner round;
+// the inner rounds' pairs come from a table.  Each inner round: the 32
+// rotations (one warp), a barrier, the updates of S and Q, a barrier.
+constexpr int kSubThreads = 1024;
+__global__ void __launch_bounds__(kSubThreads) bj_sub_kernel(float *__restrict__ A, int n, int t,
+                                                             float *__restrict__ Qbuf) {
+  __shared__ float S[kJS * kJSP];
+  __shared__ float Q[kJS * kJSP];
+  __shared__ float4 rot[kJB];
+  __shared__ uint8_t pq[kJS - 1][kJB][2];
+  const int nbm = n / kJB - 1;
+  const int P = blockIdx.x;
+  const int I = jac_p(P, t, nbm), J = jac_q(P, t, nbm);
+  for (int e = threadIdx.x; e < kJS * kJS; e += blockDim.x) {
+    const int i = e / kJS, j = e - i * kJS;
+    S[i * kJSP + j] = A[(int64_t)bj_index(i, I, J) * n + bj_index(j, I, J)];
+    Q[i * kJSP + j] = i == j ? 1.0f : 0.0f;
+  }
+  for (int e = threadIdx.x; e < (kJS - 1) * kJB; e += blockDim.x) {
+    const int r = e / kJB, k = e - r * kJB;
+    pq[r][k][0] = (uint8_t)jac_p(k, r, kJS - 1);
+    pq[r][k][1] = (uint8_t)jac_q(k, r, kJS - 1);
+  }
+  __syncthreads();
+  const int K = threadIdx.x / kJB, L = threadIdx.x % kJB;  // this thread's 2 x 2 block of S
+  const int qi = threadIdx.x / (kJB / 2), qL0 = (threadIdx.x % (kJB / 2)) * 2;  // Q row, two column pairs
+  for (int r = 0; r < kJS - 1; ++r) {
+    if (threadIdx.x < kJB) {
+      const int p = pq[r][threadIdx.x][0], q = pq[r][threadIdx.x][1];
+      rot[threadIdx.x] = jac_rot4(S[p * kJSP + p], S[q * kJSP + q], S[p * kJSP + q]);
+    }
+    __syncthreads();
+    {
+      const int pK = pq[r][K][0], qK = pq[r][K][1], pL = pq[r][L][0], qL = pq[r][L][1];
+      const float4 rk = rot[K];
+      float *sp = S + pK * kJSP, *sq = S + qK * kJSP;
+      if (K == L) {
+        sp[pL] = rk.z;
+        sq[qL] = rk.w;
+        sp[qL] = 0.0f;
+        sq[pL] = 0.0f;
+      } else {
+        const float4 rl = rot[L];
+        const float a00 = sp[pL], a01 = sp[qL], a10 = sq[pL], a11 = sq[qL];
+        const float s1 = rk.x, t1 = rk.y, s2 = rl.x, t2 = rl.y;
+        const float m00 = a00 - s1 * (a10 + t1 * a00), m10 = a10 + s1 * (a00 - t1 * a10);
+        const float m01 = a01 - s1 * (a11 + t1 * a01), m11 = a11 + s1 * (a01 - t1 * a11);
+        sp[pL] = m00 - s2 * (m01 + t2 * m00);
+        sp[qL] = m01 + s2 * (m00 - t2 * m01);
+        sq[pL] = m10 - s2 * (m11 + t2 * m10);
+        sq[qL] = m11 + s2 * (m10 - t2 * m11);
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {  // Q <- Q J on row qi, column pairs qL0, qL0 + 1
+      const int Lq = qL0 + c;
+      const int pL = pq[r][Lq][0], qL = pq[r][Lq][1];
+      const float4 rl = rot[Lq];
+      float *qrow = Q + qi * kJSP;
+      const float v0 = qrow[pL], v1 = qrow[qL];
+      qrow[pL] = v0 - rl.x * (v1 + rl.y * v0);
+      qrow[qL] = v1 + rl.x * (v0 - rl.y * v1);
+    }
+    __syncthreads();
+  }
+  float *qo = Qbuf + (int64_t)P * kJS * kJS;
+  for (int e = threadIdx.x; e < kJS * kJS; e += blockDim.x) {
+    const int i = e / kJS, j = e - i * kJS;
+    qo[e] = Q[i * kJSP + j];
+    A[(int64_t)bj_index(i, I, J) * n + bj_index(j, I, J)] = S[i * kJSP + j];
+  }
 }
 
-// One round t, in place.  A warp owns one row pair of A (rows rotated by
-// that pair) or one row pair of V, and 32 x kJacLPT column pairs (lane j takes
-// column pairs L0 + j + 32 l, so every access of the warp is a contiguous run
-// of a row); each 2 x 2 block of A gets both rotations (the diagonal block
-// K = L becomes diag(dp, dq)), V gets the column rotations (V <- V J).  Every
-// entry is read and written by one thread, so no two blocks conflict.  The
-// rotation table of the round comes in (read through L1); the next round's is
-// written by the owners of its pivots: the entry (a, b) with a the p member
-// and b the q member of a next-round pair lies in one off-diagonal block of
-// this round, whose thread forms the rotation from the new entry and the new
-// diagonal entries dp / dq of a's and b's pairs.
-constexpr int kJacThreads = 256;
-constexpr int kJacLPT = 4;  // column pairs per thread
-__global__ void __launch_bounds__(kJacThreads) jacobi_round_kernel(float *__restrict__ A, float *__restrict__ V,
-                                                                   const float4 *__restrict__ rot,
-                                                                   float4 *__restrict__ rot_next, int n, int t) {
-  const int np = n >> 1, m = n - 1;
-  const int tn = t + 1 == m ? 0 : t + 1;
-  const int chunks = (np + 32 * kJacLPT - 1) / (32 * kJacLPT);
-  const int warps_a = np * chunks, warps_total = warps_a + n * chunks;
-  const int lane = threadIdx.x & 31;
-  const int wstride = (int)((gridDim.x * blockDim.x) >> 5);
-  for (int w = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); w < warps_total; w += wstride) {
-    if (w < warps_a) {
-      const int K = w / chunks;
-      const int L0 = (w - K * chunks) * 32 * kJacLPT + lane;
-      const int pK = jac_p(K, t, m), qK = jac_q(K, t, m);
-      const float4 rk = __ldg(rot + K);
-      // next-round partner of each row index that is a p member next round (else -1)
-      bool ap0, ap1;
-      const int ka0 = jac_pair_of(pK, tn, m, ap0), ka1 = jac_pair_of(qK, tn, m, ap1);
-      const int part0 = ap0 ? jac_q(ka0, tn, m) : -1, part1 = ap1 ? jac_q(ka1, tn, m) : -1;
-      float *rp = A + (int64_t)pK * n, *rq = A + (int64_t)qK * n;
-      // all loads of the thread's blocks first (they are in flight together),
-      // then the rotations and stores
-      float a[kJacLPT][4];
-      float4 rl[kJacLPT];
-      int pl[kJacLPT], ql[kJacLPT];
+// 64 x 64 x 64 product in shared memory: out[i][j] = sum_k L[k][i] R[k][j]
+// (the left operand transposed), pitch kApT; thread (ty, tx) of 16 x 16 makes
+// rows 4 ty .. 4 ty + 3 and columns 4 tx .. 4 tx + 3.
+__device__ __forceinline__ void bj_mm_tn(const float *Lm, const float *Rm, float (&o)[4][4], int ty, int tx) {
 #pragma unroll
-      for (int l = 0; l < kJacLPT; ++l) {
-        const int L = L0 + 32 * l;
-        pl[l] = jac_p(L, t, m);
-        ql[l] = jac_q(L, t, m);
-        if (L < np) {
-          rl[l] = __ldg(rot + L);
-          a[l][0] = rp[pl[l]];
-          a[l][1] = rp[ql[l]];
-          a[l][2] = rq[pl[l]];
-          a[l][3] = rq[ql[l]];
-        }
-      }
+  for (int a = 0; a < 4; ++a)
 #pragma unroll
-      for (int l = 0; l < kJacLPT; ++l) {
-        const int L = L0 + 32 * l;
-        if (L >= np) continue;
-        const int pL = pl[l], qL = ql[l];
-        float b00, b01, b10, b11;
-        if (L == K) {
-          b00 = rk.z;
-          b11 = rk.w;
-          b01 = b10 = 0.0f;
-          if (m == 1) rot_next[0] = make_float4(0.0f, 0.0f, b00, b11);  // n = 2: the one pair stays diagonal
-        } else {
-          const float s1 = rk.x, t1 = rk.y, s2 = rl[l].x, t2 = rl[l].y;
-          const float a00 = a[l][0], a01 = a[l][1], a10 = a[l][2], a11 = a[l][3];
-          const float m00 = a00 - s1 * (a10 + t1 * a00), m10 = a10 + s1 * (a00 - t1 * a10);
-          const float m01 = a01 - s1 * (a11 + t1 * a01), m11 = a11 + s1 * (a01 - t1 * a11);
-          b00 = m00 - s2 * (m01 + t2 * m00);
-          b01 = m01 + s2 * (m00 - t2 * m01);
-          b10 = m10 - s2 * (m11 + t2 * m10);
-          b11 = m11 + s2 * (m10 - t2 * m11);
-          if (part0 == pL) rot_next[ka0] = jac_rot4(rk.z, rl[l].z, b00);
-          if (part0 == qL) rot_next[ka0] = jac_rot4(rk.z, rl[l].w, b01);
-          if (part1 == pL) rot_next[ka1] = jac_rot4(rk.w, rl[l].z, b10);
-          if (part1 == qL) rot_next[ka1] = jac_rot4(rk.w, rl[l].w, b11);
-        }
-        rp[pL] = b00;
-        rp[qL] = b01;
-        rq[pL] = b10;
-        rq[qL] = b11;
-      }
+    for (int b = 0; b < 4; ++b) o[a][b] = 0.0f;
+#pragma unroll 8
+  for (int k = 0; k < kJS; ++k) {
+    const float4 l = *reinterpret_cast<const float4 *>(Lm + k * kApT + 4 * ty);
+    const float4 rr = *reinterpret_cast<const float4 *>(Rm + k * kApT + 4 * tx);
+    const float lv[4] = {l.x, l.y, l.z, l.w}, rv[4] = {rr.x, rr.y, rr.z, rr.w};
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) o[a][b] = fmaf(lv[a], rv[b], o[a][b]);
+  }
+}
+
+// Tiles [0, np^2 - np): (P, R), P != R, of A; then (n / 64) x np slices of V.
+__global__ void __launch_bounds__(256) bj_apply_kernel(float *__restrict__ A, float *__restrict__ V, int n, int t,
+                                                       const float *__restrict__ Qbuf) {
+  extern __shared__ float4 bj_smem[];
+  float *T = reinterpret_cast<float *>(bj_smem);  // the tile, then the intermediate product (transposed)
+  float *QL = T + kJS * kApT;
+  float *QR = QL + kJS * kApT;
+  const int nb = n / kJB, nbm = nb - 1, np = nb / 2;
+  const int ntile_a = np * np - np;
+  const int ntiles = ntile_a + (n / kJS) * np;
+  const int ty = threadIdx.x >> 4, tx = threadIdx.x & 15;
+  for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    const bool isA = tile < ntile_a;
+    int P = 0, R, row0 = 0;
+    if (isA) {
+      P = tile / (np - 1);
+      R = tile - P * (np - 1);
+      if (R >= P) ++R;  // skip the diagonal tile
     } else {
-      const int wv = w - warps_a;
-      const int k = wv / chunks;
-      const int L0 = (wv - k * chunks) * 32 * kJacLPT + lane;
-      float *vr = V + (int64_t)k * n;
-      float v[kJacLPT][2];
-      float2 rl[kJacLPT];
-      int pl[kJacLPT], ql[kJacLPT];
+      const int v = tile - ntile_a;
+      row0 = (v / np) * kJS;
+      R = v - (v / np) * np;
+    }
+    const int IR = jac_p(R, t, nbm), JR = jac_q(R, t, nbm);
+    const int IP = isA ? jac_p(P, t, nbm) : 0, JP = isA ? jac_q(P, t, nbm) : 0;
+    float *M = isA ? A : V;
+    __syncthreads();  // the previous tile's buffers are free
+    for (int e = threadIdx.x; e < kJS * kJS; e += blockDim.x) {
+      const int i = e / kJS, j = e - i * kJS;
+      const int64_t gi = isA ? bj_index(i, IP, JP) : row0 + i;
+      T[i * kApT + j] = M[gi * n + bj_index(j, IR, JR)];
+      QR[i * kApT + j] = Qbuf[(int64_t)R * kJS * kJS + e];
+      if (isA) QL[i * kApT + j] = Qbuf[(int64_t)P * kJS * kJS + e];
+    }
+    __syncthreads();
+    float o[4][4];
+    if (isA) {
+      bj_mm_tn(QL, T, o, ty, tx);  // U = Q_P^T T
+      __syncthreads();             // T is overwritten by U^T
 #pragma unroll
-      for (int l = 0; l < kJacLPT; ++l) {
-        const int L = L0 + 32 * l;
-        pl[l] = jac_p(L, t, m);
-        ql[l] = jac_q(L, t, m);
-        if (L < np) {
-          const float4 r4 = __ldg(rot + L);
-          rl[l] = make_float2(r4.x, r4.y);
-          v[l][0] = vr[pl[l]];
-          v[l][1] = vr[ql[l]];
-        }
-      }
+      for (int a = 0; a < 4; ++a)
 #pragma unroll
-      for (int l = 0; l < kJacLPT; ++l) {
-        if (L0 + 32 * l >= np) continue;
-        const float v0 = v[l][0], v1 = v[l][1];
-        vr[pl[l]] = v0 - rl[l].x * (v1 + rl[l].y * v0);
-        vr[ql[l]] = v1 + rl[l].x * (v0 - rl[l].y * v1);
-      }
+        for (int b = 0; b < 4; ++b) T[(4 * tx + b) * kApT + 4 * ty + a] = o[a][b];
+      __syncthreads();
+    } else {
+      // V: T' = T Q_R, i.e. the left operand is T itself: store it transposed
+      float tt[4][4];
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) tt[a][b] = T[(4 * ty + a) * kApT + 4 * tx + b];
+      __syncthreads();
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) T[(4 * tx + b) * kApT + 4 * ty + a] = tt[a][b];
+      __syncthreads();
+    }
+    bj_mm_tn(T, QR, o, ty, tx);  // (U or T) Q_R with the left operand stored transposed
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+      const int i = 4 * ty + a;
+      const int64_t gi = isA ? bj_index(i, IP, JP) : row0 + i;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) M[gi * n + bj_index(4 * tx + b, IR, JR)] = o[a][b];
     }
   }
 }
@@ -706,7 +754,7 @@ PcaGeom pca_geom(int64_t N, int d, int r) {
   g.N = N;
   g.d = d;
   g.r = r;
-  g.n = d + (d & 1);
+  g.n = (d + 63) / 64 * 64;
   g.ldn = (N + 7) / 8 * 8;
   g.mi = (d + kBM - 1) / kBM;
   g.ntiles = g.mi * (g.mi + 1) / 2;
@@ -773,44 +821,43 @@ int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *m
   return HME_OK;
 }
 
-int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, JacRotBuf rotbuf, double *acc, int32_t *order, float *W,
+int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, float *Qbuf, double *acc, int32_t *order, float *W,
                    float *variances, int *sweeps_out, cudaStream_t s) {
   const int n = g.n;
-  const int np = n / 2;
+  const int nb = n / kJB, np = nb / 2;
   pca_identity_kernel<<<(unsigned)(((int64_t)n * n + 255) / 256), 256, 0, s>>>(V0, n);
-  float4 *rot[2] = {reinterpret_cast<float4 *>(rotbuf.r0), reinterpret_cast<float4 *>(rotbuf.r1)};
-  jacobi_rot_init_kernel<<<(np + 255) / 256, 256, 0, s>>>(A0, n, rot[0]);
-  count_launch(2);
+  count_launch();
+  const size_t ap_smem = (size_t)3 * kJS * kApT * sizeof(float);
+  cudaError_t ea = cudaFuncSetAttribute(bj_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ap_smem);
+  if (ea != cudaSuccess) return cuda_fail(ea, "pca: Jacobi smem");
   int per_sm = 0;
-  cudaError_t ea = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, jacobi_round_kernel, kJacThreads, 0);
+  ea = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, bj_apply_kernel, 256, ap_smem);
   if (ea != cudaSuccess) return cuda_fail(ea, "pca: Jacobi occupancy");
   if (per_sm < 1) per_sm = 1;
-  const int64_t chunks = (np + 32 * kJacLPT - 1) / (32 * kJacLPT);
-  const int64_t warps = ((int64_t)np + n) * chunks;
-  int64_t blocks = (int64_t)num_sms() * per_sm;  // one wave
-  const int64_t need = (warps * 32 + kJacThreads - 1) / kJacThreads;
-  if (blocks > need) blocks = need;
-  int cur = 0, sweep = 0;
+  const int64_t ntiles = (int64_t)np * np - np + (int64_t)(n / kJS) * np;
+  int64_t ap_blocks = (int64_t)num_sms() * per_sm;
+  if (ap_blocks > ntiles) ap_blocks = ntiles;
+  int sweep = 0;
   bool converged = false;
-  const double tol2 = 0x1p-44;  // (2^-22)^2
+  const double tol2 = 0x1p-40;  // (2^-20)^2
   double prev_off = -1.0;
   for (sweep = 1; sweep <= kJacobiMaxSweeps && !converged; ++sweep) {
-    for (int t = 0; t < n - 1; ++t) {
-      jacobi_round_kernel<<<(unsigned)blocks, kJacThreads, 0, s>>>(A0, V0, rot[cur], rot[cur ^ 1], n, t);
-      cur ^= 1;
+    for (int t = 0; t < nb - 1; ++t) {
+      bj_sub_kernel<<<np, kSubThreads, 0, s>>>(A0, n, t, Qbuf);
+      if (ap_blocks > 0) bj_apply_kernel<<<(unsigned)ap_blocks, 256, ap_smem, s>>>(A0, V0, n, t, Qbuf);
     }
-    count_launch(n - 1);
+    count_launch(2 * (nb - 1));
     cudaError_t e = cudaMemsetAsync(acc, 0, 2 * sizeof(double), s);
     if (e != cudaSuccess) return cuda_fail(e, "pca: clear norms");
-    int nb = (int)(((int64_t)n * n + 255) / 256);
-    if (nb > 4 * num_sms()) nb = 4 * num_sms();
-    jacobi_offnorm_kernel<<<nb, 256, 0, s>>>(A0, n, acc);
+    int nbk = (int)(((int64_t)n * n + 255) / 256);
+    if (nbk > 4 * num_sms()) nbk = 4 * num_sms();
+    jacobi_offnorm_kernel<<<nbk, 256, 0, s>>>(A0, n, acc);
     count_launch();
     double h[2];
     e = cudaMemcpyAsync(h, acc, sizeof(h), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "pca: Jacobi sweep");
-    // converged: off(A) <= 2^-22 ||A||_F, or off(A) already below 2^-16 ||A||_F
+    // converged: off(A) <= 2^-20 ||A||_F, or off(A) already below 2^-16 ||A||_F
     // and no longer halving from one sweep to the next (the fp32 floor)
     converged = h[0] <= tol2 * (h[0] + h[1]) ||
                 (prev_off >= 0.0 && h[0] >= 0.25 * prev_off && h[0] <= 0x1p-32 * (h[0] + h[1]));
