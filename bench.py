@@ -46,6 +46,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-stream", action="store_true", help="skip the streamed-from-host diagnostic")
     ap.add_argument("--no-pca", action="store_true", help="skip the PCA diagnostic")
+    ap.add_argument("--no-graph", action="store_true", help="time eager steps instead of CUDA-graph replays")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU work of the oracle sample")
     return ap.parse_args()
 
@@ -261,7 +262,7 @@ def run_ours(args, w):
     ev_assign, ev_update = [], []
     moved_dev = torch.zeros(1, dtype=torch.int32, device=dev)
 
-    def step(Xs, record=False):
+    def step(Xs, record=False, diag=False):
         C.copy_(C0)
         for t in range(T):
             labels, prev = labels_buf[t % 2], (labels_buf[(t - 1) % 2] if t > 0 else None)
@@ -277,7 +278,7 @@ def run_ours(args, w):
                 u1 = torch.cuda.Event(enable_timing=True)
             # first iteration: full pass; then only the rows whose label changed
             hme.hme_update_centroids(Xs, labels, mind, C, ws, counts, nres[t:t + 1], jex[t:t + 1], prev_labels=prev)
-            if not record and t == T - 1:  # diagnostic, outside the timed steps
+            if diag and t == T - 1:  # diagnostic, outside the timed steps
                 moved_dev.copy_(ws[32:36].view(torch.int32))
             if record:
                 u1.record(stream)
@@ -296,6 +297,23 @@ def run_ours(args, w):
     if status != hme.HME_OK:
         raise RuntimeError(f"device status {status} after warm-up: {hme.hme_last_error()}")
 
+    # The step is some 250 small launches (assign, rescore, incremental update
+    # kernels per iteration); it is captured once as a CUDA graph and the
+    # timed steps replay it.  The library makes no host synchronisation on
+    # this path, so the capture holds the whole step.
+    graph, launches_per_step = None, None
+    if not args.no_graph:
+        torch.cuda.synchronize(dev)
+        graph = torch.cuda.CUDAGraph()
+        l0 = hme.hme_launch_count()
+        with torch.cuda.graph(graph, capture_error_mode="relaxed"):
+            step(X)
+        launches_per_step = hme.hme_launch_count() - l0
+        graph.replay()  # one more warm-up step, as a replay
+        status = hme.hme_sync_status(ws)
+        if status != hme.HME_OK:
+            raise RuntimeError(f"device status {status} after the graph warm-up: {hme.hme_last_error()}")
+
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
@@ -305,19 +323,32 @@ def run_ours(args, w):
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        step(X, record=True)
+        if graph is not None:
+            graph.replay()
+        else:
+            step(X, record=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     clocks.end()
-    launches = hme.hme_launch_count() - launches0
+    # kernels launched in the timed region: the graph's kernels per replay, or
+    # the eager launches counted by the library
+    launches = launches_per_step * args.steps if graph is not None else hme.hme_launch_count() - launches0
     ck = clocks.stop()
-    hdr = ws[:16].view(torch.int32).cpu()  # queues of the last assign (the route's): pairs, all-K
-    rescored = {"pair": int(hdr[1]), "all_k": int(hdr[3])}
-    moved = int(moved_dev.item())  # rows that changed label in the last update of a warm-up step
     ms = max_over_ranks(e0.elapsed_time(e1), dev)
     status = hme.hme_sync_status(ws)
     if status != hme.HME_OK:
         raise RuntimeError(f"device status {status} after the timed steps: {hme.hme_last_error()}")
+    # per-call timings and diagnostics: one eager step after the timed region
+    # (with graph replays) or the timed eager steps themselves
+    if graph is not None:
+        step(X, record=True, diag=True)
+        torch.cuda.synchronize(dev)
+    else:
+        step(X, diag=True)
+        torch.cuda.synchronize(dev)
+    hdr = ws[:16].view(torch.int32).cpu()  # queues of the last assign (the route's): pairs, all-K
+    rescored = {"pair": int(hdr[1]), "all_k": int(hdr[3])}
+    moved = int(moved_dev.item())  # rows that changed label in the last update of the step
 
     # outside the timed steps: routing the same rows as a one-off call (no
     # preparation; fp32 rows with K <= 256 are split inside the kernel) against
@@ -475,9 +506,20 @@ def run_ours(args, w):
         out_offsets = torch.empty(K + 1, dtype=torch.int64, pin_memory=True)
         out_C = torch.empty(K, d, dtype=torch.float32, pin_memory=True)
 
+        graph_e2e = None
+        if graph is not None:  # the same step on the copied-in buffer, as a graph
+            torch.cuda.synchronize(dev)
+            Xd.copy_(X)
+            graph_e2e = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph_e2e, capture_error_mode="relaxed"):
+                step(Xd)
+
         def e2e_step():
             Xd.copy_(Xh, non_blocking=True)
-            step(Xd)
+            if graph_e2e is not None:
+                graph_e2e.replay()
+            else:
+                step(Xd)
             out_labels.copy_(expert, non_blocking=True)
             out_order.copy_(order, non_blocking=True)
             out_offsets.copy_(offsets, non_blocking=True)
@@ -516,7 +558,8 @@ def run_ours(args, w):
                     " + route of all N rows" % T + (" + partition of the routed rows with their tag lists"
                                                       if w.tags else ""),
                        "l2": "inputs larger than L2 (%.1f GB of features)" % (X.numel() * e / 1e9),
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "launch": "CUDA graph replay of the captured step" if graph is not None else "eager launches"},
             "vectors_per_s": N * iters_total / (ms / 1000.0),
             "assign_gflops": flops_assign / (t_assign / 1000.0) / 1e9,
             "kernels_ms": {"assign_call": t_assign, "assign_call_prepare_out": t_assign_first, "update_call_full": t_update, "update_call_incremental": t_incr,
