@@ -131,6 +131,9 @@ def test_pca_host_validation(lib):
     args = list(ok)
     args[11] = 64
     assert g(*args) == 2  # workspace too small
+    args = list(ok)
+    args[2], args[3], args[5] = 8193, 8193, 4
+    assert g(*args) == 1 and b"8192" in lib.hme_last_error()  # the Jacobi takes d <= 8192
     t = lib.hme_pca_transform
     t.restype = ctypes.c_int
     t.argtypes = [p, i64, i32, i64, i32, p, p, i32, p, i64, p, ctypes.c_size_t, p]

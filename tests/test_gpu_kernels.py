@@ -82,6 +82,11 @@ ASSIGN_CASES = [
     (4100, 2048, 64, "f32", None),
     (4100, 2048, 256, "bf16", None),
     (50, 96, 200, "f32", None),
+    # the largest K and d the library takes: 64 (fp32) / 128 (bf16, resident rows) N-chunks; 256 k-blocks
+    (1500, 64, 16384, "bf16", None),
+    (700, 48, 16384, "f32", None),
+    (300, 16384, 8, "f32", None),
+    (300, 16384, 40, "bf16", 16392),
 ]
 
 
