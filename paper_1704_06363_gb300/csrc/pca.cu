@@ -582,12 +582,17 @@ __global__ void __launch_bounds__(256) bj_apply_kernel(float *__restrict__ A, fl
     const int IP = isA ? jac_p(P, t, nbm) : 0, JP = isA ? jac_q(P, t, nbm) : 0;
     float *M = isA ? A : V;
     __syncthreads();  // the previous tile's buffers are free
-    for (int e = threadIdx.x; e < kJS * kJS; e += blockDim.x) {
-      const int i = e / kJS, j = e - i * kJS;
+    // 16-byte loads: a tile row is two runs of 32 floats (blocks IR and JR)
+    for (int e = threadIdx.x; e < kJS * kJS / 4; e += blockDim.x) {
+      const int i = e / (kJS / 4), j = (e - i * (kJS / 4)) * 4;
       const int64_t gi = isA ? bj_index(i, IP, JP) : row0 + i;
-      T[i * kApT + j] = M[gi * n + bj_index(j, IR, JR)];
-      QR[i * kApT + j] = Qbuf[(int64_t)R * kJS * kJS + e];
-      if (isA) QL[i * kApT + j] = Qbuf[(int64_t)P * kJS * kJS + e];
+      *reinterpret_cast<float4 *>(T + i * kApT + j) =
+          __ldg(reinterpret_cast<const float4 *>(M + gi * n + bj_index(j, IR, JR)));
+      *reinterpret_cast<float4 *>(QR + i * kApT + j) =
+          __ldg(reinterpret_cast<const float4 *>(Qbuf + (int64_t)R * kJS * kJS + i * kJS + j));
+      if (isA)
+        *reinterpret_cast<float4 *>(QL + i * kApT + j) =
+            __ldg(reinterpret_cast<const float4 *>(Qbuf + (int64_t)P * kJS * kJS + i * kJS + j));
     }
     __syncthreads();
     float o[4][4];
@@ -595,31 +600,30 @@ __global__ void __launch_bounds__(256) bj_apply_kernel(float *__restrict__ A, fl
       bj_mm_tn(QL, T, o, ty, tx);  // U = Q_P^T T
       __syncthreads();             // T is overwritten by U^T
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) T[(4 * tx + b) * kApT + 4 * ty + a] = o[a][b];
+      for (int b = 0; b < 4; ++b)
+        *reinterpret_cast<float4 *>(T + (4 * tx + b) * kApT + 4 * ty) = make_float4(o[0][b], o[1][b], o[2][b], o[3][b]);
       __syncthreads();
     } else {
       // V: T' = T Q_R, i.e. the left operand is T itself: store it transposed
       float tt[4][4];
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) tt[a][b] = T[(4 * ty + a) * kApT + 4 * tx + b];
+      for (int a = 0; a < 4; ++a) {
+        const float4 v = *reinterpret_cast<const float4 *>(T + (4 * ty + a) * kApT + 4 * tx);
+        tt[a][0] = v.x, tt[a][1] = v.y, tt[a][2] = v.z, tt[a][3] = v.w;
+      }
       __syncthreads();
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) T[(4 * tx + b) * kApT + 4 * ty + a] = tt[a][b];
+      for (int b = 0; b < 4; ++b)
+        *reinterpret_cast<float4 *>(T + (4 * tx + b) * kApT + 4 * ty) =
+            make_float4(tt[0][b], tt[1][b], tt[2][b], tt[3][b]);
       __syncthreads();
     }
     bj_mm_tn(T, QR, o, ty, tx);  // (U or T) Q_R with the left operand stored transposed
 #pragma unroll
-    for (int a = 0; a < 4; ++a) {
+    for (int a = 0; a < 4; ++a) {  // columns 4 tx .. 4 tx + 3 lie in one block run: a 16-byte store
       const int i = 4 * ty + a;
       const int64_t gi = isA ? bj_index(i, IP, JP) : row0 + i;
-#pragma unroll
-      for (int b = 0; b < 4; ++b) M[gi * n + bj_index(4 * tx + b, IR, JR)] = o[a][b];
+      *reinterpret_cast<float4 *>(M + gi * n + bj_index(4 * tx, IR, JR)) = make_float4(o[a][0], o[a][1], o[a][2], o[a][3]);
     }
   }
 }
