@@ -287,7 +287,7 @@ PcaLayout pca_layout(int64_t N, int d, int r) {
   L.mean32 = take((size_t)d * 4);
   L.yh = take((size_t)d * g.ldn * 2);
   L.yl = take((size_t)d * g.ldn * 2);
-  L.part = take((size_t)g.nchunks * g.ntiles * kBM * kBM * 8);
+  L.part = take((size_t)g.nchunks * g.ntiles * kBM * kBM * 4);
   const size_t nn = (size_t)g.n * g.n * 4;
   L.A0 = take(nn);
   L.V0 = take(nn);
@@ -563,7 +563,7 @@ int hme_pca_covariance(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t
   HME_CUDA(launch_pca_mean(Xf, g, ldx, at<double>(ws, L.slab), at<double>(ws, L.mean64), at<float>(ws, L.mean32), s),
            "pca: mean");
   HME_TRY(launch_pca_cov(Xf, g, ldx, at<float>(ws, L.mean32), at<__nv_bfloat16>(ws, L.yh),
-                         at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), cov_out, at<float>(ws, L.A0),
+                         at<__nv_bfloat16>(ws, L.yl), at<float>(ws, L.part), cov_out, at<float>(ws, L.A0),
                          at<Header>(ws, 0), s));
   HME_CUDA(cudaMemcpyAsync(mean_out, at<double>(ws, L.mean64), (size_t)d * 8, cudaMemcpyDeviceToDevice, s),
            "pca: copy mean");
@@ -585,7 +585,7 @@ int hme_pca_fit(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
   HME_CUDA(launch_pca_mean(Xf, g, ldx, at<double>(ws, L.slab), at<double>(ws, L.mean64), at<float>(ws, L.mean32), s),
            "pca: mean");
   HME_TRY(launch_pca_cov(Xf, g, ldx, at<float>(ws, L.mean32), at<__nv_bfloat16>(ws, L.yh),
-                         at<__nv_bfloat16>(ws, L.yl), at<double>(ws, L.part), nullptr, at<float>(ws, L.A0),
+                         at<__nv_bfloat16>(ws, L.yl), at<float>(ws, L.part), nullptr, at<float>(ws, L.A0),
                          at<Header>(ws, 0), s));
   int sweeps = 0;
   const int rc = run_pca_jacobi(g, at<float>(ws, L.A0), at<float>(ws, L.V0), at<float>(ws, L.qbuf), at<double>(ws, L.acc), at<int32_t>(ws, L.order), components_out, variances_out,

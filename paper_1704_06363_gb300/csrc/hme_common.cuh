@@ -138,6 +138,10 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
 // bf16 matrix rows x cols (row stride ld elements), box = box_rows x 64
 // columns, 128-byte swizzle (the operand layout of the tcgen05 kernels).
 int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows);
+// bf16 blocks of rows x cols (contiguous, row stride cols), nblk of them one
+// after another; box = box_rows x 64 columns x 1 block, 128-byte swizzle.
+int make_bf16_map_blocked(CUtensorMap *m, const void *ptr, uint64_t nblk, uint64_t rows, uint64_t cols,
+                          uint32_t box_rows);
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);
@@ -189,14 +193,16 @@ cudaError_t launch_tag_hist(const int64_t *offsets, const int64_t *tag_off, cons
                             cudaStream_t s);
 // PCA (pca.cu): see the file header for the steps.
 constexpr int64_t kCovSub = 512;  // rows per fp32 (TMEM) accumulation of the covariance
+constexpr int kCovFlush = 16;     // sub-range sums per covariance work unit (fp32 register accumulation)
 constexpr int kJacobiMaxSweeps = 40;
 struct PcaGeom {
   int64_t N;
   int d, r;
   int n;           // Jacobi order: d rounded up to a multiple of 64
-  int64_t ldn;     // row pitch (elements) of the transposed split: N rounded up to 8
+  int64_t ldn;     // rows of the transposed split, padded: nchunks * R
   int mi, ntiles;  // 128-feature tiles along d; upper-triangle tiles
-  int64_t R, nchunks, nslabs;  // rows per covariance work unit, units per tile, column-sum slabs
+  int64_t R, nchunks, nslabs;  // rows per covariance work unit (= rows per block of the transposed split),
+                               // blocks (= units per tile), column-sum slabs
 };
 PcaGeom pca_geom(int64_t N, int d, int r);
 cudaError_t launch_pca_mean(const float *X, const PcaGeom &g, int64_t ldx, double *slab_sums, double *mean64,
@@ -204,7 +210,7 @@ cudaError_t launch_pca_mean(const float *X, const PcaGeom &g, int64_t ldx, doubl
 // centred transposed split, tcgen05 covariance partials, fp64 reduction into
 // cov (d x d, may be null) and A (fp32, order g.n)
 int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *mean32, __nv_bfloat16 *yh,
-                   __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s);
+                   __nv_bfloat16 *yl, float *part, double *cov, float *A, Header *hdr, cudaStream_t s);
 // Jacobi sweeps on A0 (synchronises s once per sweep), then the r leading
 // components (rows of W, r x d) and their variances (may be null)
 int run_pca_jacobi(const PcaGeom &g, float *A0, float *V0, float *Qbuf, double *acc, int32_t *order, float *W,
@@ -285,6 +291,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// TMA: 3-D tiled bulk load global -> shared (coordinates innermost first).
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int32_t c0,
+                                            int32_t c1, int32_t c2, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar), "l"(policy)
       : "memory");
 }
 

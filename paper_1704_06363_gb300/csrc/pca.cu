@@ -8,17 +8,17 @@
 //   pca_colsum      per-slab column sums of X (fp32 over 32 rows, fp64 across);
 //   pca_mean        the slab sums added in slab order / N -> mu (fp64, fp32);
 //   pca_split_t     y = x - mu (fp32) split into bf16 y = yh + yl + O(2^-16 |y|),
-//                   written transposed (YT_hi, YT_lo: d x ldn, one row per
-//                   feature), so that the covariance is a K-major contraction
-//                   over the rows for the tensor cores;
+//                   written transposed in blocks of R rows (each block a d x R
+//                   matrix, one row per feature), so that the covariance is a
+//                   K-major contraction over the rows for the tensor cores;
 //   pca_cov         tcgen05 (kind::f16, fp32 accumulate in TMEM): work units
-//                   are (row range, 128 x 128 tile (i <= j) of the upper
+//                   are (block of rows, 128 x 128 tile (i <= j) of the upper
 //                   triangle); a unit accumulates yh.yh' + yh.yl' + yl.yh' in
 //                   TMEM over kCovSub rows at a time (short fp32 sums), its
 //                   epilogue adds each such sub-result into fp32 registers
 //                   (round to nearest) while the MMAs of the next sub-range run
-//                   in the other accumulator, and every kCovFlush sub-ranges
-//                   adds the registers into the unit's fp64 partial tile;
+//                   in the other accumulator, and stores its fp32 partial tile
+//                   once (a block has at most kCovFlush sub-ranges);
 //   pca_cov_reduce  the partial tiles added in range order in fp64, / N: the
 //                   covariance (fp64, both triangles) and A (fp32, order n = d
 //                   rounded up to even, padding row and column zero);
@@ -89,12 +89,13 @@ __device__ __forceinline__ void split_bf16(float y, uint16_t &h, uint16_t &l) {
 }
 
 // A block moves 64 rows x 64 features: loads coalesced along the features,
-// stores coalesced along the rows (128 bytes per feature row).  Rows past N
-// are zero (the columns N .. ldn-1 of YT are written as zeros).
+// stores coalesced along the rows (128 bytes per feature row) into block
+// n / R of the transposed split.  Rows past N (the padding of the last block)
+// are written as zeros.
 constexpr int kTPad = 66;  // shared row pitch in 16-bit elements (33 words: few bank conflicts)
 template <bool VEC>
 __global__ void __launch_bounds__(256) pca_split_t_kernel(const float *__restrict__ X, int64_t N, int d, int64_t ldx,
-                                                          const float *__restrict__ mu, int64_t ldn,
+                                                          const float *__restrict__ mu, int64_t R,
                                                           __nv_bfloat16 *__restrict__ yh,
                                                           __nv_bfloat16 *__restrict__ yl) {
   __shared__ __align__(16) uint16_t sh[64 * kTPad];
@@ -132,16 +133,18 @@ __global__ void __launch_bounds__(256) pca_split_t_kernel(const float *__restric
   }
   __syncthreads();
 #pragma unroll
+  // the 64 rows lie in one block c of R rows (R is a multiple of 64)
+  const int64_t c = n0 / R, x0 = n0 - c * R;
   for (int k = 0; k < 2; ++k) {
     const int idx = t + 256 * k;  // 64 features x 8 chunks of 8 rows
     const int ff = idx >> 3, ch = idx & 7;
     const int f = f0 + ff;
-    const int64_t n = n0 + ch * 8;
-    if (f < d && n < N) {
+    if (f < d) {
       const uint32_t *ph = reinterpret_cast<const uint32_t *>(sh + ff * kTPad + ch * 8);
       const uint32_t *pl = reinterpret_cast<const uint32_t *>(sl + ff * kTPad + ch * 8);
-      *reinterpret_cast<uint4 *>(yh + (int64_t)f * ldn + n) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
-      *reinterpret_cast<uint4 *>(yl + (int64_t)f * ldn + n) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
+      const int64_t o = (c * d + f) * R + x0 + ch * 8;
+      *reinterpret_cast<uint4 *>(yh + o) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+      *reinterpret_cast<uint4 *>(yl + o) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
     }
   }
 }
@@ -155,12 +158,11 @@ struct CovParams {
   int mi;          // 128-feature tiles along d
   int ntiles;      // mi (mi + 1) / 2
   int64_t nunits;  // ranges x tiles
-  double *part;    // [nunits][128][128]
+  float *part;     // [nunits][128][128]
   Header *hdr;
   uint64_t limit_ns;
 };
 constexpr int kSubKb = (int)(kCovSub / kBK);  // k-blocks per TMEM accumulation
-constexpr int kCovFlush = 16;                   // sub-range sums per fp32 register accumulation
 
 // tile t of the upper triangle, enumerated row by row: (i, j), i <= j
 __device__ __forceinline__ void cov_tile(int t, int mi, int &i, int &j) {
@@ -240,11 +242,11 @@ __global__ void __launch_bounds__(kCovThreads, 1)
           const uint32_t fb = smem_u32(&full[s]);
           mbar_arrive_expect_tx(fb, kCovStageBytes);
           const uint32_t st = ring + (uint32_t)s * kCovStageBytes;
-          const int32_t x = (int32_t)(c * p.R) + kb * kBK;
-          tma_load_2d(st, &tmH, fb, x, i * kBM, pol);
-          tma_load_2d(st + kCovOpBytes, &tmL, fb, x, i * kBM, pol);
-          tma_load_2d(st + 2 * kCovOpBytes, &tmH, fb, x, j * kBM, pol);
-          tma_load_2d(st + 3 * kCovOpBytes, &tmL, fb, x, j * kBM, pol);
+          const int32_t x = kb * kBK, z = (int32_t)c;  // column within block c
+          tma_load_3d(st, &tmH, fb, x, i * kBM, z, pol);
+          tma_load_3d(st + kCovOpBytes, &tmL, fb, x, i * kBM, z, pol);
+          tma_load_3d(st + 2 * kCovOpBytes, &tmH, fb, x, j * kBM, z, pol);
+          tma_load_3d(st + 3 * kCovOpBytes, &tmL, fb, x, j * kBM, z, pol);
         }
       }
       if (!ok) {  // every copy issued must land before the CTA ends
@@ -301,17 +303,15 @@ __global__ void __launch_bounds__(kCovThreads, 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const int col0 = ((warp - 2) >> 2) * kCovHalf;
-    // Each sub-range sum (one TMEM accumulation) is added into fp32 registers
-    // (round to nearest); every kCovFlush sub-ranges, and at the end of the
-    // unit, the registers go to the unit's fp64 partial row.
+    // Each sub-range sum (one TMEM accumulation, at most kCovFlush per unit)
+    // is added into fp32 registers (round to nearest); the unit's partial
+    // tile row is stored once at its end.
     uint32_t acc_it = 0;
     bool ok = true;
     float acc[kCovHalf];
     for (int64_t u = blockIdx.x; u < p.nunits && ok; u += gridDim.x) {
       const int nkb = kblocks(u / p.ntiles);
-      double *dst = p.part + u * (int64_t)(kBM * kBM) + (int64_t)row * kBM + col0;
-      bool first_flush = true;
-      int since = 0;
+      float *dst = p.part + u * (int64_t)(kBM * kBM) + (int64_t)row * kBM + col0;
 #pragma unroll
       for (int c = 0; c < kCovHalf; ++c) acc[c] = 0.0f;
       for (int kb0 = 0; kb0 < nkb; kb0 += kSubKb, ++acc_it) {
@@ -338,23 +338,11 @@ __global__ void __launch_bounds__(kCovThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
-        if (++since == kCovFlush || kb0 + kSubKb >= nkb) {
-#pragma unroll
-          for (int c = 0; c < kCovHalf; c += 2) {
-            double2 *d2 = reinterpret_cast<double2 *>(dst + c);
-            const double x0 = (double)acc[c], x1 = (double)acc[c + 1];
-            if (first_flush) {
-              *d2 = make_double2(x0, x1);
-            } else {
-              const double2 o = *d2;
-              *d2 = make_double2(o.x + x0, o.y + x1);
-            }
-            acc[c] = acc[c + 1] = 0.0f;
-          }
-          first_flush = false;
-          since = 0;
-        }
       }
+      if (!ok) break;
+#pragma unroll
+      for (int c = 0; c < kCovHalf; c += 4)
+        *reinterpret_cast<float4 *>(dst + c) = make_float4(acc[c], acc[c + 1], acc[c + 2], acc[c + 3]);
     }
   }
   tc_fence_before();
@@ -367,7 +355,7 @@ __global__ void __launch_bounds__(kCovThreads, 1)
 
 // cov[a][b] = cov[b][a] = (sum over chunks of the partial entries, fp64, in
 // chunk order) / N for a <= b; A (order n) gets the same values in fp32.
-__global__ void __launch_bounds__(256) pca_cov_reduce_kernel(const double *__restrict__ part, int64_t nchunks,
+__global__ void __launch_bounds__(256) pca_cov_reduce_kernel(const float *__restrict__ part, int64_t nchunks,
                                                              int ntiles, int mi, int d, int n, int64_t N,
                                                              double *__restrict__ cov, float *__restrict__ A) {
   if (blockIdx.x < blockIdx.y) return;  // 32 x 32 blocks wholly below the diagonal
@@ -381,7 +369,7 @@ __global__ void __launch_bounds__(256) pca_cov_reduce_kernel(const double *__res
     const int64_t off = (int64_t)t * (kBM * kBM) + (int64_t)(a & 127) * kBM + (b & 127);
     const int64_t stride = (int64_t)ntiles * (kBM * kBM);
     double s = 0.0;
-    for (int64_t c = 0; c < nchunks; ++c) s += part[c * stride + off];
+    for (int64_t c = 0; c < nchunks; ++c) s += (double)part[c * stride + off];
     const double v = s / (double)N;
     if (cov) {
       cov[(int64_t)a * d + b] = v;
@@ -759,16 +747,23 @@ PcaGeom pca_geom(int64_t N, int d, int r) {
   g.d = d;
   g.r = r;
   g.n = (d + 63) / 64 * 64;
-  g.ldn = (N + 7) / 8 * 8;
+
   g.mi = (d + kBM - 1) / kBM;
   g.ntiles = g.mi * (g.mi + 1) / 2;
-  // row ranges: about 8 units per SM over all tiles (152 SMs assumed for
-  // the sizing only), each range a multiple of kCovSub rows
+  // Row ranges (= blocks of the transposed split) of at most kCovFlush
+  // sub-ranges, and about 8 units per SM over all tiles (152 SMs assumed for
+  // the sizing only).  A block is a contiguous d x R bf16 matrix: a k-block of
+  // 64 rows then spans d x 2R bytes (32 MB at d = 2048), where a single d x N
+  // matrix would put its 128-byte rows N x 2 bytes apart (2 MB at N = 10^6,
+  // every row on its own page).
   int64_t ranges = (8 * 152 + g.ntiles - 1) / g.ntiles;
   const int64_t subs = (N + kCovSub - 1) / kCovSub;
   if (ranges > subs) ranges = subs > 0 ? subs : 1;
-  g.R = (subs + ranges - 1) / ranges * kCovSub;
+  int64_t per = (subs + ranges - 1) / ranges;
+  if (per > kCovFlush) per = kCovFlush;
+  g.R = per * kCovSub;
   g.nchunks = (N + g.R - 1) / g.R;
+  g.ldn = g.nchunks * g.R;
   g.nslabs = (N + kColSlab - 1) / kColSlab;
   return g;
 }
@@ -783,20 +778,22 @@ cudaError_t launch_pca_mean(const float *X, const PcaGeom &g, int64_t ldx, doubl
 }
 
 int launch_pca_cov(const float *X, const PcaGeom &g, int64_t ldx, const float *mean32, __nv_bfloat16 *yh,
-                   __nv_bfloat16 *yl, double *part, double *cov, float *A, Header *hdr, cudaStream_t s) {
+                   __nv_bfloat16 *yl, float *part, double *cov, float *A, Header *hdr, cudaStream_t s) {
   const bool vec = (reinterpret_cast<uintptr_t>(X) & 15u) == 0 && ldx % 4 == 0;
-  const dim3 tg((unsigned)((g.N + 63) / 64), (unsigned)((g.d + 63) / 64));
+  const dim3 tg((unsigned)(g.ldn / 64), (unsigned)((g.d + 63) / 64));  // every row of every block, padding included
   if (vec)
-    pca_split_t_kernel<true><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.ldn, yh, yl);
+    pca_split_t_kernel<true><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.R, yh, yl);
   else
-    pca_split_t_kernel<false><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.ldn, yh, yl);
+    pca_split_t_kernel<false><<<tg, 256, 0, s>>>(X, g.N, g.d, ldx, mean32, g.R, yh, yl);
   count_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "pca: split");
   CUtensorMap mH, mL;
   int rc;
-  if ((rc = make_bf16_map(&mH, yh, (uint64_t)g.d, (uint64_t)g.N, (uint64_t)g.ldn, kBM)) != HME_OK) return rc;
-  if ((rc = make_bf16_map(&mL, yl, (uint64_t)g.d, (uint64_t)g.N, (uint64_t)g.ldn, kBM)) != HME_OK) return rc;
+  if ((rc = make_bf16_map_blocked(&mH, yh, (uint64_t)g.nchunks, (uint64_t)g.d, (uint64_t)g.R, kBM)) != HME_OK)
+    return rc;
+  if ((rc = make_bf16_map_blocked(&mL, yl, (uint64_t)g.nchunks, (uint64_t)g.d, (uint64_t)g.R, kBM)) != HME_OK)
+    return rc;
   CovParams p;
   p.N = g.N;
   p.R = g.R;
