@@ -1234,23 +1234,6 @@ int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols,
   return make_map(m, ptr, rows, cols, ld, box_rows);
 }
 
-int make_bf16_map_blocked(CUtensorMap *m, const void *ptr, uint64_t nblk, uint64_t rows, uint64_t cols,
-                          uint32_t box_rows) {
-  EncodeTiledFn enc = get_encode_fn();
-  if (!enc) return fail(HME_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
-  cuuint64_t dims[3] = {cols, rows, nblk};
-  cuuint64_t strides[2] = {cols * 2, rows * cols * 2};
-  cuuint32_t box[3] = {(cuuint32_t)kBK, box_rows, 1};
-  cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS)
-    return fail(HME_ECUDA, "cuTensorMapEncodeTiled failed (%d) for %llu blocks of %llu x %llu", (int)r,
-                (unsigned long long)nblk, (unsigned long long)rows, (unsigned long long)cols);
-  return HME_OK;
-}
-
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {

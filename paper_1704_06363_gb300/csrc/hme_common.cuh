@@ -138,10 +138,7 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
 // bf16 matrix rows x cols (row stride ld elements), box = box_rows x 64
 // columns, 128-byte swizzle (the operand layout of the tcgen05 kernels).
 int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows);
-// bf16 blocks of rows x cols (contiguous, row stride cols), nblk of them one
-// after another; box = box_rows x 64 columns x 1 block, 128-byte swizzle.
-int make_bf16_map_blocked(CUtensorMap *m, const void *ptr, uint64_t nblk, uint64_t rows, uint64_t cols,
-                          uint32_t box_rows);
+
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);

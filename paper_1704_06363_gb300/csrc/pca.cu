@@ -34,6 +34,8 @@
 //   pca_components  the leading r columns of V, normalised, with the sign rule.
 // Transform: hme_pca_transform runs the assign kernel that splits fp32 rows in
 // the kernel, with the components as its centres, in projection mode.
+#include <mutex>
+
 #include "hme_common.cuh"
 
 namespace hme {
@@ -734,6 +736,38 @@ __global__ void __launch_bounds__(256) pca_zoff_kernel(const float *__restrict__
     for (int w = 0; w < 8; ++w) t += ps[w];
     zoff[j] = (float)t;
   }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// bf16 blocks of rows x cols (contiguous, row stride cols), nblk of them one
+// after another; box = box_rows x 64 columns x 1 block, 128-byte swizzle.
+int make_bf16_map_blocked(CUtensorMap *m, const void *ptr, uint64_t nblk, uint64_t rows, uint64_t cols,
+                          uint32_t box_rows) {
+  static EncodeTiledFn enc = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      enc = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  if (!enc) return fail(HME_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t dims[3] = {cols, rows, nblk};
+  cuuint64_t strides[2] = {cols * 2, rows * cols * 2};
+  cuuint32_t box[3] = {(cuuint32_t)kBK, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(HME_ECUDA, "cuTensorMapEncodeTiled failed (%d) for %llu blocks of %llu x %llu", (int)r,
+                (unsigned long long)nblk, (unsigned long long)rows, (unsigned long long)cols);
+  return HME_OK;
 }
 
 }  // namespace
