@@ -257,3 +257,42 @@ def test_pca_benchmark_features_full_size(dev):
     ref = (Xs - mun) @ Wn.T
     bound = _tau_z(d) * (np.abs(Xs) @ np.abs(Wn).T) + 2.0 ** -22 * (np.abs(ref) + np.abs(mun @ Wn.T))
     assert np.all(np.abs(Z[rows].double().cpu().numpy() - ref) <= bound)
+
+
+def test_fit_constant_data(dev):
+    """Every row equal: the covariance is zero, every variance 0, and the
+    components are the unit vectors in index order (ties go to the lower
+    index; the padding of the Jacobi order is never chosen)."""
+    N, d, r = 500, 70, 70
+    X = torch.full((N, d), 3.25, dtype=torch.float32)
+    mu, W, lam, sweeps = _fit(X, r, dev)
+    assert np.allclose(mu, 3.25) and np.all(lam == 0.0)
+    assert np.array_equal(W, np.eye(d)[:r])
+
+
+@pytest.mark.parametrize("d", [63, 65, 129])
+def test_fit_repeated_and_zero_variances(dev, d):
+    """Duplicated features (a repeated eigenvalue and a zero one per pair),
+    constant features (zero variance), d next to a multiple of the Jacobi
+    block: the results stay valid eigenpairs of the oracle's covariance."""
+    N, r = 3000, min(d, 40)
+    X = _features(N, d, 6, seed=d)
+    X[:, 1] = X[:, 0]          # duplicate column
+    X[:, 5] = X[:, 4]
+    X[:, d - 1] = 7.0          # constant column
+    X[:, d - 2] = 0.0
+    mu, W, lam, sweeps = _fit(X, r, dev)
+    _check_fit(X.numpy(), r, mu, W, lam, sweeps)
+
+
+def test_transform_single_component(dev):
+    X = _features(999, 130, 4, seed=3)
+    Xn = X.numpy()
+    w = np.random.default_rng(1).standard_normal((1, 130))
+    W = (w / np.linalg.norm(w)).astype(np.float32)
+    mu = Xn.mean(axis=0).astype(np.float32)
+    Z = _transform(X, mu, W, dev)
+    ref = opca.transform(Xn, mu.astype(np.float64), W.astype(np.float64))
+    bound = _tau_z(130) * (np.abs(Xn.astype(np.float64)) @ np.abs(W.astype(np.float64)).T)
+    bound += 2.0 ** -22 * (np.abs(ref) + np.abs(mu.astype(np.float64) @ W.T.astype(np.float64)))
+    assert np.all(np.abs(Z - ref) <= bound)
