@@ -366,6 +366,29 @@ def run_ours(args, w):
     status = hme.hme_sync_status(ws)
     if status != hme.HME_OK:
         raise RuntimeError(f"device status {status} after the route comparison: {hme.hme_last_error()}")
+    # outside the timed steps: serving-style routing of small query batches
+    # against the final centres (one call = assign + partition), median of 20
+    for B in (256, 4096):
+        if B > N:
+            continue
+        Qb = X[:B]
+        wq = hme.workspace(hme.HME_OP_ROUTE, B, d, K, dt, device=dev)
+        eb = torch.empty(B, dtype=torch.int32, device=dev)
+        ob = torch.empty(K + 1, dtype=torch.int64, device=dev)
+        rb = torch.empty(B, dtype=torch.int32, device=dev)
+        hme.hme_route(Qb, C, eb, ob, rb, wq)
+        lat = []
+        for _ in range(20):
+            r0 = torch.cuda.Event(enable_timing=True)
+            r1 = torch.cuda.Event(enable_timing=True)
+            r0.record(stream)
+            hme.hme_route(Qb, C, eb, ob, rb, wq)
+            r1.record(stream)
+            torch.cuda.synchronize(dev)
+            lat.append(r0.elapsed_time(r1) * 1000.0)
+        if hme.hme_sync_status(wq) != hme.HME_OK:
+            raise RuntimeError(f"route of a {B}-row batch: {hme.hme_last_error()}")
+        route_ms[f"route_batch{B}_us_median"] = sorted(lat)[len(lat) // 2]
     # outside the timed steps: the same Lloyd iterations with X streamed from
     # page-locked host memory in chunks (hme_kmeans_stream), for feature sets
     # larger than HBM
