@@ -60,9 +60,12 @@ uint64_t wait_limit_ns() {
 // tiles from L2, so for bf16 features (one product, tensor-bound when K is
 // large) two row tiles share each centre stage (MT = 2): up to 256 centres per
 // N-chunk, single-buffered in TMEM when 2 x BN needs all 512 columns.  With
-// several N-chunks and few dimensions the CTA's 256 rows stay resident in
-// shared memory (ARES) and the chunks hold 128 centres (double-buffered).  fp32
-// features (three products, 2 operands per side) keep MT = 1.
+// several N-chunks and d <= 256 the CTA's 128 rows stay resident in shared
+// memory (ARES, MT = 1) and the chunks hold 256 centres, double-buffered: with
+// so short a contraction the single MMA-issuing thread, not L2, sets the pace,
+// and N = 256 halves the MMAs it issues per flop (MT = 2 with 128-centre
+// chunks measured 114 against 96 ms per assign at N = 5e7, d = 256, K = 4096).
+// fp32 features (three products, 2 operands per side) keep MT = 1.
 AssignGeom assign_geom(int d, int K, int dtype) {
   AssignGeom g;
   g.d = d;
@@ -76,9 +79,9 @@ AssignGeom assign_geom(int d, int K, int dtype) {
   g.ares = false;
   if (g.nprod == 1) {
     g.mt = 2;
-    if (K > kMaxBN && 2 * num_kb * (kBM * kBK * 2) <= 128 * 1024) {
+    if (K > kMaxBN && num_kb * (kBM * kBK * 2) <= 64 * 1024) {
       g.ares = true;
-      max_bn = 128;
+      g.mt = 1;
     }
   }
   g.nchunks = (K + max_bn - 1) / max_bn;

@@ -21,10 +21,12 @@
 // ||x_eff - c_eff||^2 differs from ||x - c||^2 by O(2^-16 |x - c| (|x| + |c|))
 // per element.
 //
-// Warp roles (192 threads, one CTA per SM, persistent over row tiles):
+// Warp roles (one CTA per SM, persistent over row tiles):
 //   warp 0      TMA producer: A and B k-blocks into an S-stage ring,
 //   warp 1      TMEM allocator and single-thread MMA issuer,
-//   warps 2..5  epilogue; warp w reads TMEM lanes 32*(w%4) .. 32*(w%4)+31.
+//   warps 2..   epilogue; warp w reads TMEM lanes 32*(w%4) .. 32*(w%4)+31,
+//               CS warps per lane quarter and row tile, each scanning its
+//               share of every chunk's columns.
 // The accumulator is double-buffered in TMEM so the epilogue of one chunk
 // overlaps the MMAs of the next.  Every wait is bounded (see
 // mbar_wait_bounded); on expiry the kernel records HME_ETIMEOUT and ends.
@@ -76,7 +78,7 @@ struct AssignParams {
   float err_ll;     // 1.0625 * 2^-14 for split fp32 operands (the dropped xl.cl), else 0
 };
 
-constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4;
+constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4, kWhereXchg = 6;
 
 // One group of 16 accumulator columns of one row: v_j = ||c_j||^2 - 2 x.c_j.
 // The running best three values (and the indices of the best two) change only
@@ -188,9 +190,14 @@ __device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row,
 //   MT     row tiles of 128 per CTA sharing each B (centre) stage: 1 or 2
 //   ARES   the CTA's A rows (all k-blocks) stay resident in shared memory for
 //          all N-chunks; only B streams through the ring
-// Threads: warp 0 TMA, warp 1 MMA, 4*MT epilogue warps.
-template <int NPROD, bool LEAN, int MT, bool ARES>
-__global__ void __launch_bounds__(64 + 128 * MT, 1)
+//   CS     epilogue warps per (row tile, TMEM lane quarter), splitting each
+//          chunk's columns in CS shares (1, 2 or 4); at the end of every tile
+//          shares 1 .. CS-1 hand their per-row states to share 0 (through
+//          shared memory, behind two bounded mbarriers), which merges them and
+//          writes the row's result
+// Threads: warp 0 TMA, warp 1 MMA, 4*MT*CS epilogue warps.
+template <int NPROD, bool LEAN, int MT, bool ARES, int CS>
+__global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
                   const AssignParams p) {
@@ -213,8 +220,13 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
   uint64_t *drain = tempty + 2;
   uint64_t *a_full = drain + 1;
   uint64_t *a_empty = a_full + 1;
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(a_empty + 1);
-  float *cnbuf = reinterpret_cast<float *>(ctrl + 512);  // one 256-float buffer per epilogue warp
+  uint64_t *xfull = a_empty + 1;          // [2 slots][4 MT groups]: shares 1 .. CS-1 have written their states
+  uint64_t *xempty = xfull + 8 * MT;      // [2 slots][4 MT groups]: ... and share 0 has read them
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(xempty + 8 * MT);
+  // ||c||^2 of the chunk: kMaxBN / CS floats per epilogue warp (its columns)
+  float *cnbuf = reinterpret_cast<float *>(ctrl + 512);
+  // per-row states handed over to share 0: [2 slots][4 MT groups][CS - 1 shares][32 lanes]
+  float4 *xchg = reinterpret_cast<float4 *>(ctrl + 512 + (size_t)4 * MT * kMaxBN * sizeof(float));
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -227,11 +239,16 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4 * MT);
+      mbar_init(smem_u32(&tempty[a]), 4 * MT * CS);
     }
     mbar_init(smem_u32(drain), 1);
     mbar_init(smem_u32(a_full), 1);
     mbar_init(smem_u32(a_empty), 1);
+    if (CS > 1)
+      for (int b = 0; b < 8 * MT; ++b) {
+        mbar_init(smem_u32(&xfull[b]), 32 * (CS - 1));
+        mbar_init(smem_u32(&xempty[b]), 32);
+      }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -378,42 +395,49 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
     }
   } else {
     // ---------------- epilogue: argmin over the accumulator rows ----------------
-    const int e = warp - 2;          // 0 .. 4*MT-1
-    const int mt = e >> 2;           // which row tile (accumulator) of the CTA tile
+    const int e = warp - 2;          // 0 .. 4*MT*CS-1
     const int q = warp & 3;          // TMEM lane quarter this warp may access
-    float *cb = cnbuf + e * kMaxBN;  // this warp's copy of ||c||^2 for the chunk
+    const int mt = (e >> 2) % MT;    // which row tile (accumulator) of the CTA tile
+    const int half = (e >> 2) / MT;  // which share of the chunk's columns
+    const int pr = mt * 4 + q;       // the group of CS warps sharing these rows
+    // columns [c0, c1) of every chunk; shares are multiples of 16 columns
+    // (trailing shares may be empty when BN is small)
+    const int cw = CS == 1 ? p.BN : ((p.BN + CS - 1) / CS + 15) / 16 * 16;
+    const int c0 = half * cw;
+    const int c1 = min(p.BN, c0 + cw);
+    float *cb = cnbuf + e * (kMaxBN / CS);  // this warp's copy of ||c||^2 of its columns
     const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
     const float sqrt_cn_max = sqrtf(cn_max);
     const int row_in_tile = mt * kBM + q * 32 + lane;
-    uint32_t acc_it = 0;
+    uint32_t acc_it = 0, tile_it = 0;
     bool ok = true;
     double obj = 0.0;
     // ||c||^2 of the next chunk is fetched into registers while the current
     // chunk is scanned; with a single chunk the buffer is filled once.
-    constexpr int kCnRegs = kMaxBN / 32;
+    constexpr int kCnRegs = kMaxBN / CS / 32;
     float cn_next[kCnRegs];
     auto fetch_cn = [&](int ch) {
 #pragma unroll
       for (int r = 0; r < kCnRegs; ++r) {
-        const int t = lane + 32 * r;
-        cn_next[r] = (t < p.BN) ? __ldg(p.cn + ch * p.BN + t) : 0.0f;
+        const int t = c0 + lane + 32 * r;
+        cn_next[r] = (t < c1) ? __ldg(p.cn + ch * p.BN + t) : 0.0f;
       }
     };
     fetch_cn(0);
     bool cb_filled = false;
-    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x) {
+    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
       int idx1 = 0, idx2 = 0;
       float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
       int li1 = 0;
       const int64_t row = (int64_t)tile * BMT + row_in_tile;
-      const float xr = row < p.N ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
+      const float xr = (half == 0 && row < p.N) ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
         if (p.nchunks > 1 || !cb_filled) {
           __syncwarp();
 #pragma unroll
           for (int r = 0; r < kCnRegs; ++r)
-            if (lane + 32 * r < p.BN) cb[lane + 32 * r] = cn_next[r];
+            if (c0 + lane + 32 * r < c1) cb[lane + 32 * r] = cn_next[r];
           __syncwarp();
           cb_filled = true;
           if (p.nchunks > 1) fetch_cn(ch + 1 < p.nchunks ? ch + 1 : 0);
@@ -431,22 +455,25 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         // 16 columns per step; the next step's tcgen05.ld is in flight while this
         // step's distances are formed.
         uint32_t ra[16], rb[16];
-        tmem_ld16(taddr, ra);
-        tmem_ld_wait(ra);
-        for (int c = 0; c < p.BN; c += 32) {
-          const bool more1 = c + 16 < p.BN, more2 = c + 32 < p.BN;
+        if (c0 < c1) {
+          tmem_ld16(taddr + (uint32_t)c0, ra);
+          tmem_ld_wait(ra);
+        }
+        for (int c = c0; c < c1; c += 32) {
+          const bool more1 = c + 16 < c1, more2 = c + 32 < c1;
+          const float *cbc = cb + (c - c0);
           if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
           if (LEAN)
-            lean_group(ra, cb + c, kbase + c, best1, best2, idx1);
+            lean_group(ra, cbc, kbase + c, best1, best2, idx1);
           else
-            epilogue_group(ra, cb + c, kbase + c, best1, best2, best3, idx1, idx2);
+            epilogue_group(ra, cbc, kbase + c, best1, best2, best3, idx1, idx2);
           if (more1) {
             tmem_ld_wait(rb);
             if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
             if (LEAN)
-              lean_group(rb, cb + c + 16, kbase + c + 16, lb1, lb2, li1);
+              lean_group(rb, cbc + 16, kbase + c + 16, lb1, lb2, li1);
             else
-              epilogue_group(rb, cb + c + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
+              epilogue_group(rb, cbc + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
             if (more2) tmem_ld_wait(ra);
           }
         }
@@ -460,6 +487,66 @@ __global__ void __launch_bounds__(64 + 128 * MT, 1)
         best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
         best1 = take_b ? lb1 : best1;
         idx1 = take_b ? li1 : idx1;
+      }
+      if (CS > 1) {
+        // Hand-over of the other shares' states.  Two slots alternate by
+        // tile; a slot is rewritten only after share 0 has read it.
+        const uint32_t slot = tile_it & 1u, use = tile_it >> 1;
+        const int b = (int)slot * 4 * MT + pr;
+        float4 *xs = xchg + (b * (CS - 1)) * 32 + lane;
+        if (half > 0) {
+          if (!mbar_wait_bounded(smem_u32(&xempty[b]), (use & 1u) ^ 1u, p.limit_ns, p.hdr, kWhereXchg)) {
+            ok = false;
+            break;
+          }
+          // indices < 2^16 (K <= 16384): both fit one word
+          xs[(half - 1) * 32] =
+              make_float4(best1, best2, best3, __uint_as_float((uint32_t)idx1 | ((uint32_t)idx2 << 16)));
+          mbar_arrive(smem_u32(&xfull[b]));
+          continue;
+        }
+        if (!mbar_wait_bounded(smem_u32(&xfull[b]), use & 1u, p.limit_ns, p.hdr, kWhereXchg)) {
+          ok = false;
+          break;
+        }
+        float4 os[CS > 1 ? CS - 1 : 1];
+#pragma unroll
+        for (int h = 0; h < CS - 1; ++h) os[h] = xs[h * 32];
+        mbar_arrive(smem_u32(&xempty[b]));
+        // The merged result is the lexicographic minimum over (value, index)
+        // and the smallest remaining values: independent of the merge order.
+#pragma unroll
+        for (int h = 0; h < CS - 1; ++h) {
+          const float4 o = os[h];
+          const uint32_t oi = __float_as_uint(o.w);
+          const int o1 = (int)(oi & 0xffffu), o2 = (int)(oi >> 16);
+          if (LEAN) {
+            const bool take_o = o.x < best1 || (o.x == best1 && o1 < idx1);
+            best2 = fminf(fmaxf(best1, o.x), fminf(best2, o.y));
+            best1 = take_o ? o.x : best1;
+            idx1 = take_o ? o1 : idx1;
+          } else {
+            // insert the other share's best two (value, then index) and its third value
+            auto insert = [&](float v, int i) {
+              if (v < best1 || (v == best1 && i < idx1)) {
+                best3 = best2;
+                best2 = best1;
+                idx2 = idx1;
+                best1 = v;
+                idx1 = i;
+              } else if (v < best2 || (v == best2 && i < idx2)) {
+                best3 = best2;
+                best2 = v;
+                idx2 = i;
+              } else {
+                best3 = fminf(best3, v);
+              }
+            };
+            insert(o.x, o1);
+            insert(o.y, o2);
+            best3 = fminf(best3, o.z);
+          }
+        }
       }
       if (row < p.N) obj += finish_row<LEAN>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
     }
@@ -938,11 +1025,17 @@ __device__ __forceinline__ float warp_sum_f(float s) {
 template <int DT, int VW>
 __global__ void __launch_bounds__(256) rescore_pair_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
                                                            const float *__restrict__ C, int32_t *labels, float *mind,
-                                                           Header *hdr, const int32_t *__restrict__ flagged) {
+                                                           Header *hdr, const int32_t *__restrict__ flagged,
+                                                           unsigned long long *full_keys_end) {
   const int lane = threadIdx.x & 31;
   const int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int nw = (gridDim.x * blockDim.x) >> 5;
   const uint32_t count = *((volatile uint32_t *)&hdr->rescore_count);
+  if (full_keys_end) {  // the all-K re-score that follows merges into these keys
+    const uint32_t nfull = *((volatile uint32_t *)&hdr->rescore_full_count);
+    for (uint32_t f = blockIdx.x * blockDim.x + threadIdx.x; f < nfull; f += gridDim.x * blockDim.x)
+      full_keys_end[-1 - (int64_t)f] = ~0ull;
+  }
   double obj = 0.0;
   for (uint32_t f = gw; f < count; f += nw) {
     const int64_t row = flagged[3 * f + 0];
@@ -1057,29 +1150,47 @@ __global__ void __launch_bounds__(256) rescore_row_kernel(const void *__restrict
 }
 
 // Exact re-score of near-tie rows against all K centres: a small tiled
-// "distance GEMM" on the CUDA cores.  A block takes 32 queued rows and walks
-// the centres 64 at a time and the dimensions 32 at a time through shared
-// memory; thread (ty, tx) of a 16 x 16 grid owns rows {ty, ty+16} and centres
-// {tx, tx+16, tx+32, tx+48}.  sum_j (x_j - c_j)^2 is formed in fp32 per 32-wide
-// chunk and the chunk sums are added in fp32 (relative error below
-// (32 + d/32) 2^-24, all terms non-negative); the minimum over centres keeps
-// the lowest index among equal values.
+// "distance GEMM" on the CUDA cores.  A work item is 32 queued rows and one
+// slice of the centres, walked 64 centres and 32 dimensions at a time through
+// shared memory; thread (ty, tx) of a 16 x 16 grid owns rows {ty, ty+16} and
+// centres {tx, tx+16, tx+32, tx+48}.  sum_j (x_j - c_j)^2 is formed in fp32
+// per 32-wide chunk and the chunk sums are added in fp32 (relative error below
+// (32 + d/32) 2^-24, all terms non-negative).  With many queued rows a slice
+// is all K centres; with few (a small routed batch) the centres are split
+// over the blocks so that the work still spreads over the GPU.  A slice's best
+// (distance, centre) per row is merged with a 64-bit atomicMin on
+// (distance bits << 32 | centre): the distances are non-negative, so their
+// bit patterns order like the values, and equal distances keep the lower
+// centre.  rescore_full_finish_kernel then writes labels, distances and the
+// objective.
+//
+// The keys of queued row f sit at full_keys_end[-1 - f]: the 8-byte aligned
+// tail of the pair queue (3 words per row of the call).  Rows queued for a
+// pair (3 words each) and for all K (2 words each) number at most N together,
+// so 3 pairs + 2 full <= 3N - full <= 3N - 1 words: the keys never reach a
+// queued pair.
 constexpr int kFR = 32, kFC = 64, kFD = 32;
 
 template <int DT>
 __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
-                                                           const float *__restrict__ C, int K, int32_t *labels,
-                                                           float *mind, Header *hdr,
-                                                           const int32_t *__restrict__ full_rows) {
+                                                           const float *__restrict__ C, int K, const Header *hdr,
+                                                           const int32_t *__restrict__ full_rows,
+                                                           unsigned long long *full_keys_end) {
   __shared__ float xs[kFR][kFD + 1];
   __shared__ float cs[kFC][kFD + 1];
   __shared__ float best_v[kFR];
   __shared__ int best_k[kFR];
   __shared__ int64_t rows[kFR];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const uint32_t count = *((volatile uint32_t *)&hdr->rescore_full_count);
-  double obj = 0.0;
-  for (uint32_t b0 = blockIdx.x * kFR; b0 < count; b0 += gridDim.x * kFR) {
+  const uint32_t count = *((volatile const uint32_t *)&hdr->rescore_full_count);
+  const uint32_t ntiles = (count + kFR - 1) / kFR;
+  const int kt = (K + kFC - 1) / kFC;  // tiles of kFC centres
+  const int ks = (int)min((uint32_t)kt, max(1u, gridDim.x / max(ntiles, 1u)));  // slices per row tile
+  const uint32_t items = ntiles * (uint32_t)ks;
+  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) {
+    const uint32_t b0 = (it / (uint32_t)ks) * kFR;
+    const int sl = (int)(it % (uint32_t)ks);
+    const int kbeg = (sl * kt / ks) * kFC, kend = min(K, ((sl + 1) * kt / ks) * kFC);
     const int nr = (int)min((uint32_t)kFR, count - b0);
     if (threadIdx.x < kFR) {
       rows[threadIdx.x] = threadIdx.x < nr ? (int64_t)full_rows[b0 + threadIdx.x] : -1;
@@ -1087,7 +1198,7 @@ __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restric
       best_k[threadIdx.x] = 0;
     }
     __syncthreads();
-    for (int k0 = 0; k0 < K; k0 += kFC) {
+    for (int k0 = kbeg; k0 < kend; k0 += kFC) {
       float tot[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
       for (int j0 = 0; j0 < d; j0 += kFD) {
         for (int e = threadIdx.x; e < kFR * kFD; e += 256) {
@@ -1161,12 +1272,27 @@ __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restric
     }
     __syncthreads();
     if (threadIdx.x < nr) {
-      const int64_t row = rows[threadIdx.x];
-      labels[row] = best_k[threadIdx.x];
-      if (mind) mind[row] = best_v[threadIdx.x];
-      obj += (double)best_v[threadIdx.x];
+      const unsigned long long key =
+          ((unsigned long long)__float_as_uint(best_v[threadIdx.x]) << 32) | (uint32_t)best_k[threadIdx.x];
+      atomicMin(&full_keys_end[-1 - (int64_t)(b0 + threadIdx.x)], key);
     }
     __syncthreads();
+  }
+}
+
+// The all-K re-score's result per queued row: label, distance, objective.
+__global__ void __launch_bounds__(256) rescore_full_finish_kernel(int32_t *labels, float *mind, Header *hdr,
+                                                                  const int32_t *__restrict__ full_rows,
+                                                                  const unsigned long long *full_keys_end) {
+  const uint32_t count = *((volatile uint32_t *)&hdr->rescore_full_count);
+  double obj = 0.0;
+  for (uint32_t f = blockIdx.x * blockDim.x + threadIdx.x; f < count; f += gridDim.x * blockDim.x) {
+    const unsigned long long key = full_keys_end[-1 - (int64_t)f];
+    const int64_t row = full_rows[f];
+    const float v = __uint_as_float((uint32_t)(key >> 32));
+    labels[row] = (int32_t)(uint32_t)(key & 0xffffffffu);
+    if (mind) mind[row] = v;
+    obj += (double)v;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
@@ -1234,6 +1360,10 @@ int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols,
   return make_map(m, ptr, rows, cols, ld, box_rows);
 }
 
+// Epilogue warps per lane quarter of the resident-row kernel.  Two measured
+// 96 ms per assign at N = 5e7, d = 256, K = 4096; one 117 ms, four 104 ms.
+constexpr int kAresCS = 2;
+
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
@@ -1262,7 +1392,11 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   const int nops = g.nprod == 3 ? 2 : 1;
   p.a_res_bytes = g.ares ? (uint32_t)(g.mt * p.num_kb * nops) * p.a_bytes : 0u;
   p.stage_bytes = nops * ((g.ares ? 0u : (uint32_t)g.mt * p.a_bytes) + p.b_bytes);
-  const size_t ctrl_bytes = 512 + (size_t)4 * g.mt * kMaxBN * sizeof(float);
+  // epilogue warps per (row tile, lane quarter): two for bf16 features, whose
+  // one product per k-step leaves the epilogue scan as the longer pipeline
+  const int cs = g.nprod == 3 ? 1 : (g.ares ? kAresCS : 2);
+  const size_t ctrl_bytes = 512 + (size_t)4 * g.mt * kMaxBN * sizeof(float) +
+                            (size_t)2 * 4 * g.mt * (cs - 1) * 32 * sizeof(float4);
   const size_t budget = 227 * 1024 - 1024 - ctrl_bytes - p.a_res_bytes;
   int stages = (int)(budget / p.stage_bytes);
   if (stages > 8) stages = 8;
@@ -1293,14 +1427,14 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
   if (g.nprod == 3)
-    kern = lean ? assign_kernel<3, true, 1, false> : assign_kernel<3, false, 1, false>;
+    kern = lean ? assign_kernel<3, true, 1, false, 1> : assign_kernel<3, false, 1, false, 1>;
   else if (g.ares)
-    kern = assign_kernel<1, true, 2, true>;
+    kern = assign_kernel<1, true, 1, true, kAresCS>;
   else
-    kern = lean ? assign_kernel<1, true, 2, false> : assign_kernel<1, false, 2, false>;
+    kern = lean ? assign_kernel<1, true, 2, false, 2> : assign_kernel<1, false, 2, false, 2>;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
-  kern<<<grid, 64 + 128 * g.mt, smem, s>>>(mA0, mA1, mB0, mB1, p);
+  kern<<<grid, 64 + 128 * g.mt * cs, smem, s>>>(mA0, mA1, mB0, mB1, p);
   count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");
@@ -1395,7 +1529,7 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
 }
 
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
-                           int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           int32_t *labels, float *mind, Header *hdr, int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   const int grid = num_sms() * 4;
@@ -1404,6 +1538,9 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
   const bool row_path = K <= 128;
   const bool cvec = (reinterpret_cast<uintptr_t>(C) & 15u) == 0 && d % 4 == 0;
   const size_t row_smem = (size_t)d * sizeof(float);
+  // keys of the all-K re-score: the 8-byte aligned tail of the pair queue (3N words)
+  unsigned long long *keys_end =
+      row_path ? nullptr : reinterpret_cast<unsigned long long *>(flagged + ((3 * N) & ~(int64_t)1));
   if (row_path && row_smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(dtype == HME_BF16 ? rescore_row_kernel<HME_BF16, 1>
                                                            : (cvec ? rescore_row_kernel<HME_F32, 4>
@@ -1413,26 +1550,27 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
   }
   if (dtype == HME_BF16) {
     if (al && d % 8 == 0 && ldx % 8 == 0)
-      rescore_pair_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     else
-      rescore_pair_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     if (row_path)
       rescore_row_kernel<HME_BF16, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else
-      rescore_full_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+      rescore_full_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   } else {
     if (al && d % 4 == 0 && ldx % 4 == 0)
-      rescore_pair_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     else
-      rescore_pair_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged);
+      rescore_pair_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     if (row_path && cvec)
       rescore_row_kernel<HME_F32, 4><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else if (row_path)
       rescore_row_kernel<HME_F32, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else
-      rescore_full_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+      rescore_full_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   }
-  count_launch(2);
+  if (!row_path) rescore_full_finish_kernel<<<grid, 256, 0, s>>>(labels, mind, hdr, full_rows, keys_end);
+  count_launch(row_path ? 2 : 3);
   return cudaGetLastError();
 }
 

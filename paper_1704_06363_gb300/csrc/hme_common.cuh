@@ -140,7 +140,7 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
 int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld, uint32_t box_rows);
 
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
-                           int32_t *labels, float *mind, Header *hdr, const int32_t *flagged,
+                           int32_t *labels, float *mind, Header *hdr, int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);
 cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
                              int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,

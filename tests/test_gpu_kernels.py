@@ -205,6 +205,34 @@ def test_assign_near_ties_are_rescored_exactly(dev, dtype, K, copies):
     assert st["mismatches"] <= st["near_ties"]
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_small_batch_all_k_rescore_splits_the_centres(dev, dtype):
+    """A few near-tie rows against many centres: the all-K re-score splits the
+    centres over the blocks (up to 32 slices per row tile here) and merges the
+    slices' best per row; labels, distances and the objective match the oracle
+    for an assign and for a route of the same batch."""
+    B, d, K = 37, 96, 2000
+    X = _mixture(B, d, 8, dtype, seed=77)
+    C = hme_synth.random_centroids(K, d, seed=78, scale=3.0)
+    g = torch.Generator().manual_seed(79)
+    C[:B] = X.float()
+    for r in (1, 2):  # three centres 1e-5 apart at every row: all-K re-scores
+        C[r * B:(r + 1) * B] = C[:B] + 1e-5 * torch.randn(B, d, generator=g)
+    lab, md, obj = _assign(X, C, dev)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ROUTE, B, d, K, dt, device=dev)
+    expert = torch.empty(B, dtype=torch.int32, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    order = torch.empty(B, dtype=torch.int32, device=dev)
+    hme.hme_route(X.to(dev), C.to(dev), expert, offs, order, ws)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    e = expert.cpu().numpy()
+    assert np.array_equal(e, lab)
+    parity.check_partition(dict(offsets=offs.cpu().numpy(), perm=order.cpu().numpy()), e, K)
+
+
 def test_route_reuses_prepared_features(dev):
     N, d, K = 4000, 128, 16
     X = _mixture(N, d, K, "f32", seed=8)
