@@ -78,6 +78,7 @@ ASSIGN_CASES = [
     (129, 64, 1, "f32", None),
     (129, 64, 1, "bf16", None),
     (2000, 512, 1024, "f32", None),
+    (2000, 512, 1024, "bf16", None),  # several N-chunks, rows streamed (d > 256): MT = 2, lean scan
     (2000, 256, 4096, "bf16", None),
     (4100, 2048, 64, "f32", None),
     (4100, 2048, 256, "bf16", None),
