@@ -62,3 +62,26 @@ def test_single_process_timing_is_unchanged():
     sys.path.insert(0, ROOT)
     import bench
     assert bench.max_over_ranks(3.5) == 3.5
+
+
+def test_profiled_traffic_only_for_the_profiled_source(tmp_path, monkeypatch):
+    """roofline.traffic comes from a committed ncu summary only while the kernel
+    source hashes to the value recorded with the counters."""
+    import hashlib
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    csrc = tmp_path / "paper_1704_06363_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "profiles").mkdir()
+    src = csrc / "k.cu"
+    src.write_text("// kernel v1\n")
+    sha = hashlib.sha256(src.read_bytes()).hexdigest()
+    (tmp_path / "profiles" / "k_work.md").write_text(
+        f"traffic_bytes_per_launch: 1.5e+09\nsource_sha256: {sha}\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profiled_traffic("k.cu", "k_work") == 1.5e9
+    assert bench.profiled_traffic("k.cu", "missing") is None
+    src.write_text("// kernel v2\n")  # the kernel changed since the capture
+    assert bench.profiled_traffic("k.cu", "k_work") is None
