@@ -120,6 +120,9 @@ HME_API int hme_sync_status(void *ws, void *stream);
  * X: N x d (ldx, dtype), read only.  C_out: K x d float32, written (each row a
  * copy of a row of X).  Requires N >= 1.  Not on the timed Lloyd path: it
  * makes about 2K kernel launches.
+ * Errors: HME_EINVAL for N < 1, an unknown method, sizes outside the limits, a
+ * NULL X or C_out; HME_ENOMEM for a workspace smaller than
+ * hme_workspace_bytes(HME_OP_INIT, ...).
  */
 HME_API int hme_kmeans_init(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
                     uint64_t seed, int32_t method, float *C_out, void *ws, size_t ws_bytes, void *stream);
@@ -135,7 +138,11 @@ HME_API int hme_kmeans_init(const void *X, int64_t N, int32_t d, int64_t ldx, in
  * with K <= 256 whose rows TMA can read (X on a 16-byte boundary,
  * ldx % 4 == 0) split each fp32 row inside the kernel as it arrives: one pass
  * over X instead of three for a one-off call.  With it they read the prepared
- * split, which streams faster when the same X is assigned many times.
+ * split, which streams faster when the same X is assigned many times.  (The
+ * split and the norms are this library's evaluation of Eq. 2's distances,
+ * not a step of the paper.)
+ * Errors: HME_EINVAL for sizes outside the limits or a NULL or misaligned X;
+ * HME_ENOMEM for a workspace smaller than hme_workspace_bytes(HME_OP_ASSIGN, ...).
  */
 HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
                          void *ws, size_t ws_bytes, void *stream);
@@ -198,6 +205,8 @@ HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t
  * untaken rows).  When every row is taken, a remaining empty centre is kept.
  * *n_reseeded_out (device int32, may be NULL) = clusters re-seeded.
  * Labels outside [0, K) are skipped and reported by hme_sync_status.
+ * Errors: HME_EINVAL for sizes outside the limits, a NULL X, C_inout or (N > 0)
+ * labels; HME_ENOMEM for a workspace smaller than hme_workspace_bytes(HME_OP_ASSIGN, ...).
  */
 HME_API int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype,
                                  const int32_t *labels, const int32_t *prev_labels, const float *mind, int32_t K,
@@ -232,6 +241,10 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
  * when ws already holds Q prepared by hme_prepare_features or a PREPARE_OUT
  * call (e.g. routing the training set with the workspace of the Lloyd loop:
  * HME_OP_ROUTE and HME_OP_ASSIGN sizes agree).
+ * Errors: HME_EINVAL for sizes outside the limits, a NULL or misaligned Q, a
+ * NULL C or offsets_out, a NULL expert_out / order_out with B > 0, unknown or
+ * conflicting flags; HME_ENOMEM for a workspace smaller than
+ * hme_workspace_bytes(HME_OP_ROUTE, ...).
  */
 HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, const float *C, int32_t K,
                       int32_t flags, int32_t *expert_out, int64_t *offsets_out, int32_t *order_out, void *ws,
@@ -257,6 +270,11 @@ HME_API int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t 
  * d, K, dtype) bytes of device memory.  The call creates one stream and four
  * events of its own for the copies (so it cannot be captured into a graph);
  * the caller's stream is ordered after all of its work.
+ * Errors: HME_EINVAL for N < 1, iters < 0, chunk_rows < 1, ldx < d, sizes
+ * outside the limits, a NULL X, C_inout, labels_out or mind_out, X in pageable
+ * host memory, a NULL or misaligned ws; HME_ENOMEM for a workspace smaller than
+ * hme_workspace_bytes(HME_OP_STREAM, chunk_rows, ...); HME_ECUDA when creating
+ * the copy stream or events or a copy fails.
  */
 HME_API int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, int32_t K,
                               int32_t iters, int64_t chunk_rows, float *C_inout, int32_t *labels_out, float *mind_out,
@@ -342,6 +360,12 @@ HME_API int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K, i
  *   and mean.components_j (fp64, stored fp32) subtracted in the epilogue.
  *   1 <= r <= 256; X on a 16-byte boundary with ldx % 4 == 0 (TMA).
  *   Workspace: hme_workspace_bytes(HME_OP_PCA, 0, d, r, HME_F32) or larger.
+ *
+ * Errors of all three: HME_EINVAL for a dtype other than HME_F32, sizes
+ * outside the limits or the bounds above (hme_pca_fit: d <= 8192), NULL
+ * outputs, ldz < r, a misaligned X (hme_pca_transform); HME_ENOMEM for a
+ * workspace smaller than hme_workspace_bytes(HME_OP_PCA, ...); HME_EINTERNAL
+ * as above.
  */
 HME_API int hme_pca_covariance(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, double *mean_out,
                                double *cov_out, void *ws, size_t ws_bytes, void *stream);
