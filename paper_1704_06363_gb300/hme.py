@@ -88,8 +88,25 @@ def _check(rc: int, fn: str):
         raise HmeError(rc, fn, lib().hme_last_error().decode(errors="replace"))
 
 
-def _ptr(t: Optional[torch.Tensor]):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+def _ptr(t: Optional[torch.Tensor], host_ok: bool = False):
+    """The tensor's address for the C ABI, which takes device pointers on the
+    current CUDA device (hme_kmeans_stream's features may also be page-locked
+    host memory).  Anything else would reach a kernel as an address it cannot
+    read, so it is refused here, before any call into the library."""
+    if t is None:
+        return None
+    if t.is_cuda:
+        cur = torch.cuda.current_device()
+        if t.device.index != cur:
+            raise HmeError(HME_EINVAL, "argument check",
+                           f"a tensor on {t.device} was passed while the current CUDA device is cuda:{cur}; "
+                           "the library runs on the current device")
+    elif not (host_ok and t.is_pinned()):
+        raise HmeError(HME_EINVAL, "argument check",
+                       "arguments must be CUDA tensors (device memory)"
+                       + (" or, for the features, page-locked host tensors" if host_ok else "")
+                       + f"; got a tensor on {t.device}")
+    return ctypes.c_void_p(t.data_ptr())
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -111,7 +128,7 @@ def _features(X: torch.Tensor):
 
 
 def _ws(ws: torch.Tensor):
-    return ctypes.c_void_p(ws.data_ptr()), ws.numel() * ws.element_size()
+    return _ptr(ws), ws.numel() * ws.element_size()
 
 
 def hme_workspace_bytes(op: int, N: int, d: int, K: int, dtype: int) -> int:
@@ -202,7 +219,8 @@ def hme_kmeans_stream(X: torch.Tensor, K: int, iters: int, chunk_rows: int, C_in
     """Lloyd's iterations on X in page-locked host memory (or device memory), streamed in chunks."""
     N, d, ldx, dt = _features(X)
     w, wb = _ws(ws)
-    _check(lib().hme_kmeans_stream(_ptr(X), N, d, ldx, dt, K, iters, chunk_rows, _ptr(C_inout), _ptr(labels_out),
+    _check(lib().hme_kmeans_stream(_ptr(X, host_ok=True), N, d, ldx, dt, K, iters, chunk_rows, _ptr(C_inout),
+                                   _ptr(labels_out),
                                    _ptr(mind_out), _ptr(objectives_out), _ptr(counts_out), _ptr(n_reseeded_out), w,
                                    wb, _stream(stream)), "hme_kmeans_stream")
 

@@ -147,3 +147,32 @@ def test_pca_host_validation(lib):
     c.argtypes = [p, i64, i32, i64, i32, p, p, p, ctypes.c_size_t, p]
     assert c(p(256), 0, 4, 4, 0, p(256), p(256), p(256), 1 << 20, None) == 1  # N = 0
     assert c(p(256), 10, 4, 4, 0, None, p(256), p(256), 1 << 20, None) == 1
+
+
+def test_binding_refuses_host_tensors_before_calling_the_library():
+    """The C ABI takes device pointers; the binding refuses CPU tensors (and, for
+    the streamed features, pageable host memory) with HME_EINVAL before any
+    call, so that no kernel is handed a host address."""
+    import torch
+
+    from paper_1704_06363_gb300 import hme
+
+    X = torch.zeros(8, 4)
+    C = torch.zeros(2, 4)
+    ws = torch.zeros(1 << 16, dtype=torch.uint8)
+    cases = [
+        lambda: hme.hme_assign(X, C, torch.zeros(8, dtype=torch.int32), ws),
+        lambda: hme.hme_prepare_features(X, 2, ws),
+        lambda: hme.hme_route(X, C, torch.zeros(8, dtype=torch.int32), torch.zeros(3, dtype=torch.int64),
+                              torch.zeros(8, dtype=torch.int32), ws),
+        lambda: hme.hme_partition(torch.zeros(8, dtype=torch.int32), 2, torch.zeros(2, dtype=torch.int64),
+                                  torch.zeros(3, dtype=torch.int64), torch.zeros(8, dtype=torch.int32), ws),
+        lambda: hme.hme_kmeans_stream(X, 2, 1, 4, C, torch.zeros(8, dtype=torch.int32), torch.zeros(8), ws),
+        lambda: hme.hme_pca_covariance(X, torch.zeros(4, dtype=torch.float64),
+                                       torch.zeros(4, 4, dtype=torch.float64), ws),
+    ]
+    for call in cases:
+        with pytest.raises(hme.HmeError) as ei:
+            call()
+        assert ei.value.code == hme.HME_EINVAL
+        assert "CUDA tensors" in str(ei.value)
