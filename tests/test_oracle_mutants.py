@@ -63,6 +63,12 @@ C_MUTANTS = [
     ("splitmix64: the counter starts at 0",
      "uint64_t z = seed + (j + 1) * SM64_GAMMA;",
      "uint64_t z = seed + j * SM64_GAMMA;"),
+    ("objective: the centre table indexed without its row stride",
+     "- Ct[(int64_t)labels[i] * d + j];",
+     "- Ct[(int64_t)labels[i] + j];"),
+    ("objective: unsquared distances summed",
+     "        J += s;\n    }\n    free(Ct);\n    *objective = J;",
+     "        J += sqrt(s);\n    }\n    free(Ct);\n    *objective = J;"),
     ("tag statistics: l1 / l2^2 instead of l1 / l2",
      "l1 / sqrt(l2sq)",
      "l1 / l2sq"),
