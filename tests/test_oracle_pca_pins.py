@@ -41,6 +41,24 @@ def test_known_spectrum_and_directions():
         assert W[k, np.argmax(np.abs(W[k]))] > 0
 
 
+def test_projection_of_the_known_spectrum_rows():
+    """Row mu +- sqrt(d lam_j) q_j projects to +- sqrt(d lam_j) s_j e_j on the
+    r leading components (s_j the component's sign) and to 0 for j >= r."""
+    d, r = 10, 4
+    lam = np.array([8.0, 6.0, 5.0, 3.0, 2.0, 1.5, 1.0, 0.6, 0.3, 0.1])
+    mu = np.linspace(2.0, -1.0, d)
+    X, Q = _known_spectrum(d, lam, mu, seed=17)
+    m, W, _, _ = pca.fit(X, r)
+    Z = pca.transform(X, m, W)
+    signs = np.sign(np.sum(W * Q[:, :r].T, axis=1))  # W[k] = s_k q_k
+    for j in range(d):
+        want = np.zeros(r)
+        if j < r:
+            want[j] = signs[j] * np.sqrt(d * lam[j])
+        assert np.allclose(Z[2 * j], want, atol=1e-9)
+        assert np.allclose(Z[2 * j + 1], -want, atol=1e-9)
+
+
 def test_two_by_two_closed_form():
     rng = np.random.default_rng(7)
     X = rng.standard_normal((500, 2)) @ np.array([[2.0, 0.7], [0.0, 0.9]]) + np.array([4.0, -1.0])
