@@ -109,6 +109,39 @@ def _ptr(t: Optional[torch.Tensor], host_ok: bool = False):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _arg(t: Optional[torch.Tensor], name: str, dtype: torch.dtype, numel: int, host_ok: bool = False):
+    """The address of an array argument after checking what the kernels assume
+    of it: element type `dtype`, contiguous, at least `numel` elements (the
+    kernels read or write that many), on the current device.  A mismatch would
+    let a kernel write past the tensor or misread it, so it is refused with
+    HME_EINVAL before any call into the library.  None passes through (the C
+    ABI's NULL)."""
+    if t is None:
+        return None
+    if t.dtype != dtype:
+        raise HmeError(HME_EINVAL, "argument check", f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise HmeError(HME_EINVAL, "argument check", f"{name} must be contiguous")
+    if t.numel() < numel:
+        raise HmeError(HME_EINVAL, "argument check",
+                       f"{name} has {t.numel()} elements; the call needs at least {numel}")
+    return _ptr(t, host_ok)
+
+
+def _labels(t: torch.Tensor, name: str = "labels") -> int:
+    """N of a label vector: a 1-D int32 tensor."""
+    if t.dim() != 1:
+        raise HmeError(HME_EINVAL, "argument check", f"{name} must be 1-D, got shape {tuple(t.shape)}")
+    return t.shape[0]
+
+
+def _centres(C: torch.Tensor, d: int, name: str = "C") -> int:
+    """K of a centre matrix: K x d float32, contiguous."""
+    if C.dim() != 2 or C.shape[1] != d:
+        raise HmeError(HME_EINVAL, "argument check", f"{name} must be K x {d}, got shape {tuple(C.shape)}")
+    return C.shape[0]
+
+
 def _stream(stream) -> ctypes.c_void_p:
     if stream is None:
         stream = torch.cuda.current_stream()
@@ -128,6 +161,8 @@ def _features(X: torch.Tensor):
 
 
 def _ws(ws: torch.Tensor):
+    if not ws.is_contiguous():
+        raise HmeError(HME_EINVAL, "argument check", "the workspace must be contiguous")
     return _ptr(ws), ws.numel() * ws.element_size()
 
 
@@ -156,8 +191,11 @@ def hme_last_error() -> str:
 def hme_kmeans_init(X: torch.Tensor, K: int, seed: int, method: int, C_out: torch.Tensor, ws: torch.Tensor,
                     stream=None):
     N, d, ldx, dt = _features(X)
+    if _centres(C_out, d, "C_out") != K:
+        raise HmeError(HME_EINVAL, "argument check", f"C_out must have K = {K} rows")
     w, wb = _ws(ws)
-    _check(lib().hme_kmeans_init(_ptr(X), N, d, ldx, dt, K, seed & (2**64 - 1), method, _ptr(C_out), w, wb,
+    _check(lib().hme_kmeans_init(_ptr(X), N, d, ldx, dt, K, seed & (2**64 - 1), method,
+                                 _arg(C_out, "C_out", torch.float32, K * d), w, wb,
                                  _stream(stream)), "hme_kmeans_init")
 
 
@@ -171,10 +209,13 @@ def hme_assign(X: torch.Tensor, C: torch.Tensor, labels_out: torch.Tensor, ws: t
                mind_out: Optional[torch.Tensor] = None, objective_out: Optional[torch.Tensor] = None,
                flags: int = HME_ASSIGN_DEFAULT, stream=None):
     N, d, ldx, dt = _features(X)
-    K = C.shape[0]
+    K = _centres(C, d)
     w, wb = _ws(ws)
-    _check(lib().hme_assign(_ptr(X), N, d, ldx, dt, _ptr(C), K, flags, _ptr(labels_out), _ptr(mind_out),
-                            _ptr(objective_out), w, wb, _stream(stream)), "hme_assign")
+    _check(lib().hme_assign(_ptr(X), N, d, ldx, dt, _arg(C, "C", torch.float32, K * d), K, flags,
+                            _arg(labels_out, "labels_out", torch.int32, N),
+                            _arg(mind_out, "mind_out", torch.float32, N),
+                            _arg(objective_out, "objective_out", torch.float64, 1), w, wb, _stream(stream)),
+           "hme_assign")
 
 
 def hme_update_centroids(X: torch.Tensor, labels: torch.Tensor, mind: Optional[torch.Tensor], C_inout: torch.Tensor,
@@ -183,11 +224,15 @@ def hme_update_centroids(X: torch.Tensor, labels: torch.Tensor, mind: Optional[t
                          prev_labels: Optional[torch.Tensor] = None, stream=None):
     """Centre step.  prev_labels: the labels of the previous call on this ws (incremental update)."""
     N, d, ldx, dt = _features(X)
-    K = C_inout.shape[0]
+    K = _centres(C_inout, d, "C_inout")
     w, wb = _ws(ws)
-    _check(lib().hme_update_centroids(_ptr(X), N, d, ldx, dt, _ptr(labels), _ptr(prev_labels), _ptr(mind), K,
-                                      _ptr(C_inout),
-                                      _ptr(counts_out), _ptr(n_reseeded_out), _ptr(objective_out), w, wb,
+    _check(lib().hme_update_centroids(_ptr(X), N, d, ldx, dt, _arg(labels, "labels", torch.int32, N),
+                                      _arg(prev_labels, "prev_labels", torch.int32, N),
+                                      _arg(mind, "mind", torch.float32, N), K,
+                                      _arg(C_inout, "C_inout", torch.float32, K * d),
+                                      _arg(counts_out, "counts_out", torch.int64, K),
+                                      _arg(n_reseeded_out, "n_reseeded_out", torch.int32, 1),
+                                      _arg(objective_out, "objective_out", torch.float64, 1), w, wb,
                                       _stream(stream)),
            "hme_update_centroids")
 
@@ -196,20 +241,32 @@ def hme_partition(labels: torch.Tensor, K: int, hist_out: torch.Tensor, offsets_
                   perm_out: torch.Tensor, ws: torch.Tensor, sorted_labels_out: Optional[torch.Tensor] = None,
                   tag_off: Optional[torch.Tensor] = None, tags: Optional[torch.Tensor] = None,
                   tag_off_out: Optional[torch.Tensor] = None, tags_out: Optional[torch.Tensor] = None, stream=None):
-    N = labels.shape[0]
+    N = _labels(labels)
+    lists = [t is None for t in (tag_off, tags, tag_off_out, tags_out)]
+    if any(lists) and not all(lists):
+        raise HmeError(HME_EINVAL, "argument check", "tag_off, tags, tag_off_out and tags_out: all four or none")
+    T = tags.numel() if tags is not None else 0
     w, wb = _ws(ws)
-    _check(lib().hme_partition(_ptr(labels), N, K, _ptr(hist_out), _ptr(offsets_out), _ptr(perm_out),
-                               _ptr(sorted_labels_out), _ptr(tag_off), _ptr(tags), _ptr(tag_off_out), _ptr(tags_out),
+    _check(lib().hme_partition(_arg(labels, "labels", torch.int32, N), N, K,
+                               _arg(hist_out, "hist_out", torch.int64, K),
+                               _arg(offsets_out, "offsets_out", torch.int64, K + 1),
+                               _arg(perm_out, "perm_out", torch.int32, N),
+                               _arg(sorted_labels_out, "sorted_labels_out", torch.int32, N),
+                               _arg(tag_off, "tag_off", torch.int64, N + 1), _arg(tags, "tags", torch.int32, 0),
+                               _arg(tag_off_out, "tag_off_out", torch.int64, N + 1),
+                               _arg(tags_out, "tags_out", torch.int32, T),
                                w, wb, _stream(stream)), "hme_partition")
 
 
 def hme_route(Q: torch.Tensor, C: torch.Tensor, expert_out: torch.Tensor, offsets_out: torch.Tensor,
               order_out: torch.Tensor, ws: torch.Tensor, flags: int = HME_ASSIGN_DEFAULT, stream=None):
     B, d, ldq, dt = _features(Q)
-    K = C.shape[0]
+    K = _centres(C, d)
     w, wb = _ws(ws)
-    _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _ptr(C), K, flags, _ptr(expert_out), _ptr(offsets_out),
-                           _ptr(order_out), w, wb, _stream(stream)), "hme_route")
+    _check(lib().hme_route(_ptr(Q), B, d, ldq, dt, _arg(C, "C", torch.float32, K * d), K, flags,
+                           _arg(expert_out, "expert_out", torch.int32, B),
+                           _arg(offsets_out, "offsets_out", torch.int64, K + 1),
+                           _arg(order_out, "order_out", torch.int32, B), w, wb, _stream(stream)), "hme_route")
 
 
 def hme_kmeans_stream(X: torch.Tensor, K: int, iters: int, chunk_rows: int, C_inout: torch.Tensor,
@@ -218,10 +275,16 @@ def hme_kmeans_stream(X: torch.Tensor, K: int, iters: int, chunk_rows: int, C_in
                       n_reseeded_out: Optional[torch.Tensor] = None, stream=None):
     """Lloyd's iterations on X in page-locked host memory (or device memory), streamed in chunks."""
     N, d, ldx, dt = _features(X)
+    if _centres(C_inout, d, "C_inout") != K:
+        raise HmeError(HME_EINVAL, "argument check", f"C_inout must have K = {K} rows")
     w, wb = _ws(ws)
-    _check(lib().hme_kmeans_stream(_ptr(X, host_ok=True), N, d, ldx, dt, K, iters, chunk_rows, _ptr(C_inout),
-                                   _ptr(labels_out),
-                                   _ptr(mind_out), _ptr(objectives_out), _ptr(counts_out), _ptr(n_reseeded_out), w,
+    _check(lib().hme_kmeans_stream(_ptr(X, host_ok=True), N, d, ldx, dt, K, iters, chunk_rows,
+                                   _arg(C_inout, "C_inout", torch.float32, K * d),
+                                   _arg(labels_out, "labels_out", torch.int32, N),
+                                   _arg(mind_out, "mind_out", torch.float32, N),
+                                   _arg(objectives_out, "objectives_out", torch.float64, max(iters, 0)),
+                                   _arg(counts_out, "counts_out", torch.int64, K),
+                                   _arg(n_reseeded_out, "n_reseeded_out", torch.int32, 1), w,
                                    wb, _stream(stream)), "hme_kmeans_stream")
 
 
@@ -229,20 +292,22 @@ def hme_tag_cluster_hist(offsets: torch.Tensor, tag_off: torch.Tensor, tags: tor
                          counts_out: torch.Tensor, ws: torch.Tensor, sparsity_out: Optional[torch.Tensor] = None,
                          stream=None):
     """Section 4.5 tag statistics from hme_partition's outputs: counts_out[K, V] int64, sparsity_out[V] fp64."""
-    N = tag_off.shape[0] - 1
+    N = _labels(tag_off, "tag_off") - 1
     w, wb = _ws(ws)
-    _check(lib().hme_tag_cluster_hist(_ptr(offsets), _ptr(tag_off), _ptr(tags), N, K, V, _ptr(counts_out),
-                                      _ptr(sparsity_out), w, wb, _stream(stream)), "hme_tag_cluster_hist")
+    _check(lib().hme_tag_cluster_hist(_arg(offsets, "offsets", torch.int64, K + 1),
+                                      _arg(tag_off, "tag_off", torch.int64, N + 1), _arg(tags, "tags", torch.int32, 0),
+                                      N, K, V, _arg(counts_out, "counts_out", torch.int64, K * V),
+                                      _arg(sparsity_out, "sparsity_out", torch.float64, V), w, wb, _stream(stream)),
+           "hme_tag_cluster_hist")
 
 
 def hme_pca_covariance(X: torch.Tensor, mean_out: torch.Tensor, cov_out: torch.Tensor, ws: torch.Tensor,
                        stream=None):
     """Section 4.2 PCA: column mean (fp64, d) and covariance (fp64, d x d) of fp32 features."""
     N, d, ldx, dt = _features(X)
-    if not (mean_out.is_contiguous() and cov_out.is_contiguous()):
-        raise ValueError("mean_out and cov_out must be contiguous")
     w, wb = _ws(ws)
-    _check(lib().hme_pca_covariance(_ptr(X), N, d, ldx, dt, _ptr(mean_out), _ptr(cov_out), w, wb, _stream(stream)),
+    _check(lib().hme_pca_covariance(_ptr(X), N, d, ldx, dt, _arg(mean_out, "mean_out", torch.float64, d),
+                                    _arg(cov_out, "cov_out", torch.float64, d * d), w, wb, _stream(stream)),
            "hme_pca_covariance")
 
 
@@ -251,11 +316,11 @@ def hme_pca_fit(X: torch.Tensor, r: int, mean_out: torch.Tensor, components_out:
     """Section 4.2 PCA: mean (fp32, d), r leading components (fp32, r x d) and their variances; returns the
     Jacobi sweeps made (the call synchronises the stream once per sweep)."""
     N, d, ldx, dt = _features(X)
-    if not (mean_out.is_contiguous() and components_out.is_contiguous()):
-        raise ValueError("mean_out and components_out must be contiguous")
     w, wb = _ws(ws)
     sweeps = ctypes.c_int32(0)
-    _check(lib().hme_pca_fit(_ptr(X), N, d, ldx, dt, r, _ptr(mean_out), _ptr(components_out), _ptr(variances_out),
+    _check(lib().hme_pca_fit(_ptr(X), N, d, ldx, dt, r, _arg(mean_out, "mean_out", torch.float32, d),
+                             _arg(components_out, "components_out", torch.float32, r * d),
+                             _arg(variances_out, "variances_out", torch.float32, r),
                              ctypes.byref(sweeps), w, wb, _stream(stream)), "hme_pca_fit")
     return int(sweeps.value)
 
@@ -264,13 +329,15 @@ def hme_pca_transform(X: torch.Tensor, mean: torch.Tensor, components: torch.Ten
                       ws: torch.Tensor, stream=None):
     """Z_out[i, j] = components[j] . (x_i - mean), fp32 (N x r)."""
     N, d, ldx, dt = _features(X)
-    r = components.shape[0]
+    r = _centres(components, d, "components")
     if Z_out.dim() != 2 or Z_out.stride(1) != 1:
         raise ValueError("Z_out must be a 2-D tensor with unit column stride")
-    if not (components.is_contiguous() and mean.is_contiguous()):
-        raise ValueError("components (r x d) and mean (d) must be contiguous")
+    if Z_out.dtype != torch.float32 or Z_out.shape[0] < N or Z_out.shape[1] < r:
+        raise HmeError(HME_EINVAL, "argument check",
+                       f"Z_out must be float32 with at least {N} x {r} elements, got {Z_out.dtype} {tuple(Z_out.shape)}")
     w, wb = _ws(ws)
-    _check(lib().hme_pca_transform(_ptr(X), N, d, ldx, dt, _ptr(mean), _ptr(components), r, _ptr(Z_out),
+    _check(lib().hme_pca_transform(_ptr(X), N, d, ldx, dt, _arg(mean, "mean", torch.float32, d),
+                                   _arg(components, "components", torch.float32, r * d), r, _ptr(Z_out),
                                    max(Z_out.stride(0), r), w, wb, _stream(stream)), "hme_pca_transform")
 
 
@@ -278,9 +345,13 @@ def hme_partition_noalloc(labels: torch.Tensor, K: int, hist_out: torch.Tensor, 
                           perm_out: torch.Tensor, sorted_labels_out: Optional[torch.Tensor] = None,
                           status_out: Optional[torch.Tensor] = None, stream=None):
     """hme_partition without a workspace (for callers that cannot allocate device memory)."""
-    N = labels.shape[0]
-    _check(lib().hme_partition_noalloc(_ptr(labels), N, K, _ptr(hist_out), _ptr(offsets_out), _ptr(perm_out),
-                                       _ptr(sorted_labels_out), _ptr(status_out), _stream(stream)),
+    N = _labels(labels)
+    _check(lib().hme_partition_noalloc(_arg(labels, "labels", torch.int32, N), N, K,
+                                       _arg(hist_out, "hist_out", torch.int64, K),
+                                       _arg(offsets_out, "offsets_out", torch.int64, K + 1),
+                                       _arg(perm_out, "perm_out", torch.int32, N),
+                                       _arg(sorted_labels_out, "sorted_labels_out", torch.int32, N),
+                                       _arg(status_out, "status_out", torch.int32, 1), _stream(stream)),
            "hme_partition_noalloc")
 
 

@@ -56,13 +56,24 @@ def distance_bound(Xd, Cd, labels, D, dtype):
     return b
 
 
+def rel_gap(d1, d2):
+    """The oracle's top-2 gap (D2 - D1) / D2 per row; +inf where there is no
+    runner-up (K = 1: D2 = inf), so such rows are never near ties."""
+    d1 = np.asarray(d1, np.float64)
+    d2 = np.asarray(d2, np.float64)
+    gap = np.full(d1.shape, np.inf)
+    fin = np.isfinite(d2)
+    gap[fin] = (d2[fin] - d1[fin]) / np.maximum(d2[fin], 1e-30)
+    return gap
+
+
 def check_assign(Xh, dtype, C, labels, mind=None, objective=None, ref=None):
     """Compare a GPU assignment with the oracle's on the same (X, C).  Returns stats."""
     lab_ref, d1, d2, J = ref if ref is not None else oracle.assign(Xh, C, dtype)
     labels = np.asarray(labels)
     N = labels.shape[0]
     assert labels.min(initial=0) >= 0 and labels.max(initial=0) < C.shape[0]
-    gap = (d2 - d1) / np.maximum(d2, 1e-30)
+    gap = rel_gap(d1, d2)
     bad = np.nonzero(labels != lab_ref)[0]
     assert np.all(gap[bad] < ASSIGN_GAP), (
         f"{bad.size} label mismatches, {(gap[bad] >= ASSIGN_GAP).sum()} outside near ties; "

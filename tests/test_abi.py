@@ -176,3 +176,86 @@ def test_binding_refuses_host_tensors_before_calling_the_library():
             call()
         assert ei.value.code == hme.HME_EINVAL
         assert "CUDA tensors" in str(ei.value)
+
+
+def test_binding_checks_array_types_and_sizes_before_calling_the_library(monkeypatch):
+    """Every array argument is checked for its element type, contiguity and
+    length before the C entry point is called: a wrong dtype or a short output
+    would otherwise let a kernel write past the tensor.  The device check is
+    stubbed out (no GPU here) and the library replaced by a recorder, which must
+    never be reached."""
+    import torch
+
+    from paper_1704_06363_gb300 import hme
+
+    calls = []
+
+    class Recorder:
+        def __getattr__(self, name):
+            def f(*a):
+                calls.append(name)
+                return hme.HME_OK
+            return f
+
+        def hme_last_error(self):
+            return b""
+
+    monkeypatch.setattr(hme, "lib", lambda: Recorder())
+    monkeypatch.setattr(hme, "_ptr", lambda t, host_ok=False: None if t is None else 16)
+    monkeypatch.setattr(hme, "_stream", lambda stream: None)
+
+    N, d, K = 8, 4, 3
+    X = torch.zeros(N, d)
+    C = torch.zeros(K, d)
+    ws = torch.zeros(256, dtype=torch.uint8)
+    i32, i64, f32, f64 = torch.int32, torch.int64, torch.float32, torch.float64
+
+    def z(n, dt):
+        return torch.zeros(n, dtype=dt)
+
+    good_part = dict(hist_out=z(K, i64), offsets_out=z(K + 1, i64), perm_out=z(N, i32))
+    bad = [
+        # hme_assign: labels int64, labels short, mind float64, C float64, C not contiguous
+        lambda: hme.hme_assign(X, C, z(N, i64), ws),
+        lambda: hme.hme_assign(X, C, z(N - 1, i32), ws),
+        lambda: hme.hme_assign(X, C, z(N, i32), ws, mind_out=z(N, f64)),
+        lambda: hme.hme_assign(X, C.double(), z(N, i32), ws),
+        lambda: hme.hme_assign(X, torch.zeros(d, K).t(), z(N, i32), ws),
+        lambda: hme.hme_assign(X, C, z(N, i32), ws, objective_out=z(1, f32)),
+        # hme_update_centroids: counts int32, counts short, prev_labels short
+        lambda: hme.hme_update_centroids(X, z(N, i32), None, C, ws, counts_out=z(K, i32)),
+        lambda: hme.hme_update_centroids(X, z(N, i32), None, C, ws, counts_out=z(K - 1, i64)),
+        lambda: hme.hme_update_centroids(X, z(N, i32), None, C, ws, prev_labels=z(N - 2, i32)),
+        lambda: hme.hme_update_centroids(X, z(N, i64), None, C, ws),
+        # hme_partition: hist int32, offsets of K entries, perm short, labels int64, sorted labels short
+        lambda: hme.hme_partition(z(N, i32), K, z(K, i32), z(K + 1, i64), z(N, i32), ws),
+        lambda: hme.hme_partition(z(N, i32), K, z(K, i64), z(K, i64), z(N, i32), ws),
+        lambda: hme.hme_partition(z(N, i32), K, z(K, i64), z(K + 1, i64), z(N - 1, i32), ws),
+        lambda: hme.hme_partition(z(N, i64), K, **good_part, ws=ws),
+        lambda: hme.hme_partition(z(N, i32), K, **good_part, ws=ws, sorted_labels_out=z(N - 1, i32)),
+        lambda: hme.hme_partition(z(N, i32), K, **good_part, ws=ws, tag_off=z(N + 1, i64), tags=z(20, i32),
+                                  tag_off_out=z(N + 1, i64), tags_out=z(19, i32)),
+        lambda: hme.hme_partition(z(N, i32), K, **good_part, ws=ws, tag_off=z(N + 1, i64), tags=z(20, i32)),
+        # hme_route: expert short, order int64
+        lambda: hme.hme_route(X, C, z(N - 1, i32), z(K + 1, i64), z(N, i32), ws),
+        lambda: hme.hme_route(X, C, z(N, i32), z(K + 1, i64), z(N, i64), ws),
+        # hme_partition_noalloc: hist short, perm int64
+        lambda: hme.hme_partition_noalloc(z(N, i32), K, z(K - 1, i64), z(K + 1, i64), z(N, i32)),
+        lambda: hme.hme_partition_noalloc(z(N, i32), K, z(K, i64), z(K + 1, i64), z(N, i64)),
+        # hme_tag_cluster_hist: counts short
+        lambda: hme.hme_tag_cluster_hist(z(K + 1, i64), z(N + 1, i64), z(10, i32), K, 5, z(K * 5 - 1, i64), ws),
+        # hme_kmeans_init: C_out with the wrong number of rows
+        lambda: hme.hme_kmeans_init(X, K + 1, 0, hme.HME_INIT_KMEANSPP, C, ws),
+        # hme_pca_covariance: cov short
+        lambda: hme.hme_pca_covariance(X, z(d, f64), torch.zeros(d, d - 1, dtype=f64), ws),
+    ]
+    for i, call in enumerate(bad):
+        with pytest.raises(hme.HmeError) as ei:
+            call()
+        assert ei.value.code == hme.HME_EINVAL, i
+    assert calls == []
+    # the same calls with well-formed arguments reach the library
+    hme.hme_assign(X, C, z(N, i32), ws, z(N, f32), z(1, f64))
+    hme.hme_partition(z(N, i32), K, **good_part, ws=ws, sorted_labels_out=z(N, i32))
+    hme.hme_partition_noalloc(z(N, i32), K, z(K, i64), z(K + 1, i64), z(N, i32))
+    assert calls == ["hme_assign", "hme_partition", "hme_partition_noalloc"]

@@ -102,6 +102,33 @@ def test_assign_parity(dev, N, d, K, dtype, ld):
     assert st["mismatches"] <= st["near_ties"]
 
 
+# One case per assign kernel variant with at least two row tiles for every
+# persistent CTA (one CTA per SM): rows = 2 x SMs x (rows per CTA tile) + 77,
+# so each CTA reuses its accumulators and the epilogue's exchange slots across
+# tiles, and the last tile is ragged.
+#   dtype, d, K, prepared, rows per CTA tile: kernel variant
+MULTI_TILE_CASES = [
+    ("f32", 256, 64, True, 128),     # three split products, one N-chunk
+    ("f32", 256, 64, False, 128),    # fp32 rows split inside the kernel
+    ("f32", 200, 600, True, 128),    # three split products, lean scan over three N-chunks
+    ("bf16", 256, 1024, True, 128),  # resident rows, four 256-centre N-chunks (the K = 4096, d = 256 kernel)
+    ("bf16", 512, 520, True, 256),   # two row tiles per centre stage, lean scan
+    ("bf16", 1024, 256, True, 256),  # two row tiles per centre stage, one 512-column accumulator (K = 256)
+]
+
+
+@pytest.mark.parametrize("dtype,d,K,prepared,bmt", MULTI_TILE_CASES, ids=lambda v: str(v))
+def test_assign_parity_several_tiles_per_cta(dev, dtype, d, K, prepared, bmt):
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    N = 2 * sms * bmt + 77
+    X = _mixture(N, d, min(K, 64), dtype, seed=N + d + K)
+    C = hme_synth.random_centroids(K, d, seed=K + d + 1, scale=3.0)
+    C[: K // 2] = X[: K // 2].float()
+    lab, md, obj = _assign(X, C, dev, prepared=prepared)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+
+
 @pytest.mark.parametrize("dtype,d,K", [("bf16", 256, 32), ("f32", 130, 300)])
 def test_assign_prepared_equals_unprepared(dev, dtype, d, K):
     """Where both calls run the same kernel (bf16 features; fp32 with several
@@ -128,7 +155,7 @@ def test_assign_split_in_kernel_and_prepared_agree(dev, N, d, K):
     sa = parity.check_assign(Xh, "f32", C.numpy(), a[0], a[1], a[2], ref=ref)
     sb = parity.check_assign(Xh, "f32", C.numpy(), b[0], b[1], b[2], ref=ref)
     assert sa["mismatches"] <= sa["near_ties"] and sb["mismatches"] <= sb["near_ties"]
-    gap = (ref[2] - ref[1]) / np.maximum(ref[2], 1e-30)
+    gap = parity.rel_gap(ref[1], ref[2])
     differ = np.nonzero(a[0] != b[0])[0]
     assert np.all(gap[differ] < parity.ASSIGN_GAP)
 
@@ -169,7 +196,7 @@ def test_assign_prepare_out_leaves_the_prepared_split(dev, N, d, K):
     for r in (a, b):
         st = parity.check_assign(Xh, "f32", C2.numpy(), r[0], r[1], r[2], ref=ref)
         assert st["mismatches"] <= st["near_ties"]
-    gap = (ref[2] - ref[1]) / np.maximum(ref[2], 1e-30)
+    gap = parity.rel_gap(ref[1], ref[2])
     assert np.all(gap[np.nonzero(a[0] != b[0])[0]] < parity.ASSIGN_GAP)
 
 

@@ -6,8 +6,10 @@
 - Workloads 2-5 on row subsamples of the same recipes (several tiles and a ragged
   tail): seeding, two teacher-forced iterations, the partition (workload 4 moves its
   tag lists) and the route of a fresh batch.
-- Workloads 2 and 5 at full size, in the launch configuration bench.py times: sampled
-  rows against the oracle, exact counts and partition, sampled cluster means.
+- Workloads 2-5 at full size, in the launch configuration bench.py times: sampled
+  rows against the oracle, exact counts and partition (workload 4 moves its tag
+  lists), sampled cluster means.  Workloads 3 and 4 are the two whose feature
+  matrices hold more than 2^31 elements.
 """
 import dataclasses
 
@@ -177,7 +179,7 @@ def _gather_rows(Xg, rows, dtype):
     return hme_synth.host_array(Xg.index_select(0, idx), dtype)
 
 
-@pytest.mark.parametrize("wid", [2, 5])
+@pytest.mark.parametrize("wid", [2, 3, 4, 5])
 def test_workload_full_size_sampled(dev, wid):
     w = hme_synth.WORKLOADS[wid]
     X, _ = hme_synth.make_features(w, device=dev)
@@ -189,21 +191,29 @@ def test_workload_full_size_sampled(dev, wid):
         L.assign(C)
         lab = L.labels.cpu().numpy()
         rows = np.sort(rng.choice(w.N, 2048, replace=False))
+        # the last rows of the matrix too: past 2^31 elements for workloads 3 and 4
+        rows = np.unique(np.concatenate([rows, np.arange(w.N - 5, w.N)]))
         Xs = _gather_rows(X, rows, w.dtype)
         st = parity.check_assign(Xs, w.dtype, C_t, lab[rows], L.mind.cpu().numpy()[rows])
         assert st["mismatches"] <= st["near_ties"]
         L.update(C)
         counts = L.counts.cpu().numpy()
         assert np.array_equal(counts, np.bincount(lab, minlength=w.K))
-        # sampled cluster means: the oracle on the gathered members of a few clusters
+        # sampled cluster means: the oracle on the gathered members of a few
+        # clusters (of at most 300,000 members, to bound the host copy)
         Cg = C.cpu().numpy()
-        nonempty = np.nonzero(counts)[0]
-        pick = rng.choice(nonempty, min(4, nonempty.size), replace=False)
+        eligible = np.nonzero((counts > 0) & (counts <= 300_000))[0]
+        pick = rng.choice(eligible, min(4, eligible.size), replace=False)
         for k in pick:
             members = np.nonzero(lab == k)[0]
             Xk = _gather_rows(X, members, w.dtype)
             Cref, _, _ = oracle.update(Xk, np.zeros(members.size, np.int32), None, C_t[k:k + 1], w.dtype)
             parity.check_centres(Cg[k:k + 1], Cref)
-    # the partition of the full label vector, bit-exact
-    got = _partition(L.labels, w.K, dev)
-    parity.check_partition(got, lab, w.K)
+    # the partition of the full label vector, bit-exact (workload 4 with its tag lists)
+    if w.tags:
+        tag_off, tags = hme_synth.make_tags(w, device=dev)
+        got = _partition(L.labels, w.K, dev, tag_off, tags)
+        parity.check_partition(got, lab, w.K, tag_off.cpu().numpy(), tags.cpu().numpy())
+    else:
+        got = _partition(L.labels, w.K, dev)
+        parity.check_partition(got, lab, w.K)
