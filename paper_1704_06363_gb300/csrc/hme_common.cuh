@@ -59,20 +59,16 @@ struct AssignGeom {
 AssignGeom assign_geom(int d, int K, int dtype);
 
 struct PartLayout {
-  int64_t tile;     // items per partition tile (one warp each)
+  int64_t tile;     // items per partition tile (one CTA each), a multiple of kPartChunk
   int64_t ntiles;
-  bool two_pass;    // K > kOnePassMaxK: two stable passes, low then high label bits
-  int bits1, bits2; // digit bits of the two passes (two_pass)
-  int bins;         // buckets of a pass: K, or 2^bits1 (>= 2^bits2) when two_pass
-  size_t tilecnt;   // int32[ntiles * bins]
+  int b0, b1;       // digit bits of the chunk sort's passes (b1 = 0: one pass)
+  size_t tilecnt;   // int32[ntiles * K]
   size_t hist;      // int64[K]
   size_t offs;      // int64[K + 1]
-  size_t dig;       // two_pass: int64[4 (bins + 1)]: the passes' bucket totals and offsets
-  size_t tmp;       // two_pass: int32[3 N]: order and labels after pass 1, sorted labels
   size_t misc;      // int64 scratch for scans (block sums), up to end
   size_t end;
 };
-constexpr int kOnePassMaxK = 256;
+constexpr int kPartChunk = 4096;  // items a partition CTA sorts in shared memory per step
 PartLayout part_layout(size_t base, int64_t N, int K);
 
 struct Layout {

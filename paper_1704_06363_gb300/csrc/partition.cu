@@ -2,103 +2,104 @@
 // trained "on its own share of the training data"; Section 2 also says no
 // attempt is made to balance the clusters, so buckets can be very unequal).
 //
-// A stable counting sort of the labels, integer-exact:
-//   1. count    each warp owns a contiguous tile of labels and counts it into
-//               private shared-memory bins (one shared atomic per label);
-//               tile counts go to an ntiles x bins int32 matrix.
+// A stable counting sort of the labels, integer-exact, in one pass over the
+// items for every K (up to 16384):
+//   1. count    the items are cut into ntiles contiguous tiles, one CTA each
+//               (two per SM); a CTA counts its tile into a shared-memory
+//               histogram of K bins and writes its row of the ntiles x K
+//               matrix of tile counts.
 //   2. colscan  exclusive prefix of that matrix down each column (per bucket)
-//               and the bucket totals.
-//   3. offsets  exclusive prefix of the totals.
-//   4. scatter  each warp walks its tile again in index order, kChunk labels
-//               at a time: every item gets its rank among the chunk's items of
-//               its bucket (one ballot per key bit finds the lanes of a round
-//               with the same key -- much cheaper than __match_any_sync here),
-//               the chunk is reordered by bucket in shared memory, and the
-//               items are stored in that order, so consecutive lanes write
-//               consecutive slots of a bucket.  An item's slot is offsets[k] +
-//               (items of bucket k in earlier tiles and chunks) + its rank, so
-//               within a bucket indices ascend.
-// With many buckets (K > kOnePassMaxK) a chunk holds too few items per bucket
-// for the stores to coalesce, so the sort runs as two stable passes of at
-// most 128 buckets, on the low and then the high label bits (a least-
-// significant-digit radix sort: the second pass keeps the first one's order
-// within a bucket, so the result is ordered by label and, within a label, by
-// index); offsets and hist then come from a binary search of the sorted labels.
-// Labels are staged kChunk at a time through a per-warp shared buffer with
-// 16-byte loads.  Labels outside [0, K) set kStatusBadLabel and are skipped.
+//               and the bucket totals (hist).
+//   3. offsets  exclusive prefix of hist.
+//   4. scatter  each CTA walks its tile in index order, kPChunk items at a
+//               time.  A chunk is sorted by label inside shared memory with a
+//               stable least-significant-digit radix sort of one or two
+//               passes (digits of at most 8 bits; each warp ranks its items
+//               with one ballot per digit bit, then one block-wide scan over
+//               (digit, warp) gives every item its place), so that items of a
+//               bucket become one run, in index order.  The CTA keeps one
+//               output cursor per bucket, offsets[k] + (items of bucket k in
+//               earlier tiles) + (items already placed by this tile); the run
+//               of bucket k is stored at cursor[k], cursor[k] + 1, ... by
+//               consecutive threads, so stores coalesce wherever a bucket has
+//               several items in a chunk, and each tile advances one write
+//               front per bucket: ntiles x K fronts, few enough for L2 to
+//               gather the partial sectors before they go to DRAM.
+// Within a bucket indices ascend (the tile order, then the chunk order, then
+// the stable sort), which is the definition of the stable partition.  Labels
+// outside [0, K) set kStatusBadLabel in the count pass and are sorted behind
+// every valid label by the scatter, which stores none of them.
 #include "hme_common.cuh"
 
 namespace hme {
 
 namespace {
 
-constexpr int kChunk = 512;        // labels staged per warp step
+constexpr int kPThreads = 512;                // threads of a count / scatter CTA
+constexpr int kPWarps = kPThreads / 32;
+constexpr int kPR = kPartChunk / kPThreads;   // items per thread per chunk
+constexpr int kMaxDigitBits = 8;
+constexpr int kPartTilesPerSM = 2;
+constexpr int kPartSMs = 152;                 // GB300: the tile count fills two CTAs per SM
+static_assert(kPartChunk % kPThreads == 0 && kPartChunk <= 65536, "chunk positions fit 16 bits");
 
-// Per-warp shared layout: [bins, padded to a multiple of 4][kChunk staged labels]
-// so that the staging buffer starts on a 16-byte boundary (int4 stores).
-__host__ __device__ __forceinline__ int bins_stride(int K) { return (K + 3) / 4 * 4; }
-__host__ __device__ __forceinline__ int count_words(int bins) { return bins_stride(bins) + kChunk; }
-__host__ __device__ __forceinline__ int scatter_words(int bins) { return 3 * bins_stride(bins) + 4 * kChunk; }
-constexpr int64_t kTargetTiles = 2432;
+__host__ __device__ __forceinline__ int round4(int k) { return (k + 3) / 4 * 4; }
 
-__device__ __forceinline__ void stage_labels(const int32_t *__restrict__ labels, int64_t pos, int64_t end,
-                                             int32_t *buf, int lane, bool aligned) {
-  if (aligned && pos + kChunk <= end) {
-    int4 v[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) v[u] = __ldg(reinterpret_cast<const int4 *>(labels + pos + 128 * u + 4 * lane));
-#pragma unroll
-    for (int u = 0; u < 4; ++u) *reinterpret_cast<int4 *>(buf + 128 * u + 4 * lane) = v[u];
-  } else {
-    for (int j = lane; j < kChunk; j += 32) buf[j] = (pos + j < end) ? __ldg(labels + pos + j) : -1;
-  }
-  __syncwarp();
+// Shared-memory words of the scatter CTA: cursors, two key buffers, the
+// per-warp digit counts (rows of 2^bmax + 1 words: the scan walks them
+// column-wise without bank conflicts) and the scan's warp totals.
+__host__ __device__ __forceinline__ size_t scatter_smem_words(int K, int bmax) {
+  return (size_t)round4(K) + 2 * (size_t)kPartChunk + (size_t)kPWarps * ((1 << bmax) + 1) + 32;
 }
 
-// Lanes of the warp whose key equals this lane's key (valid keys are in
-// [0, 2^nbits)); keys < 0 match no valid lane and get an empty mask.
-__device__ __forceinline__ unsigned same_key_lanes(int key, int nbits) {
-  unsigned peers = __ballot_sync(0xffffffffu, key >= 0);
-  for (int b = 0; b < nbits; ++b) {
-    const bool bit = (key >> b) & 1;
-    const unsigned m = __ballot_sync(0xffffffffu, bit);
-    peers &= bit ? m : ~m;
-  }
-  return key >= 0 ? peers : 0u;
-}
-
-// Items of a tile: [start, min(n, start + tile)) with n = min(N, *n_dev) (or
-// N).  The bucket of a valid label is (label >> shift) & mask.
-__global__ void part_count_kernel(const int32_t *__restrict__ labels, int64_t N, const int64_t *__restrict__ n_dev,
-                                  int K, int bins, int shift, int mask, bool check, int64_t tile, int64_t ntiles,
-                                  int32_t *__restrict__ tilecnt, Header *hdr, int wpb) {
-  extern __shared__ int32_t psm[];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * wpb + warp;
-  if (gw >= ntiles) return;
-  int32_t *cnt = psm + (size_t)warp * count_words(bins);
-  int32_t *buf = cnt + bins_stride(bins);
-  for (int k = lane; k < bins; k += 32) cnt[k] = 0;
-  __syncwarp();
-  const int64_t n = n_dev ? min(N, *n_dev) : N;
-  const int64_t start = gw * tile;
-  const int64_t end = min(n, start + tile);
-  const bool aligned = (reinterpret_cast<uintptr_t>(labels) & 15u) == 0;
+// Count each tile into a shared-memory histogram and write its row of tile counts.
+__global__ void __launch_bounds__(kPThreads) part_count_kernel(const int32_t *__restrict__ labels, int64_t N, int K,
+                                                               int64_t tile, int32_t *__restrict__ tilecnt,
+                                                               Header *hdr) {
+  extern __shared__ int32_t hcnt[];
+  for (int k = threadIdx.x; k < K; k += kPThreads) hcnt[k] = 0;
+  __syncthreads();
+  const int64_t start = (int64_t)blockIdx.x * tile;
+  const int64_t end = min(N, start + tile);
   bool bad = false;
-  for (int64_t pos = start; pos < end; pos += kChunk) {
-    stage_labels(labels, pos, end, buf, lane, aligned);
-    const int rounds = (int)min((int64_t)kChunk, end - pos + 31) / 32;
-    for (int r = 0; r < rounds; ++r) {
-      const int64_t i = pos + 32 * r + lane;
-      const int label = buf[32 * r + lane];
-      const bool valid = label >= 0 && label < K;
-      if (check && i < end && !valid) bad = true;
-      if (i < end && valid) atomicAdd(&cnt[(label >> shift) & mask], 1);
+  auto take = [&](int v) {
+    if (v >= 0 && v < K)
+      atomicAdd(&hcnt[v], 1);
+    else
+      bad = true;
+  };
+  // start is a multiple of kPartChunk, so an aligned base keeps every int4 aligned
+  if ((reinterpret_cast<uintptr_t>(labels) & 15u) == 0) {
+    const int64_t nvec = (end - start) / 4;
+    const int4 *v4 = reinterpret_cast<const int4 *>(labels + start);
+    int64_t j = threadIdx.x;
+    for (; j + 3 * kPThreads < nvec; j += 4 * kPThreads) {
+      int4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = __ldg(v4 + j + u * kPThreads);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        take(v[u].x);
+        take(v[u].y);
+        take(v[u].z);
+        take(v[u].w);
+      }
     }
-    __syncwarp();
+    for (; j < nvec; j += kPThreads) {
+      const int4 v = __ldg(v4 + j);
+      take(v.x);
+      take(v.y);
+      take(v.z);
+      take(v.w);
+    }
+    for (int64_t i = start + 4 * nvec + threadIdx.x; i < end; i += kPThreads) take(__ldg(labels + i));
+  } else {
+    for (int64_t i = start + threadIdx.x; i < end; i += kPThreads) take(__ldg(labels + i));
   }
   if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadLabel);
-  for (int k = lane; k < bins; k += 32) tilecnt[gw * bins + k] = cnt[k];
+  __syncthreads();
+  int32_t *row = tilecnt + (int64_t)blockIdx.x * K;
+  for (int k = threadIdx.x; k < K; k += kPThreads) row[k] = hcnt[k];
 }
 
 // Exclusive prefix down each column of the ntiles x K matrix; hist[k] = column total.
@@ -170,114 +171,165 @@ __global__ void __launch_bounds__(1024) part_offsets_kernel(const int64_t *__res
   if (t == 1023) offsets[K] = run;
 }
 
-// Stable scatter of a tile, kChunk items at a time, reordered by bucket in
-// shared memory before the stores: perm_out[slot] = payload ? payload[i] : i,
-// labels_out[slot] = label.  Per-warp shared layout: run, cnt, loff (bins
-// each, padded), staged labels, staged payload, reordered labels and payload.
-__global__ void part_scatter_kernel(const int32_t *__restrict__ labels, const int32_t *__restrict__ payload,
-                                    int64_t N, const int64_t *__restrict__ n_dev, int K, int bins, int shift,
-                                    int mask, int nbits, int64_t tile, int64_t ntiles,
-                                    const int32_t *__restrict__ tileoff, const int64_t *__restrict__ offsets,
-                                    int32_t *__restrict__ perm_out, int32_t *__restrict__ labels_out, int wpb) {
-  extern __shared__ int32_t psm[];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t gw = (int64_t)blockIdx.x * wpb + warp;
-  if (gw >= ntiles) return;
-  const int bs = bins_stride(bins);
-  int32_t *run = psm + (size_t)warp * scatter_words(bins);
-  int32_t *cnt = run + bs;
-  int32_t *loff = cnt + bs;
-  int32_t *buf = loff + bs;
-  int32_t *pbuf = buf + kChunk;
-  int32_t *olab = pbuf + kChunk;
-  int32_t *opay = olab + kChunk;
-  for (int k = lane; k < bins; k += 32) run[k] = (int32_t)(offsets[k] + tileoff[gw * bins + k]);
-  const int64_t n = n_dev ? min(N, *n_dev) : N;
-  const int64_t start = gw * tile;
-  const int64_t end = min(n, start + tile);
-  const bool aligned = (reinterpret_cast<uintptr_t>(labels) & 15u) == 0;
-  const bool paligned = payload && (reinterpret_cast<uintptr_t>(payload) & 15u) == 0;
-  const unsigned lt = (1u << lane) - 1u;
-  constexpr int R = kChunk / 32;
-  for (int64_t pos = start; pos < end; pos += kChunk) {
-    for (int k = lane; k < bins; k += 32) cnt[k] = 0;
-    stage_labels(labels, pos, end, buf, lane, aligned);
-    if (payload) stage_labels(payload, pos, end, pbuf, lane, paligned);
-    // rank of every item among the chunk's items of its bucket, in index order
-    int key[R], rk[R];
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int64_t i = pos + 32 * r + lane;
-      const int label = buf[32 * r + lane];
-      key[r] = (i < end && label >= 0 && label < K) ? (label >> shift) & mask : -1;
-      const unsigned peers = same_key_lanes(key[r], nbits);
-      rk[r] = key[r] >= 0 ? cnt[key[r]] + __popc(peers & lt) : 0;
-      __syncwarp();
-      if (key[r] >= 0 && lane == __ffs(peers) - 1) cnt[key[r]] += __popc(peers);
-      __syncwarp();
-    }
-    // loff = exclusive prefix of cnt over the buckets (each lane a run of them)
-    const int per = (bins + 31) / 32;
-    const int k0 = lane * per, k1 = min(bins, k0 + per);
-    int local = 0;
-    for (int k = k0; k < k1; ++k) local += cnt[k];
-    int incl = local;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    const int nvalid = __shfl_sync(0xffffffffu, incl, 31);
-    int acc = incl - local;
-    for (int k = k0; k < k1; ++k) {
-      loff[k] = acc;
-      acc += cnt[k];
-    }
-    __syncwarp();
-    // reorder the chunk by bucket
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      if (key[r] >= 0) {
-        const int at = loff[key[r]] + rk[r];
-        olab[at] = buf[32 * r + lane];
-        opay[at] = payload ? pbuf[32 * r + lane] : (int32_t)(pos + 32 * r + lane);
-      }
-    }
-    __syncwarp();
-    // consecutive lanes store consecutive slots of a bucket
-    for (int j = lane; j < nvalid; j += 32) {
-      const int label = olab[j];
-      const int k = (label >> shift) & mask;
-      const int32_t slot = run[k] + (j - loff[k]);
-      perm_out[slot] = opay[j];
-      if (labels_out) labels_out[slot] = label;
-    }
-    __syncwarp();
-    for (int k = lane; k < bins; k += 32) run[k] += cnt[k];
-    __syncwarp();
+// Lanes of the warp whose digit equals this lane's (digits in [0, 2^b)).
+__device__ __forceinline__ unsigned same_digit_lanes(unsigned dig, int b) {
+  unsigned peers = 0xffffffffu;
+  for (int i = 0; i < b; ++i) {
+    const unsigned bit = (dig >> i) & 1u;
+    const unsigned m = __ballot_sync(0xffffffffu, bit);
+    peers &= bit ? m : ~m;
   }
+  return peers;
 }
 
-// Two-pass partition: offsets[k] = first position of label k in the sorted
-// labels (binary search; offsets[K] = items), hist[k] = offsets[k+1] - offsets[k].
-__global__ void part_bounds_kernel(const int32_t *__restrict__ sorted, const int64_t *__restrict__ n_dev, int K,
-                                   int64_t *__restrict__ hist, int64_t *__restrict__ offsets) {
-  const int64_t n = *n_dev;
-  auto lower = [&](int k) -> int64_t {
-    int64_t lo = 0, hi = n;
-    while (lo < hi) {
-      const int64_t mid = (lo + hi) >> 1;
-      if (__ldg(sorted + mid) < k)
-        lo = mid + 1;
-      else
-        hi = mid;
+// One stable counting pass of the block-local radix sort.  Item r of this
+// thread sits at position warp * 32 kPR + 32 r + lane of the current order
+// and has packed value v[r] = key << 16 | (position in the chunk's index
+// order); its digit is (key >> shift) mod 2^b.  Every item is written to
+// out[its position in the order by (digit, current position)].
+__device__ __forceinline__ void rank_pass(const uint32_t (&v)[kPR], uint32_t *out, int shift, int b, int32_t *wcnt,
+                                          int32_t *wsum) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nd = 1 << b, stride = nd + 1;
+  int32_t *mine = wcnt + warp * stride;
+  for (int g = lane; g < nd; g += 32) mine[g] = 0;
+  __syncwarp();
+  const unsigned lt = (1u << lane) - 1u;
+  unsigned dig[kPR];
+  int rk[kPR];
+#pragma unroll
+  for (int r = 0; r < kPR; ++r) {
+    dig[r] = (v[r] >> (16 + shift)) & (unsigned)(nd - 1);
+    const unsigned peers = same_digit_lanes(dig[r], b);
+    const int before = mine[dig[r]];
+    rk[r] = before + __popc(peers & lt);
+    __syncwarp();
+    if (lane == __ffs(peers) - 1) mine[dig[r]] = before + __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+  // exclusive scan over the (digit, warp) counts, digit-major
+  const int n = nd * kPWarps;
+  const int per = (n + kPThreads - 1) / kPThreads;
+  const int e0 = threadIdx.x * per, e1 = min(n, e0 + per);
+  int local = 0;
+  for (int e = e0; e < e1; ++e) local += wcnt[(e % kPWarps) * stride + e / kPWarps];
+  int incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int w = lane < kPWarps ? wsum[lane] : 0;
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += t;
     }
-    return lo;
-  };
-  for (int k = blockIdx.x * blockDim.x + threadIdx.x; k <= K; k += gridDim.x * blockDim.x) {
-    const int64_t a = lower(k);
-    offsets[k] = a;
-    if (k < K) hist[k] = lower(k + 1) - a;
+    if (lane < kPWarps) wsum[lane] = wi - w;
+  }
+  __syncthreads();
+  int run = wsum[warp] + incl - local;
+  for (int e = e0; e < e1; ++e) {
+    int32_t *c = wcnt + (e % kPWarps) * stride + e / kPWarps;
+    const int t = *c;
+    *c = run;
+    run += t;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < kPR; ++r) out[mine[dig[r]] + rk[r]] = v[r];
+  __syncthreads();
+}
+
+// The stable scatter (see the file comment).  perm_out[slot] = item index,
+// labels_out[slot] = label (may be NULL).
+__global__ void __launch_bounds__(kPThreads, kPartTilesPerSM) part_scatter_kernel(const int32_t *__restrict__ labels, int64_t N, int K,
+                                                                 int b0, int b1, int64_t tile,
+                                                                 const int32_t *__restrict__ tileoff,
+                                                                 const int64_t *__restrict__ offsets,
+                                                                 int32_t *__restrict__ perm_out,
+                                                                 int32_t *__restrict__ labels_out) {
+  extern __shared__ uint32_t psm[];
+  int32_t *cursor = reinterpret_cast<int32_t *>(psm);
+  uint32_t *ka = psm + round4(K);
+  uint32_t *kb = ka + kPartChunk;
+  int32_t *wcnt = reinterpret_cast<int32_t *>(kb + kPartChunk);
+  const int bmax = b0 > b1 ? b0 : b1;
+  int32_t *wsum = wcnt + kPWarps * ((1 << bmax) + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t t = blockIdx.x;
+  for (int k = threadIdx.x; k < K; k += kPThreads) cursor[k] = (int32_t)(offsets[k] + tileoff[t * K + k]);
+  const int64_t start = t * tile;
+  const int64_t end = min(N, start + tile);
+  // item r of a thread: chunk position warp * 32 kPR + 32 r + lane (32 consecutive labels per warp load)
+  const int pbase = warp * 32 * kPR + lane;
+  int32_t lab[kPR];
+#pragma unroll
+  for (int r = 0; r < kPR; ++r) {
+    const int64_t i = start + pbase + 32 * r;
+    lab[r] = i < end ? __ldg(labels + i) : -1;
+  }
+  for (int64_t pos = start; pos < end; pos += kPartChunk) {
+    uint32_t v[kPR];
+#pragma unroll
+    for (int r = 0; r < kPR; ++r) {
+      const unsigned key = (lab[r] >= 0 && lab[r] < K) ? (unsigned)lab[r] : (unsigned)K;
+      v[r] = (key << 16) | (unsigned)(pbase + 32 * r);
+    }
+    // the next chunk's labels are in flight during the sort of this one
+    const int64_t nxt = pos + kPartChunk;
+#pragma unroll
+    for (int r = 0; r < kPR; ++r) {
+      const int64_t i = nxt + pbase + 32 * r;
+      lab[r] = i < end ? __ldg(labels + i) : -1;
+    }
+    rank_pass(v, kb, 0, b0, wcnt, wsum);
+    const uint32_t *sorted = kb;
+    if (b1 > 0) {
+      uint32_t w[kPR];
+#pragma unroll
+      for (int r = 0; r < kPR; ++r) w[r] = kb[pbase + 32 * r];
+      rank_pass(w, ka, b0, b1, wcnt, wsum);
+      sorted = ka;
+    }
+    // runs of equal keys: the first item of a run turns the bucket's cursor
+    // into its base (cursor - position), every item stores at base + position,
+    // the last item moves the cursor past the run
+    uint32_t sv[kPR];
+    bool last[kPR];
+#pragma unroll
+    for (int j = 0; j < kPR; ++j) {
+      const int q = threadIdx.x + kPThreads * j;
+      sv[j] = sorted[q];
+      const unsigned key = sv[j] >> 16;
+      const unsigned prev = q > 0 ? (sorted[q - 1] >> 16) : 0xFFFFFFFFu;
+      const unsigned next = q + 1 < kPartChunk ? (sorted[q + 1] >> 16) : 0xFFFFFFFFu;
+      last[j] = key != next;
+      if (key < (unsigned)K && key != prev) cursor[key] -= q;
+    }
+    __syncthreads();
+    int32_t slot[kPR];
+#pragma unroll
+    for (int j = 0; j < kPR; ++j) {
+      const int q = threadIdx.x + kPThreads * j;
+      const unsigned key = sv[j] >> 16;
+      slot[j] = -1;
+      if (key < (unsigned)K) {
+        slot[j] = cursor[key] + q;
+        perm_out[slot[j]] = (int32_t)(pos + (sv[j] & 0xFFFFu));
+        if (labels_out) labels_out[slot[j]] = (int32_t)key;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < kPR; ++j)
+      if (slot[j] >= 0 && last[j]) cursor[sv[j] >> 16] = slot[j] + 1;
+    // the next chunk's first rank pass synchronises before its key buffer is read here again
   }
 }
 
@@ -377,44 +429,26 @@ __global__ void tag_copy_kernel(const int32_t *__restrict__ perm, int64_t N,
   for (int64_t t = 0; t < len; ++t) tags_out[dst + t] = tags[src + t];
 }
 
-int warps_per_block(int words) {
-  const size_t per_warp = (size_t)words * sizeof(int32_t);
-  int w = (int)((96 * 1024) / per_warp);
-  if (w > 8) w = 8;
-  if (w < 1) w = 1;
-  return w;
-}
-
 }  // namespace
 
 PartLayout part_layout(size_t base, int64_t N, int K) {
   PartLayout pl;
-  int nbits = 0;
-  while ((1 << nbits) < K) ++nbits;
-  pl.two_pass = K > kOnePassMaxK;
-  pl.bits1 = pl.two_pass ? (nbits + 1) / 2 : nbits;
-  pl.bits2 = pl.two_pass ? nbits - pl.bits1 : 0;
-  pl.bins = pl.two_pass ? (1 << pl.bits1) : K;
-  int64_t tile = (N + kTargetTiles - 1) / kTargetTiles;
-  if (tile < 1024) tile = 1024;
-  if (tile < 4 * (int64_t)pl.bins) tile = 4 * (int64_t)pl.bins;
-  tile = (tile + kChunk - 1) / kChunk * kChunk;
+  int bits = 0;
+  while ((1 << bits) < K + 1) ++bits;  // labels 0 .. K-1 and the key K of an invalid label
+  pl.b0 = bits <= kMaxDigitBits ? bits : bits / 2;
+  pl.b1 = bits - pl.b0;
+  int64_t tile = (N + kPartTilesPerSM * kPartSMs - 1) / (kPartTilesPerSM * kPartSMs);
+  tile = (tile + kPartChunk - 1) / kPartChunk * kPartChunk;
+  if (tile < kPartChunk) tile = kPartChunk;
   pl.tile = tile;
   pl.ntiles = N > 0 ? (N + tile - 1) / tile : 0;
   size_t off = align_up(base, 256);
   pl.tilecnt = off;
-  off = align_up(off + (size_t)(pl.ntiles > 0 ? pl.ntiles : 1) * pl.bins * sizeof(int32_t), 256);
+  off = align_up(off + (size_t)(pl.ntiles > 0 ? pl.ntiles : 1) * K * sizeof(int32_t), 256);
   pl.hist = off;
   off = align_up(off + (size_t)K * sizeof(int64_t), 256);
   pl.offs = off;
   off = align_up(off + (size_t)(K + 1) * sizeof(int64_t), 256);
-  pl.dig = pl.tmp = 0;
-  if (pl.two_pass) {
-    pl.dig = off;
-    off = align_up(off + (size_t)4 * (pl.bins + 1) * sizeof(int64_t), 256);
-    pl.tmp = off;
-    off = align_up(off + (size_t)3 * (N > 0 ? N : 1) * sizeof(int32_t), 256);
-  }
   pl.misc = off;
   const int64_t nb = (N + kScanItems) / kScanItems + 1;
   off = align_up(off + (size_t)nb * sizeof(int64_t), 256);
@@ -422,16 +456,13 @@ PartLayout part_layout(size_t base, int64_t N, int K) {
   return pl;
 }
 
-namespace {
-
-// One stable counting-sort pass over the buckets (label >> shift) & mask.
-cudaError_t sort_pass(const int32_t *keys, const int32_t *payload, int64_t N, const int64_t *n_dev, int K, int bins,
-                      int shift, int mask, int nbits, bool check, const PartLayout &pl, int32_t *tilecnt,
-                      int64_t *hist, int64_t *offsets, int32_t *perm_out, int32_t *labels_out, Header *hdr,
-                      cudaStream_t s) {
-  const int wc = warps_per_block(count_words(bins)), ws = warps_per_block(scatter_words(bins));
-  const size_t smc = (size_t)wc * count_words(bins) * sizeof(int32_t);
-  const size_t sms = (size_t)ws * scatter_words(bins) * sizeof(int32_t);
+cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
+                             int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,
+                             cudaStream_t s) {
+  int32_t *tilecnt = reinterpret_cast<int32_t *>(ws + pl.tilecnt);
+  const size_t smc = (size_t)K * sizeof(int32_t);
+  const int bmax = pl.b0 > pl.b1 ? pl.b0 : pl.b1;
+  const size_t sms = scatter_smem_words(K, bmax) * sizeof(uint32_t);
   cudaError_t e;
   if (smc > 48 * 1024) {
     e = cudaFuncSetAttribute(part_count_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smc);
@@ -442,49 +473,17 @@ cudaError_t sort_pass(const int32_t *keys, const int32_t *payload, int64_t N, co
     if (e != cudaSuccess) return e;
   }
   if (pl.ntiles > 0) {
-    part_count_kernel<<<(unsigned)((pl.ntiles + wc - 1) / wc), 32 * wc, smc, s>>>(
-        keys, N, n_dev, K, bins, shift, mask, check, pl.tile, pl.ntiles, tilecnt, hdr, wc);
+    part_count_kernel<<<(unsigned)pl.ntiles, kPThreads, smc, s>>>(labels, N, K, pl.tile, tilecnt, hdr);
     count_launch();
   }
-  part_colscan_kernel<<<(bins + 31) / 32, 1024, 0, s>>>(tilecnt, pl.ntiles, bins, hist);
-  part_offsets_kernel<<<1, 1024, 0, s>>>(hist, bins, offsets);
+  part_colscan_kernel<<<(K + 31) / 32, 1024, 0, s>>>(tilecnt, pl.ntiles, K, hist);
+  part_offsets_kernel<<<1, 1024, 0, s>>>(hist, K, offsets);
   count_launch(2);
   if (pl.ntiles > 0) {
-    part_scatter_kernel<<<(unsigned)((pl.ntiles + ws - 1) / ws), 32 * ws, sms, s>>>(
-        keys, payload, N, n_dev, K, bins, shift, mask, nbits, pl.tile, pl.ntiles, tilecnt, offsets, perm_out,
-        labels_out, ws);
+    part_scatter_kernel<<<(unsigned)pl.ntiles, kPThreads, sms, s>>>(labels, N, K, pl.b0, pl.b1, pl.tile, tilecnt,
+                                                                    offsets, perm, sorted_labels);
     count_launch();
   }
-  return cudaGetLastError();
-}
-
-}  // namespace
-
-cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
-                             int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,
-                             cudaStream_t s) {
-  int32_t *tilecnt = reinterpret_cast<int32_t *>(ws + pl.tilecnt);
-  if (!pl.two_pass) {
-    int nbits = 0;
-    while ((1 << nbits) < K) ++nbits;
-    return sort_pass(labels, nullptr, N, nullptr, K, K, 0, 0x7FFFFFFF, nbits, true, pl, tilecnt, hist, offsets,
-                     perm, sorted_labels, hdr, s);
-  }
-  int64_t *dig = reinterpret_cast<int64_t *>(ws + pl.dig);
-  int64_t *hist1 = dig, *offs1 = dig + (pl.bins + 1), *hist2 = dig + 2 * (pl.bins + 1),
-          *offs2 = dig + 3 * (pl.bins + 1);
-  int32_t *tmp = reinterpret_cast<int32_t *>(ws + pl.tmp);
-  int32_t *order1 = tmp, *labels1 = tmp + N, *sorted = sorted_labels ? sorted_labels : tmp + 2 * N;
-  // pass 1: low bits of the input labels (checked); pass 2: high bits of pass 1's output
-  cudaError_t e = sort_pass(labels, nullptr, N, nullptr, K, pl.bins, 0, (1 << pl.bits1) - 1, pl.bits1, true, pl,
-                            tilecnt, hist1, offs1, order1, labels1, hdr, s);
-  if (e != cudaSuccess) return e;
-  const int bins2 = 1 << pl.bits2;
-  e = sort_pass(labels1, order1, N, offs1 + pl.bins, K, bins2, pl.bits1, bins2 - 1, pl.bits2, false, pl, tilecnt,
-                hist2, offs2, perm, sorted, hdr, s);
-  if (e != cudaSuccess) return e;
-  part_bounds_kernel<<<(K + 256) / 256, 256, 0, s>>>(sorted, offs1 + pl.bins, K, hist, offsets);
-  count_launch();
   return cudaGetLastError();
 }
 

@@ -14,7 +14,10 @@
 // - Set-up: the first call on each device, with that device current, looks up
 //   the array's device address with cudaGetSymbolAddress (host code cannot use
 //   the array's name as a device address).  Make that first call before any
-//   stream capture.
+//   stream capture.  The address belongs to the device's current CUDA context:
+//   it is kept together with that context and looked up again when the
+//   context changes (after cudaDeviceReset, for example), so a stale address
+//   is never passed to a kernel.
 // - Every call shares the array and it keeps the last call's contents: the
 //   status word is cleared at the start of each call; the tile counts are fully
 //   rewritten.  Calls that overlap on the GPU (different streams, or several
@@ -31,27 +34,52 @@ namespace hme {
 namespace {
 
 constexpr size_t kStaticScratchBytes = size_t(16) << 20;
-constexpr int64_t kStaticTileRound = 512;
 
 static __device__ __align__(256) unsigned char g_partition_scratch[kStaticScratchBytes];
 
-std::mutex g_scratch_mu;
-void *g_scratch_ptr[64] = {};
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
 
-// Device address of g_partition_scratch on the current device (set-up on first use).
+std::mutex g_scratch_mu;
+struct ScratchAddr {
+  CUcontext ctx;
+  void *ptr;
+};
+ScratchAddr g_scratch[64] = {};
+
+CtxGetCurrentFn ctx_get_current_fn() {
+  static CtxGetCurrentFn fn = [] {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      return reinterpret_cast<CtxGetCurrentFn>(f);
+    return static_cast<CtxGetCurrentFn>(nullptr);
+  }();
+  return fn;
+}
+
+// Device address of g_partition_scratch in the current device's context (set
+// up on the first call in that context).
 int static_scratch(void **out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(HME_EINTERNAL, "hme_partition_noalloc: device %d out of range", dev);
+  CtxGetCurrentFn get = ctx_get_current_fn();
+  if (!get) return fail(HME_ECUDA, "hme_partition_noalloc: cuCtxGetCurrent is not available from the driver");
+  CUcontext ctx = nullptr;
+  if (get(&ctx) != CUDA_SUCCESS) ctx = nullptr;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
+  if (!ctx || g_scratch[dev].ctx != ctx || !g_scratch[dev].ptr) {
+    // (the lookup also creates and binds the device's primary context when
+    // this thread has none yet)
     void *p = nullptr;
     e = cudaGetSymbolAddress(&p, g_partition_scratch);
     if (e != cudaSuccess) return cuda_fail(e, "hme_partition_noalloc: cudaGetSymbolAddress");
-    g_scratch_ptr[dev] = p;
+    if (get(&ctx) != CUDA_SUCCESS || !ctx) return fail(HME_ECUDA, "hme_partition_noalloc: no current CUDA context");
+    g_scratch[dev] = ScratchAddr{ctx, p};
   }
-  *out = g_scratch_ptr[dev];
+  *out = g_scratch[dev].ptr;
   return HME_OK;
 }
 
@@ -68,22 +96,15 @@ extern "C" int hme_partition_noalloc(const int32_t *labels, int64_t N, int32_t K
   if (!hist_out || !offsets_out) return fail(HME_EINVAL, "hist_out / offsets_out is NULL");
   if (N > 0 && (!labels || !perm_out)) return fail(HME_EINVAL, "labels / perm_out is NULL");
 
-  // One counting-sort pass (the two-pass form needs 12 bytes of scratch per
-  // label); tile counts go right after the 256-byte header; lengthen tiles
-  // until they fit.
+  // Tile counts go right after the 256-byte header; tiles lengthen (in whole
+  // sort chunks) until the ntiles x K counts fit.
   PartLayout pl = part_layout(sizeof(Header), N, K);
-  if (pl.two_pass) {
-    pl.two_pass = false;
-    pl.bins = K;
-    if (pl.tile < 4 * (int64_t)K) pl.tile = (4 * (int64_t)K + kStaticTileRound - 1) / kStaticTileRound * kStaticTileRound;
-    pl.ntiles = N > 0 ? (N + pl.tile - 1) / pl.tile : 0;
-  }
   const size_t room = kStaticScratchBytes - sizeof(Header);
   const int64_t max_tiles = (int64_t)(room / ((size_t)K * sizeof(int32_t)));
   if (max_tiles < 1) return fail(HME_EINVAL, "K = %d needs more than %zu bytes of static scratch", K, room);
   if (pl.ntiles > max_tiles) {
     int64_t tile = (N + max_tiles - 1) / max_tiles;
-    tile = (tile + kStaticTileRound - 1) / kStaticTileRound * kStaticTileRound;
+    tile = (tile + kPartChunk - 1) / kPartChunk * kPartChunk;
     pl.tile = tile;
     pl.ntiles = (N + tile - 1) / tile;
   }
