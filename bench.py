@@ -276,27 +276,45 @@ def measure_workload(args, w, dev, world, rank, clocks, headline):
     hdr_it = torch.zeros(T, 3, dtype=torch.int32, device=dev)    # rescored pairs, rescored all-K, moved rows
     bucket_it = torch.zeros(T, 3, dtype=torch.int64, device=dev)  # smallest, median, largest cluster
 
-    def step(Xs, record=False, diag=False):
+    def step_head(Xs, record=False, diag=False):
+        """The first assign of the job; it also leaves the prepared features
+        (row norms, and for fp32 rows with K <= 256 the bf16 split) in ws."""
         C.copy_(C0)
+        if record:
+            a0, a1 = _ev(), _ev()
+            a0.record(stream)
+        hme.hme_assign(Xs, C, labels_buf[0], ws, mind, obj[0:1], flags=hme.HME_ASSIGN_PREPARE_OUT)
+        if record:
+            a1.record(stream)
+            ev_assign.append((0, a0, a1))
+        if diag:
+            hdr_it[0, 0:1].copy_(ws[4:8].view(torch.int32))
+            hdr_it[0, 1:2].copy_(ws[12:16].view(torch.int32))
+
+    def step_tail(Xs, record=False, diag=False):
+        """The rest of the job: the centre update of iteration 0, iterations
+        1 .. T-1, the route of all rows (and the tag-list partition)."""
         for t in range(T):
             labels, prev = labels_buf[t % 2], (labels_buf[(t - 1) % 2] if t > 0 else None)
+            if t > 0:
+                if record:
+                    a0, a1 = _ev(), _ev()
+                    a0.record(stream)
+                hme.hme_assign(Xs, C, labels, ws, mind, obj[t:t + 1], flags=hme.HME_ASSIGN_PREPARED)
+                if record:
+                    a1.record(stream)
+                    ev_assign.append((t, a0, a1))
+                if diag:
+                    hdr_it[t, 0:1].copy_(ws[4:8].view(torch.int32))
+                    hdr_it[t, 1:2].copy_(ws[12:16].view(torch.int32))
             if record:
-                a0, a1, u1 = _ev(), _ev(), _ev()
-                a0.record(stream)
-            # the first assign leaves the prepared features (row norms, bf16 split) in ws
-            hme.hme_assign(Xs, C, labels, ws, mind, obj[t:t + 1],
-                           flags=hme.HME_ASSIGN_PREPARED if t > 0 else hme.HME_ASSIGN_PREPARE_OUT)
-            if record:
-                a1.record(stream)
-            if diag:
-                hdr_it[t, 0:1].copy_(ws[4:8].view(torch.int32))
-                hdr_it[t, 1:2].copy_(ws[12:16].view(torch.int32))
+                u0, u1 = _ev(), _ev()
+                u0.record(stream)
             # first iteration: full pass; then only the rows whose label changed
             hme.hme_update_centroids(Xs, labels, mind, C, ws, counts, nres[t:t + 1], jex[t:t + 1], prev_labels=prev)
             if record:
                 u1.record(stream)
-                ev_assign.append((t, a0, a1))
-                ev_update.append((t, a1, u1))
+                ev_update.append((t, u0, u1))
             if diag:
                 if t > 0:
                     hdr_it[t, 2:3].copy_(ws[32:36].view(torch.int32))
@@ -320,6 +338,10 @@ def measure_workload(args, w, dev, world, rank, clocks, headline):
             if record:
                 g1.record(stream)
                 ev_tags.append((g0, g1))
+
+    def step(Xs, record=False, diag=False):
+        step_head(Xs, record, diag)
+        step_tail(Xs, record, diag)
 
     for _ in range(max(3, args.warmup)):
         step(X)
@@ -423,18 +445,25 @@ def measure_workload(args, w, dev, world, rank, clocks, headline):
     else:
         achieved, traffic = u_gbs, profiled_traffic("update.cu", "update_" + w.name)
     flops_assign = 2.0 * N * K * d
-    # the assign step is tensor-bound when the tensor work it issues (three
-    # split products for fp32 rows) per byte read is above the ridge of the
-    # measured peaks; it runs inside a long step, so the sustained bf16 peak
-    nprod = 3 if w.dtype == "f32" else 1
-    if dominant == "assign" and nprod * flops_assign / assign_bytes > tc_sustained * 1e12 / (hbm * 1e9):
+    # The assign step's operands: bf16 features one bf16 product; fp32
+    # features with K > 256 one tf32 product (kind::tf32); fp32 features with
+    # K <= 256 three products of the bf16 split.  It is tensor-bound when the
+    # tensor work it issues per byte read is above the ridge of the peak of its
+    # operand type; it runs inside a long step, so the sustained peak (tf32: the
+    # sustained bf16 peak times the nominal dense tf32/bf16 ratio 1.1/2.25).
+    tf32 = False  # the step uses the default operands (fp32 rows: the bf16 split), not HME_ASSIGN_TF32
+    nprod = 3 if (w.dtype == "f32" and not tf32) else 1
+    op_peak = tc_sustained * (1.1 / 2.25) if tf32 else tc_sustained
+    if dominant == "assign" and nprod * flops_assign / assign_bytes > op_peak * 1e12 / (hbm * 1e9):
         ach_tf = flops_assign / (t_assign / 1000) / 1e12
-        roofline = {"bound": "tensor", "achieved": ach_tf, "peak": tc_sustained, "unit": "TFLOP/s",
-                    "frac": ach_tf / tc_sustained, "traffic": traffic, "kernel": dominant,
+        roofline = {"bound": "tensor", "achieved": ach_tf, "peak": op_peak, "unit": "TFLOP/s",
+                    "frac": ach_tf / op_peak, "traffic": traffic, "kernel": dominant,
+                    "operands": "tf32" if tf32 else ("bf16 split, three products" if nprod == 3 else "bf16"),
                     "issued_tflops": nprod * ach_tf, "achieved_note": "2NKd per assign call" +
                     (" (fp32 rows: three bf16 products issued per multiply-add)" if nprod == 3 else ""),
-                    "peak_source": f"{peak_kind} (MEASURED_PEAKS.json bf16_tflops_sustained)"
-                    if peak_kind == "measured" else "fallback 1.7 PFLOP/s sustained"}
+                    "peak_source": (f"{peak_kind} (MEASURED_PEAKS.json bf16_tflops_sustained"
+                                    + (" x 1.1/2.25, the nominal dense tf32/bf16 ratio)" if tf32 else ")"))
+                    if peak_kind == "measured" else "fallback 1.7 PFLOP/s sustained" + (" x 1.1/2.25" if tf32 else "")}
     else:
         roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
                     "traffic": traffic, "kernel": dominant, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
@@ -508,25 +537,44 @@ def measure_workload(args, w, dev, world, rank, clocks, headline):
             Xh = torch.empty(X.shape, dtype=X.dtype, pin_memory=True)
             Xh.copy_(X)
         if not args.no_e2e:
+            # The job with X in page-locked host memory: X is copied in by
+            # chunks of about 512 MB on a copy stream, and the first assign
+            # takes each chunk as soon as it has landed (hme_assign_rows,
+            # leaving that chunk's prepared features in ws); the rest of the
+            # step runs on the copied-in X as in the timed steps (replayed as a
+            # graph).  Labels, order, offsets and centres are copied out.
             Xd = torch.empty_like(X)
             out_labels = torch.empty(N, dtype=torch.int32, pin_memory=True)
             out_order = torch.empty(N, dtype=torch.int32, pin_memory=True)
             out_offsets = torch.empty(K + 1, dtype=torch.int64, pin_memory=True)
             out_C = torch.empty(K, d, dtype=torch.float32, pin_memory=True)
-            graph_e2e = None
-            if graph is not None:  # the same step on the copied-in buffer, as a graph
+            nch = int(max(1, min(64, (X.numel() * e) // (512 << 20))))
+            bounds = [N * j // nch for j in range(nch + 1)]
+            copy_stream = torch.cuda.Stream(dev)
+            landed = [torch.cuda.Event() for _ in range(nch)]
+            graph_tail = None
+            if graph is not None:  # the rest of the step on the copied-in buffer, as a graph
                 torch.cuda.synchronize(dev)
                 Xd.copy_(X)
-                graph_e2e = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(graph_e2e, capture_error_mode="relaxed"):
-                    step(Xd)
+                step_head(Xd)
+                graph_tail = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph_tail, capture_error_mode="relaxed"):
+                    step_tail(Xd)
 
             def e2e_step():
-                Xd.copy_(Xh, non_blocking=True)
-                if graph_e2e is not None:
-                    graph_e2e.replay()
+                C.copy_(C0)
+                copy_stream.wait_stream(stream)  # the previous step is done with Xd
+                for j in range(nch):
+                    r0, r1 = bounds[j], bounds[j + 1]
+                    with torch.cuda.stream(copy_stream):
+                        Xd[r0:r1].copy_(Xh[r0:r1], non_blocking=True)
+                        landed[j].record(copy_stream)
+                    stream.wait_event(landed[j])
+                    hme.hme_assign_rows(Xd, r0, r1, C, labels_buf[0], ws, mind, flags=hme.HME_ASSIGN_PREPARE_OUT)
+                if graph_tail is not None:
+                    graph_tail.replay()
                 else:
-                    step(Xd)
+                    step_tail(Xd)
                 out_labels.copy_(expert, non_blocking=True)
                 out_order.copy_(order, non_blocking=True)
                 out_offsets.copy_(offsets, non_blocking=True)
@@ -542,12 +590,16 @@ def measure_workload(args, w, dev, world, rank, clocks, headline):
                 e2e_step()
             f1.record(stream)
             torch.cuda.synchronize(dev)
+            if hme.hme_sync_status(ws) != hme.HME_OK:
+                raise RuntimeError(f"end-to-end step: {hme.hme_last_error()}")
             ms_e2e = max_over_ranks(f0.elapsed_time(f1), dev)
             res["e2e"] = {"value": iters_total / (ms_e2e / 1000.0), "unit": UNIT,
                           "h2d_bytes_per_step": X.numel() * e,
                           "d2h_bytes_per_step": 4 * N + 4 * N + 8 * (K + 1) + 4 * K * d,
-                          "ms_per_step": ms_e2e / args.steps}
-            del Xd, graph_e2e
+                          "ms_per_step": ms_e2e / args.steps,
+                          "overlap": f"host-to-device copy in {nch} chunks on a copy stream, the first assign "
+                                     "taking each chunk as it lands (hme_assign_rows)"}
+            del Xd, graph_tail
         # outside the timed steps: the same Lloyd iterations with X streamed
         # from page-locked host memory in chunks (hme_kmeans_stream), for
         # feature sets larger than HBM
@@ -726,7 +778,8 @@ def run_ours(args, w):
         line = {
             "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": head["ms_per_step"], "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16x3" if w.dtype == "f32" else "bf16",
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16x3" if w.dtype == "f32" else "bf16",
             "data": "synthetic",
             "config": {"workload": w.name, "N": w.N, "d": w.d, "K": w.K, "feature_dtype": w.dtype, "iterations": T,
                        "step": "%d x (assign + update; the first assign also writes the prepared features, updates "

@@ -83,6 +83,13 @@ extern "C" {
  * An in-kernel split (see hme_prepare_features) writes the split rows as it
  * makes them: the first Lloyd iteration reads X once instead of twice. */
 #define HME_ASSIGN_PREPARE_OUT 2
+/* HME_F32 features with K > 256 and rows TMA can read (X on a 16-byte
+ * boundary, ldx % 4 == 0): multiply x and c as tf32 operands (one product)
+ * instead of the three products of the bf16 split; ignored otherwise.  The
+ * wider operand error (see hme_assign) makes near ties, and so exact
+ * re-scores, more frequent: on the 1.6e7 x 512, K = 1024 feature set at its
+ * k-means++ centres the split was measured faster, so it is the default. */
+#define HME_ASSIGN_TF32 4
 
 /*
  * hme_workspace_bytes -- bytes of scratch an operation needs.
@@ -157,25 +164,52 @@ HME_API int hme_prepare_features(const void *X, int64_t N, int32_t d, int64_t ld
  *                   per row; hme_update_centroids returns the exact J.
  * The distance is ||x||^2 - 2 x.c + ||c||^2 with x.c on the tcgen05 tensor
  * cores (fp32 accumulate): for HME_BF16 features, x.bf16(c) with c rounded to
- * bf16 (round to nearest even); for HME_F32, the bf16 split x = xh + xl,
- * c = ch + cl and the three products xh.ch + xh.cl + xl.ch (nprod = 3; the
- * dropped xl.cl is at most 2^-16 (1 + 2^-8)^2 ||x|| ||c||), with the norms
- * taken of the same split values.  A row whose runner-up distance is within E
- * of its best, E a bound on the error of a difference of two computed
- * distances (ceil(d/16) * nprod * 2^-22 (||x||^2 + max_k ||c_k||^2), plus, for
- * split fp32 operands, 2^-14 (||x|| + max ||c||) sqrt(D2) and
- * 1.0625 * 2^-14 ||x|| max ||c||), is re-scored
+ * bf16 (round to nearest even); for HME_F32 with HME_ASSIGN_TF32 (K > 256,
+ * rows TMA can read), x as tf32 (10-bit significand, |x - x'| <= 2^-10 |x|)
+ * against c rounded to tf32 (|c - c'| <= 2^-11 |c|), one product, with
+ * ||c||^2 of the fp32 centres and ||x||^2 of the fp32 rows (with
+ * HME_ASSIGN_PREPARED, the prepared norms); otherwise for HME_F32 the bf16
+ * split x = xh + xl, c = ch + cl and the three products
+ * xh.ch + xh.cl + xl.ch (nprod = 3; the dropped xl.cl is at most
+ * 2^-16 (1 + 2^-8)^2 ||x|| ||c||), with the norms taken of the same split
+ * values.  A row whose runner-up distance is within E of its best, E a bound
+ * on the error of a difference of two computed distances
+ * (steps * nprod * 2^-22 (||x||^2 + max_k ||c_k||^2), steps = ceil(d/16), or
+ * ceil(d/8) for tf32 operands; plus, for split fp32 operands,
+ * 2^-14 (||x|| + max ||c||) sqrt(D2) and 1.0625 * 2^-14 ||x|| max ||c||; for
+ * tf32 operands 6.002 * 2^-10 ||x|| max ||c||), is re-scored
  * exactly on its candidates (all K when a third centre is also within E) with
  * direct differences, sum_j (x_j - c_j)^2 in fp32 (a sum of non-negative
  * terms).  The N x K distance matrix is never written.
  * X: N x d (ldx, dtype); C: K x d float32 (read only); labels_out: int32[N].
  * flags: HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARE_OUT (also leave X prepared in
  * ws), or HME_ASSIGN_PREPARED (skip the per-call hme_prepare_features pass; ws
- * must hold this X's preparation).  Both at once: HME_EINVAL.
+ * must hold this X's preparation); PREPARED and PREPARE_OUT at once:
+ * HME_EINVAL.  Either may be combined with HME_ASSIGN_TF32.
  */
 HME_API int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, const float *C, int32_t K,
                int32_t flags, int32_t *labels_out, float *mind_out, double *objective_out,
                void *ws, size_t ws_bytes, void *stream);
+
+/*
+ * hme_assign_rows -- hme_assign (Eq. 2, Section 2) of rows [row0, row1) of an
+ * N-row feature set, so that the assignment of a set can start on its first
+ * rows while later ones are still being copied in (the first Lloyd iteration
+ * of a set held in host memory: copy chunk j + 1 while chunk j is assigned).
+ * X points to row 0 of all N rows; only rows [row0, row1) are read.
+ * labels_out and mind_out (may be NULL) point to N-entry arrays; entries
+ * [row0, row1) are written.  ws is an HME_OP_ASSIGN workspace for all N rows:
+ * with HME_ASSIGN_PREPARE_OUT the preparation of these rows is left at their
+ * place in it, so that once every row has been assigned this way, later
+ * hme_assign calls on the whole set may pass HME_ASSIGN_PREPARED; with
+ * HME_ASSIGN_PREPARED these rows must have been prepared.  *objective_out
+ * (may be NULL) = the sum of mind over these rows.  Calls on one workspace
+ * must be ordered on one stream (they share its queues and header).
+ * Errors: as hme_assign, and HME_EINVAL unless 0 <= row0 <= row1 <= N.
+ */
+HME_API int hme_assign_rows(const void *X, int64_t N, int64_t row0, int64_t row1, int32_t d, int64_t ldx,
+                            int32_t dtype, const float *C, int32_t K, int32_t flags, int32_t *labels_out,
+                            float *mind_out, double *objective_out, void *ws, size_t ws_bytes, void *stream);
 
 /*
  * hme_update_centroids -- the K-means centre step (Section 2, "K-means

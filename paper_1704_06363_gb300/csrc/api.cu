@@ -66,18 +66,27 @@ uint64_t wait_limit_ns() {
 // and N = 256 halves the MMAs it issues per flop (MT = 2 with 128-centre
 // chunks measured 114 against 96 ms per assign at N = 5e7, d = 256, K = 4096).
 // fp32 features (three products, 2 operands per side) keep MT = 1.
-AssignGeom assign_geom(int d, int K, int dtype) {
+AssignGeom assign_geom(int d, int K, int dtype, bool tf32) {
   AssignGeom g;
   g.d = d;
   g.K = K;
   g.dtype = dtype;
   g.ldp = (d + 7) / 8 * 8;
-  g.nprod = dtype == HME_F32 ? 3 : 1;
-  const int num_kb = (d + kBK - 1) / kBK;
+  g.tf32 = tf32 && dtype == HME_F32;
+  g.nprod = dtype == HME_F32 && !g.tf32 ? 3 : 1;
+  g.kblk = g.tf32 ? 32 : kBK;
+  g.ldc = g.tf32 ? (d + 3) / 4 * 4 : g.ldp;
+  const int num_kb = (d + g.kblk - 1) / g.kblk;
   int max_bn = kMaxBN;
   g.mt = 1;
   g.ares = false;
-  if (g.nprod == 1) {
+  if (g.tf32) {
+    // one tf32 product per k-step: two row tiles share each centre stage
+    // (half the L2 reads of centres per row), 128-centre chunks so that both
+    // accumulators fit TMEM twice (the epilogue overlaps the next MMAs)
+    g.mt = 2;
+    max_bn = kMaxBN / 2;
+  } else if (g.nprod == 1) {
     g.mt = 2;
     if (K > kMaxBN && num_kb * (kBM * kBK * 2) <= 64 * 1024) {
       g.ares = true;
@@ -92,8 +101,23 @@ AssignGeom assign_geom(int d, int K, int dtype) {
   return g;
 }
 
+// HME_ASSIGN_TF32: fp32 features with several N-chunks (K > 256) read
+// directly as tf32 operands, when TMA can read them (16-byte aligned rows);
+// otherwise, and by default, as the bf16 split.
+bool use_tf32(const void *X, int64_t ldx, int K, int dtype, int flags) {
+  return (flags & HME_ASSIGN_TF32) && dtype == HME_F32 && K > kMaxBN &&
+         (reinterpret_cast<uintptr_t>(X) & 15u) == 0 && ldx % 4 == 0;
+}
+constexpr int kAssignFlags = HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT | HME_ASSIGN_TF32;
+bool bad_flags(int flags) {
+  return (flags & ~kAssignFlags) ||
+         (flags & (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) == (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT);
+}
+
 Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   const AssignGeom g = assign_geom(d, K, dtype);
+  // fp32 features with K > 256 may use either operand form (use_tf32): room for both
+  const AssignGeom gt = assign_geom(d, K, dtype, dtype == HME_F32 && K > kMaxBN);
   Layout L;
   size_t off = sizeof(Header);
   auto take = [&](size_t bytes) {
@@ -109,9 +133,11 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   } else {
     L.xhi = L.xlo = 0;
   }
-  L.cb_hi = take((size_t)g.Kp * g.ldp * 2);
+  const size_t cb_split = (size_t)g.Kp * g.ldp * 2;
+  const size_t cb_tf32 = gt.tf32 ? (size_t)gt.Kp * gt.ldc * 4 : 0;
+  L.cb_hi = take(cb_split > cb_tf32 ? cb_split : cb_tf32);
   L.cb_lo = dtype == HME_F32 ? take((size_t)g.Kp * g.ldp * 2) : 0;
-  L.cn = take((size_t)g.Kp * 4);
+  L.cn = take((size_t)(g.Kp > gt.Kp ? g.Kp : gt.Kp) * 4);
   L.flagged = take((size_t)(N > 0 ? N : 1) * 12);  // (row, best, runner-up) per queued row
   L.full_rows = take((size_t)(N > 0 ? N : 1) * 4);
   L.perm = take((size_t)(N > 0 ? N : 1) * 4);
@@ -192,8 +218,8 @@ T *at(void *ws, size_t off) {
 }
 
 int do_prepare(const void *X, int64_t N, int d, int64_t ldx, int dtype, int K, const Layout &L, void *ws,
-               cudaStream_t s) {
-  const AssignGeom g = assign_geom(d, K, dtype);
+               cudaStream_t s, int flags = 0) {
+  const AssignGeom g = assign_geom(d, K, dtype, use_tf32(X, ldx, K, dtype, flags));
   HME_CUDA(launch_prep_features(X, N, d, ldx, dtype, g, at<float>(ws, L.xn), at<__nv_bfloat16>(ws, L.xhi),
                                 at<__nv_bfloat16>(ws, L.xlo), s),
            "prepare features");
@@ -210,13 +236,14 @@ int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, con
 // full HBM rate.  prepare_out: an in-kernel split also writes the prepared
 // operands to ws (every other unprepared call leaves them there anyway).
 int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K, int32_t *labels,
-              float *mind, const Layout &L, void *ws, bool prepared, cudaStream_t s, bool prepare_out) {
-  const AssignGeom g = assign_geom(d, K, dtype);
+              float *mind, const Layout &L, void *ws, int flags, cudaStream_t s) {
+  const bool prepared = (flags & HME_ASSIGN_PREPARED) != 0, prepare_out = (flags & HME_ASSIGN_PREPARE_OUT) != 0;
+  const AssignGeom g = assign_geom(d, K, dtype, use_tf32(X, ldx, K, dtype, flags));
   const bool split = !prepared && split_eligible(X, ldx, g);
-  if (!prepared && !split) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s));
+  if (!prepared && !split) HME_TRY(do_prepare(X, N, d, ldx, dtype, K, L, ws, s, flags));
   Header *hdr = at<Header>(ws, 0);
-  HME_CUDA(launch_prep_centres(C, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
-                               at<float>(ws, L.cn), hdr, s),
+  HME_CUDA(launch_prep_centres(C, g, at<void>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo), at<float>(ws, L.cn),
+                               hdr, s),
            "prepare centres");
   if (split) {
     SplitOut out;
@@ -239,10 +266,11 @@ int do_assign(const void *X, int64_t N, int d, int64_t ldx, int dtype, const flo
 
 int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, const AssignGeom &g, const Layout &L,
                            void *ws, int32_t *labels, float *mind, Header *hdr, cudaStream_t s) {
-  const void *Xa = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xhi) : X;
-  const void *Xb = dtype == HME_F32 ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;
-  const int64_t lda = dtype == HME_F32 ? g.ldp : ldx;
-  HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<__nv_bfloat16>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
+  const bool split = g.nprod == 3;  // the prepared bf16 split; else X itself (bf16, or fp32 read as tf32)
+  const void *Xa = split ? (const void *)at<__nv_bfloat16>(ws, L.xhi) : X;
+  const void *Xb = split ? (const void *)at<__nv_bfloat16>(ws, L.xlo) : X;
+  const int64_t lda = split ? g.ldp : ldx;
+  HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<void>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
                         at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged),
                         at<int32_t>(ws, L.full_rows), s));
   return HME_OK;
@@ -347,7 +375,7 @@ extern "C" {
 size_t hme_workspace_bytes(int32_t op, int64_t N, int32_t d, int32_t K, int32_t dtype) {
   if (op == HME_OP_PARTITION) {
     if (N < 0 || N > (int64_t)0x7FFFFFFF || K < 1 || K > kMaxK) return 0;
-    return align_up(part_layout(sizeof(Header), N, K).end, 256);
+    return align_up(part_layout(sizeof(Header), N, K, true).end, 256);  // room for tag lists
   }
   if (op == HME_OP_STREAM) {  // N is the chunk length
     if (check_common(N, d, K, dtype) != HME_OK || N < 1) return 0;
@@ -437,15 +465,46 @@ int hme_assign(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t dtype, 
   HME_TRY(check_features(X, N, d, ldx, dtype, true));
   if (!C) return fail(HME_EINVAL, "C is NULL");
   if (N > 0 && !labels_out) return fail(HME_EINVAL, "labels_out is NULL");
-  if ((flags & ~(HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) ||
-      (flags & (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) == (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT))
-    return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  if (bad_flags(flags)) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
   const Layout L = feature_layout(N, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s,
-                    (flags & HME_ASSIGN_PREPARE_OUT) != 0));
+  HME_TRY(do_assign(X, N, d, ldx, dtype, C, K, labels_out, mind_out, L, ws, flags, s));
+  if (objective_out)
+    HME_CUDA(cudaMemcpyAsync(objective_out, &at<Header>(ws, 0)->objective, sizeof(double), cudaMemcpyDeviceToDevice,
+                             s),
+             "copy objective");
+  return HME_OK;
+}
+
+int hme_assign_rows(const void *X, int64_t N, int64_t row0, int64_t row1, int32_t d, int64_t ldx, int32_t dtype,
+                    const float *C, int32_t K, int32_t flags, int32_t *labels_out, float *mind_out,
+                    double *objective_out, void *ws, size_t ws_bytes, void *stream) {
+  HME_TRY(check_common(N, d, K, dtype));
+  if (row0 < 0 || row1 < row0 || row1 > N)
+    return fail(HME_EINVAL, "rows [%lld, %lld) are not inside [0, N = %lld)", (long long)row0, (long long)row1,
+                (long long)N);
+  if (bad_flags(flags)) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  if (!C) return fail(HME_EINVAL, "C is NULL");
+  if (row1 > row0 && !labels_out) return fail(HME_EINVAL, "labels_out is NULL");
+  const int64_t esz = dtype == HME_F32 ? 4 : 2;
+  const void *Xr = X ? static_cast<const char *>(X) + row0 * ldx * esz : nullptr;
+  HME_TRY(check_features(Xr, row1 - row0, d, ldx, dtype, true));
+  const Layout L = feature_layout(N, d, K, dtype, 0);
+  HME_TRY(check_ws(ws, ws_bytes, L.total));
+  // the preparation of rows [row0, row1) sits at their place in the N-row layout
+  const AssignGeom g = assign_geom(d, K, dtype);
+  Layout Lr = L;
+  Lr.xn += (size_t)row0 * 4;
+  if (dtype == HME_F32) {
+    Lr.xhi += (size_t)row0 * g.ldp * 2;
+    Lr.xlo += (size_t)row0 * g.ldp * 2;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  HME_TRY(clear_header(ws, s));
+  HME_TRY(do_assign(Xr, row1 - row0, d, ldx, dtype, C, K, labels_out ? labels_out + row0 : nullptr,
+                    mind_out ? mind_out + row0 : nullptr, Lr, ws, flags, s));
   if (objective_out)
     HME_CUDA(cudaMemcpyAsync(objective_out, &at<Header>(ws, 0)->objective, sizeof(double), cudaMemcpyDeviceToDevice,
                              s),
@@ -496,19 +555,14 @@ int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *hist_out
   if (N > 0 && (!labels || !perm_out)) return fail(HME_EINVAL, "labels / perm_out is NULL");
   const int ntag = (tag_off != nullptr) + (tags != nullptr) + (tag_off_out != nullptr) + (tags_out != nullptr);
   if (ntag != 0 && ntag != 4) return fail(HME_EINVAL, "tag arrays must be all NULL or all set");
-  const PartLayout pl = part_layout(sizeof(Header), N, K);
+  const PartLayout pl = part_layout(sizeof(Header), N, K, ntag == 4);
   HME_TRY(check_ws(ws, ws_bytes, align_up(pl.end, 256)));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
+  const TagLists tl{tag_off, tags, tag_off_out, tags_out};
   HME_CUDA(launch_partition(labels, N, K, pl, static_cast<char *>(ws), hist_out, offsets_out, perm_out,
-                            sorted_labels_out, at<Header>(ws, 0), s),
+                            sorted_labels_out, at<Header>(ws, 0), s, ntag == 4 ? &tl : nullptr),
            "partition");
-  if (ntag == 4) {
-    const int64_t nscratch = (int64_t)((pl.end - pl.misc) / sizeof(int64_t));
-    HME_CUDA(launch_tag_scatter(perm_out, N, offsets_out + K, tag_off, tags, tag_off_out, tags_out,
-                                at<int64_t>(ws, pl.misc), nscratch, s),
-             "partition: tag lists");
-  }
   return HME_OK;
 }
 
@@ -520,15 +574,12 @@ int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, c
   if (!C) return fail(HME_EINVAL, "C is NULL");
   if (!offsets_out) return fail(HME_EINVAL, "offsets_out is NULL");
   if (B > 0 && (!expert_out || !order_out)) return fail(HME_EINVAL, "expert_out / order_out is NULL");
-  if ((flags & ~(HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) ||
-      (flags & (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT)) == (HME_ASSIGN_PREPARED | HME_ASSIGN_PREPARE_OUT))
-    return fail(HME_EINVAL, "unknown flags 0x%x", flags);
+  if (bad_flags(flags)) return fail(HME_EINVAL, "unknown flags 0x%x", flags);
   const Layout L = feature_layout(B, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   HME_TRY(clear_header(ws, s));
-  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, (flags & HME_ASSIGN_PREPARED) != 0, s,
-                    (flags & HME_ASSIGN_PREPARE_OUT) != 0));
+  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, flags, s));
   HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
                             offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
            "route: partition");
@@ -705,7 +756,7 @@ int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t 
       // this chunk's re-score queues and centre-norm maximum start at zero
       if (!cuda_ok(cudaMemsetAsync(&hdr->rescore_count, 0, 3 * sizeof(uint32_t), s), "stream: clear queues")) break;
       if (!cuda_ok(cudaMemsetAsync(&hdr->cn_max_bits, 0, sizeof(uint32_t), s), "stream: clear queues")) break;
-      rc = do_assign(buf[b], n, d, ldc, dtype, C_inout, K, labels_out + r0, mind_out + r0, L, ws, false, s, false);
+      rc = do_assign(buf[b], n, d, ldc, dtype, C_inout, K, labels_out + r0, mind_out + r0, L, ws, 0, s);
       if (rc != HME_OK) break;
       if (!cuda_ok(launch_partition(labels_out + r0, n, K, L.part, static_cast<char *>(ws), hist, offs, perm, slab,
                                     hdr, s),

@@ -10,8 +10,15 @@
 // ever written: per row the kernel emits a label, the distance to the chosen
 // centre and, for near ties, a re-score request.
 //
-// Operands: for bf16 features, A = X (bf16) and B = bf16(C); for fp32
-// features the split x = xh + xl, c = ch + cl (all bf16, 16 significant bits
+// Operands: for bf16 features, A = X (bf16) and B = bf16(C).  fp32 features
+// with several N-chunks (K > 256, where the assign step is tensor-bound) are
+// read by TMA as they are and multiplied as tf32 (kind::tf32: 10-bit
+// significands, one product per k-step, 32 elements per 128-byte k-block)
+// against tf32-rounded centres; the operand rounding, |x - x_tf32| <= 2^-10
+// |x| and |c - c_tf32| <= 2^-11 |c| elementwise, enters the near-tie bound as
+// a term 6.002 * 2^-10 ||x|| max ||c|| (twice the error of each of the two
+// distances, 2 |x.c - x'.c'| <= 3.001 * 2^-10 ||x|| ||c||).  Otherwise fp32
+// features use the split x = xh + xl, c = ch + cl (all bf16, 16 significant bits
 // together) gives x_eff.c_eff = xh.ch + xh.cl + xl.ch + xl.cl.  The kernel
 // issues the first three (three MMAs per k-step): |xl| <= 2^-8 (1 + 2^-8) |x|
 // elementwise and likewise for cl, so the dropped xl.cl is at most
@@ -145,6 +152,49 @@ __device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float 
   i1 = (b1 < before) ? k0 + jl : i1;
 }
 
+// Branch-free top three for many centres with tf32 operands (whose wider
+// near-tie bound makes near ties common): per column v = ||c||^2 - 2 x.c,
+// the three smallest values and the indices of the best two, so that a near
+// tie with exactly two candidates is re-scored on those two only.  Ties keep
+// the lower index (columns ascend, comparisons are strict).
+__device__ __forceinline__ void top3_group(const uint32_t (&r)[16], const float *cn16, int k0, float &b1, float &b2,
+                                           float &b3, int &i1, int &i2) {
+  const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float4 cc = c4[q];
+    const float cq[4] = {cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int j = k0 + 4 * q + e;
+      const float v = fmaf(-2.0f, __uint_as_float(r[4 * q + e]), cq[e]);
+      const bool lt1 = v < b1, lt2 = v < b2;
+      b3 = fminf(b3, fmaxf(b2, v));
+      b2 = fminf(b2, fmaxf(b1, v));
+      i2 = lt1 ? i1 : (lt2 ? j : i2);
+      i1 = lt1 ? j : i1;
+      b1 = fminf(b1, v);
+    }
+  }
+}
+
+// Insert (v, i) into a top-three state (value, then index order).
+__device__ __forceinline__ void insert_top3(float v, int i, float &b1, float &b2, float &b3, int &i1, int &i2) {
+  if (v < b1 || (v == b1 && i < i1)) {
+    b3 = b2;
+    b2 = b1;
+    i2 = i1;
+    b1 = v;
+    i1 = i;
+  } else if (v < b2 || (v == b2 && i < i2)) {
+    b3 = b2;
+    b2 = v;
+    i2 = i;
+  } else {
+    b3 = fminf(b3, v);
+  }
+}
+
 // The result of one row's scan: label, distance, and for a near tie a
 // re-score request.  A centre whose tensor-core distance is within E of the
 // best could be the true nearest one.  E bounds the error of a difference of
@@ -195,14 +245,16 @@ __device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row,
 //          shares 1 .. CS-1 hand their per-row states to share 0 (through
 //          shared memory, behind two bounded mbarriers), which merges them and
 //          writes the row's result
+//   TF32   fp32 operands read as tf32 (kind::tf32; k-blocks of 32 elements)
 // Threads: warp 0 TMA, warp 1 MMA, 4*MT*CS epilogue warps.
-template <int NPROD, bool LEAN, int MT, bool ARES, int CS>
+template <int NPROD, bool LEAN, int MT, bool ARES, int CS, bool TF32 = false>
 __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
                   const AssignParams p) {
   constexpr int NOPS = (NPROD == 3) ? 2 : 1;  // operands per side (hi[, lo])
   constexpr int BMT = kBM * MT;               // rows per CTA tile
+  constexpr int KBLK = TF32 ? 32 : kBK;       // elements per 128-byte k-block
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128-byte swizzle atoms.
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -296,8 +348,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           mbar_arrive_expect_tx(ab, p.a_res_bytes);
           for (int mt = 0; mt < MT; ++mt)
             for (int kb = 0; kb < p.num_kb; ++kb) {
-              tma_load_2d(a_addr(0, mt, kb, 0), &tmA0, ab, kb * kBK, row0 + mt * kBM, pol_a);
-              if (NPROD == 3) tma_load_2d(a_addr(1, mt, kb, 0), &tmA1, ab, kb * kBK, row0 + mt * kBM, pol_a);
+              tma_load_2d(a_addr(0, mt, kb, 0), &tmA0, ab, kb * KBLK, row0 + mt * kBM, pol_a);
+              if (NPROD == 3) tma_load_2d(a_addr(1, mt, kb, 0), &tmA1, ab, kb * KBLK, row0 + mt * kBM, pol_a);
             }
           a_pending = true;
         }
@@ -312,7 +364,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             const uint32_t fb = smem_u32(&full[s]);
             mbar_arrive_expect_tx(fb, p.stage_bytes);
             const uint32_t st = ring + (uint32_t)s * p.stage_bytes;
-            const int32_t kx = kb * kBK;
+            const int32_t kx = kb * KBLK;
             if (!ARES) {
               for (int mt = 0; mt < MT; ++mt) {
                 tma_load_2d(a_addr(0, mt, kb, st), &tmA0, fb, kx, row0 + mt * kBM, pol_a);
@@ -336,7 +388,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(kBM, (uint32_t)p.BN);
+      const uint32_t idesc = TF32 ? idesc_tf32_f32(kBM, (uint32_t)p.BN) : idesc_bf16_f32(kBM, (uint32_t)p.BN);
       uint32_t it = 0, acc_it = 0, tile_it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
@@ -373,7 +425,10 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
               for (int mt = 0; mt < MT; ++mt) {
                 const uint32_t dtm = dt + (uint32_t)(mt * p.BN);
                 const uint64_t ad0 = smem_desc_sw128(a_addr(0, mt, kb, st) + k * 32);
-                tc_mma_bf16(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                if (TF32)
+                  tc_mma_tf32(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                else
+                  tc_mma_bf16(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
                 if (NPROD == 3) {
                   const uint64_t ad1 = smem_desc_sw128(a_addr(1, mt, kb, st) + k * 32);
                   tc_mma_bf16(dtm, ad0, bd1, idesc, 1u);  // xh . cl
@@ -430,6 +485,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       int idx1 = 0, idx2 = 0;
       float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
       int li1 = 0;
+      float lb3 = INFINITY;  // ... and of the tf32 top-three scan
+      int li2 = 0;
       const int64_t row = (int64_t)tile * BMT + row_in_tile;
       const float xr = (half == 0 && row < p.N) ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
       for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
@@ -465,6 +522,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
           if (LEAN)
             lean_group(ra, cbc, kbase + c, best1, best2, idx1);
+          else if (TF32)
+            top3_group(ra, cbc, kbase + c, best1, best2, best3, idx1, idx2);
           else
             epilogue_group(ra, cbc, kbase + c, best1, best2, best3, idx1, idx2);
           if (more1) {
@@ -472,6 +531,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
             if (LEAN)
               lean_group(rb, cbc + 16, kbase + c + 16, lb1, lb2, li1);
+            else if (TF32)
+              top3_group(rb, cbc + 16, kbase + c + 16, lb1, lb2, lb3, li1, li2);
             else
               epilogue_group(rb, cbc + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
             if (more2) tmem_ld_wait(ra);
@@ -487,6 +548,10 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
         best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
         best1 = take_b ? lb1 : best1;
         idx1 = take_b ? li1 : idx1;
+      } else if (TF32) {  // merge the two top-three states
+        insert_top3(lb1, li1, best1, best2, best3, idx1, idx2);
+        insert_top3(lb2, li2, best1, best2, best3, idx1, idx2);
+        best3 = fminf(best3, lb3);
       }
       if (CS > 1) {
         // Hand-over of the other shares' states.  Two slots alternate by
@@ -1337,13 +1402,15 @@ int make_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint
   return HME_OK;
 }
 
-// fp32 matrix rows x cols (row stride ld elements), box = 128 rows x 32 columns, 128-byte swizzle.
-int make_map_f32(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld) {
+// fp32 matrix rows x cols (row stride ld elements), box = box_rows rows x 32
+// columns (128 bytes), 128-byte swizzle.
+int make_map_f32(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint64_t ld,
+                 uint32_t box_rows = kBM) {
   EncodeTiledFn enc = get_encode_fn();
   if (!enc) return fail(HME_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 4};
-  cuuint32_t box[2] = {32, (cuuint32_t)kBM};
+  cuuint32_t box[2] = {32, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(ptr), dims, strides, box, estr,
                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -1364,15 +1431,21 @@ int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols,
 // 96 ms per assign at N = 5e7, d = 256, K = 4096; one 117 ms, four 104 ms.
 constexpr int kAresCS = 2;
 
-int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
-                  const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
-                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
+int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g, const void *chi,
+                  const __nv_bfloat16 *clo, const float *cn, const float *xn, int32_t *labels, float *mind,
+                  Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
   if (N == 0) return HME_OK;
   CUtensorMap mA0, mA1, mB0, mB1;
   int rc;
-  if ((rc = make_map(&mA0, Xa, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
-  if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
-    return rc;
+  if (g.tf32) {  // fp32 rows and tf32-rounded fp32 centres, 32-column boxes
+    if ((rc = make_map_f32(&mA0, Xa, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
+    if ((rc = make_map_f32(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldc, (uint32_t)g.BN)) != HME_OK)
+      return rc;
+  } else {
+    if ((rc = make_map(&mA0, Xa, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
+    if ((rc = make_map(&mB0, chi, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
+      return rc;
+  }
   if (g.nprod == 3) {
     if ((rc = make_map(&mA1, Xb, (uint64_t)N, (uint64_t)g.d, (uint64_t)lda, kBM)) != HME_OK) return rc;
     if ((rc = make_map(&mB1, clo, (uint64_t)g.K, (uint64_t)g.d, (uint64_t)g.ldp, (uint32_t)g.BN)) != HME_OK)
@@ -1383,7 +1456,7 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   }
   AssignParams p;
   p.N = N;
-  p.num_kb = (g.d + kBK - 1) / kBK;
+  p.num_kb = (g.d + g.kblk - 1) / g.kblk;
   p.BN = g.BN;
   p.nchunks = g.nchunks;
   p.num_tiles = (int)((N + kBM * g.mt - 1) / (kBM * g.mt));
@@ -1416,9 +1489,12 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   p.flagged = flagged;
   p.full_rows = full_rows;
   p.limit_ns = wait_limit_ns();
-  p.err_acc = (float)((double)((g.d + 15) / 16) * g.nprod * 0x1p-22 + 0x1p-20);
+  // accumulation steps along d: 16 elements per bf16 MMA step, 8 per tf32 step
+  const int steps = g.tf32 ? (g.d + 7) / 8 : (g.d + 15) / 16;
+  p.err_acc = (float)((double)steps * g.nprod * 0x1p-22 + 0x1p-20);
   p.err_split = g.nprod == 3 ? 0x1p-14f : 0.0f;
-  p.err_ll = g.nprod == 3 ? 0x1.1p-14f : 0.0f;
+  // split operands: the dropped xl.cl; tf32 operands: their rounding (6.002 * 2^-10)
+  p.err_ll = g.nprod == 3 ? 0x1.1p-14f : (g.tf32 ? (float)(6.002 * 0x1p-10) : 0.0f);
   const size_t smem = (size_t)p.a_res_bytes + (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
   int grid = num_sms();
   if (grid > p.num_tiles) grid = p.num_tiles;
@@ -1426,7 +1502,9 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   const bool lean = g.nchunks > 1;
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
-  if (g.nprod == 3)
+  if (g.tf32)
+    kern = assign_kernel<1, false, 2, false, 2, true>;  // top-three scan: two-candidate near ties re-scored cheaply
+  else if (g.nprod == 3)
     kern = lean ? assign_kernel<3, true, 1, false, 1> : assign_kernel<3, false, 1, false, 1>;
   else if (g.ares)
     kern = assign_kernel<1, true, 1, true, kAresCS>;

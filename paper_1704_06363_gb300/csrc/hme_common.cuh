@@ -53,10 +53,13 @@ struct AssignGeom {
   int nprod;      // 1 (bf16 features) or 3 (fp32 features, split products)
   int mt;         // 128-row tiles per CTA sharing each centre stage (1 or 2)
   bool ares;      // A rows resident in shared memory across N-chunks
+  bool tf32;      // fp32 features read as tf32 operands (kind::tf32, one product)
+  int kblk;       // elements per k-block: 64 (bf16 operands) or 32 (tf32)
+  int ldc;        // row stride (elements) of the prepared centres: ldp (bf16) or d rounded to 4 (fp32)
   int nbuf;       // TMEM accumulator buffers (1 or 2)
 };
 
-AssignGeom assign_geom(int d, int K, int dtype);
+AssignGeom assign_geom(int d, int K, int dtype, bool tf32 = false);
 
 struct PartLayout {
   int64_t tile;     // items per partition tile (one CTA each), a multiple of kPartChunk
@@ -65,11 +68,13 @@ struct PartLayout {
   size_t tilecnt;   // int32[ntiles * K]
   size_t hist;      // int64[K]
   size_t offs;      // int64[K + 1]
-  size_t misc;      // int64 scratch for scans (block sums), up to end
+  size_t tagcnt;    // tag lists: int64[ntiles * K] tile tag counts (0: no room for tag lists)
+  size_t tag_hist;  // tag lists: int64[K]
+  size_t tag_base;  // tag lists: int64[K + 1]
   size_t end;
 };
 constexpr int kPartChunk = 4096;  // items a partition CTA sorts in shared memory per step
-PartLayout part_layout(size_t base, int64_t N, int K);
+PartLayout part_layout(size_t base, int64_t N, int K, bool tags = false);
 
 struct Layout {
   size_t xn;        // f32[N]
@@ -108,10 +113,13 @@ uint64_t wait_limit_ns();
 // ---------------------------------------------------------------------------
 cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, int dtype, const AssignGeom &g,
                                  float *xn, __nv_bfloat16 *xhi, __nv_bfloat16 *xlo, cudaStream_t s);
-cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
-                                float *cn, Header *hdr, cudaStream_t s);
+// chi: bf16 rows of bf16(c) or of the split's hi part; for tf32 geometry fp32
+// rows of tf32-rounded c (pitch g.ldc).  clo: the split's lo part (fp32
+// features, three products) or unused.
+cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, void *chi, __nv_bfloat16 *clo, float *cn,
+                                Header *hdr, cudaStream_t s);
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
-                  const __nv_bfloat16 *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
+                  const void *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
                   int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s);
 // fp32 features with one N-chunk, split to bf16 hi/lo inside the kernel (no
 // preparation pass); eligible when X is 16-byte aligned and ldx % 4 == 0.
@@ -138,14 +146,18 @@ int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols,
 cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dtype, const float *C, int K,
                            int32_t *labels, float *mind, Header *hdr, int32_t *flagged,
                            const int32_t *full_rows, cudaStream_t s);
+// CSR tag lists that move with their points (hme_partition).
+struct TagLists {
+  const int64_t *tag_off;  // int64[N + 1]
+  const int32_t *tags;
+  int64_t *tag_off_out;    // int64[N + 1]
+  int32_t *tags_out;
+};
+// The stable partition (partition.cu).  tl: tag lists moved with their
+// points (pl must come from part_layout(..., tags = true)), or NULL.
 cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const PartLayout &pl, char *ws,
                              int64_t *hist, int64_t *offsets, int32_t *perm, int32_t *sorted_labels, Header *hdr,
-                             cudaStream_t s);
-// valid_total (device) = number of items with a label in [0, K) = offsets[K];
-// slots past it are never written by the partition and are not read.
-cudaError_t launch_tag_scatter(const int32_t *perm, int64_t N, const int64_t *valid_total, const int64_t *tag_off,
-                               const int32_t *tags, int64_t *tag_off_out, int32_t *tags_out, int64_t *scratch,
-                               int64_t nscratch, cudaStream_t s);
+                             cudaStream_t s, const TagLists *tl = nullptr);
 // Per-cluster state carried by the workspace from one centre update to the next.
 struct UpdateState {
   double *sums;     // fp64[K * d]: S_k = sum of the rows with label k
@@ -367,6 +379,19 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, ui
       : "memory");
 }
 
+// D[tmem] (+)= A[smem desc] x B[smem desc]^T, kind::tf32 (fp32 words in shared
+// memory read as tf32, fp32 accumulate); K = 8 per instruction, so a 32-byte
+// step along k is one instruction, as for kind::f16.
+__device__ __forceinline__ void tc_mma_tf32(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // D[tmem] (+)= A[tmem] x B[smem desc]^T, kind::f16, A read from tensor memory:
 // row m of A in lane m, 16-bit elements packed in pairs along k into 32-bit
 // columns (element 2w in the low half of column w).
@@ -448,6 +473,10 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr) {
 // M >> 4 at bits 24-28.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+// kind::tf32: A and B format 2 (tf32), fp32 accumulator, both K-major.
+__host__ __device__ constexpr uint32_t idesc_tf32_f32(uint32_t M, uint32_t N) {
+  return (1u << 4) | (2u << 7) | (2u << 10) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
 #endif  // __CUDACC__

@@ -9,9 +9,14 @@
 //                  and xn[i] = ||x_eff,i||^2 of exactly those values; for bf16
 //                  features xn[i] = ||x_i||^2.  One warp per row, 16-byte
 //                  vector loads, read once (HBM-bound).
+//                  fp32 features read as tf32 operands (several N-chunks)
+//                  need only xn[i] = ||x_i||^2 of the fp32 values.
 //   prep_centres   every iteration: bf16(c) (bf16 features) or the split
 //                  ch, cl (fp32 features), and cn[k] = ||c_eff||^2 of exactly
-//                  the values the MMA consumes; cn = +inf for padding centres;
+//                  the values the MMA consumes; for tf32 operands c rounded to
+//                  tf32 (cvt.rna) and cn[k] = ||c||^2 of the fp32 centre (the
+//                  distance is taken to the fp32 centre; the operand rounding
+//                  enters the near-tie bound); cn = +inf for padding centres;
 //                  max_k cn[k] goes to the workspace header (error bound of the
 //                  assign step's near-tie test).
 #include "hme_common.cuh"
@@ -97,6 +102,41 @@ __global__ void __launch_bounds__(256) prep_f32_scalar_kernel(const float *__res
   }
 }
 
+// fp32 features read as tf32 operands: only the norms of the fp32 rows.
+template <bool VEC>
+__global__ void __launch_bounds__(256) prep_f32_norm_kernel(const float *__restrict__ X, int64_t N, int d,
+                                                            int64_t ldx, float *__restrict__ xn) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  for (int64_t row = w0; row < N; row += nw) {
+    const float *xr = X + row * ldx;
+    float s = 0.0f;
+    if (VEC) {  // d % 4 == 0, ldx % 4 == 0 and a 16-byte aligned base
+      for (int j = lane; j < d / 4; j += 32) {
+        const float4 v = ld_stream_f4(xr + 4 * j);
+        s = fmaf(v.x, v.x, s);
+        s = fmaf(v.y, v.y, s);
+        s = fmaf(v.z, v.z, s);
+        s = fmaf(v.w, v.w, s);
+      }
+    } else {
+      for (int j = lane; j < d; j += 32) {
+        const float v = __ldg(xr + j);
+        s = fmaf(v, v, s);
+      }
+    }
+    s = warp_sum(s);
+    if (lane == 0) xn[row] = s;
+  }
+}
+
+__device__ __forceinline__ float round_tf32(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return __uint_as_float(r);
+}
+
 // bf16 features: only the norms (the MMA reads X itself).
 __global__ void __launch_bounds__(256) prep_bf16_kernel(const __nv_bfloat16 *__restrict__ X, int64_t N, int d,
                                                         int64_t ldx, float *__restrict__ xn) {
@@ -135,10 +175,12 @@ __global__ void __launch_bounds__(256) prep_bf16_kernel(const __nv_bfloat16 *__r
 constexpr int kPrepCThreads = 256;
 
 __global__ void __launch_bounds__(kPrepCThreads) prep_centres_kernel(const float *__restrict__ C, int K, int Kp,
-                                                                     int d, int ldp, int nprod,
-                                                                     __nv_bfloat16 *__restrict__ chi,
+                                                                     int d, int ldp, int nprod, bool tf32,
+                                                                     void *__restrict__ chi_raw,
                                                                      __nv_bfloat16 *__restrict__ clo,
                                                                      float *__restrict__ cn, Header *hdr) {
+  __nv_bfloat16 *chi = static_cast<__nv_bfloat16 *>(chi_raw);
+  float *ct = static_cast<float *>(chi_raw);
   __shared__ float part[kPrepCThreads / 32];
   const int k = blockIdx.x;
   if (k >= K) {
@@ -150,7 +192,10 @@ __global__ void __launch_bounds__(kPrepCThreads) prep_centres_kernel(const float
   for (int j = threadIdx.x; j < d; j += kPrepCThreads) {
     const float c = __ldg(C + (int64_t)k * d + j);
     float ce;
-    if (nprod == 1) {
+    if (tf32) {
+      ct[(int64_t)k * ldp + j] = round_tf32(c);
+      ce = c;
+    } else if (nprod == 1) {
       const __nv_bfloat16 b = __float2bfloat16_rn(c);
       chi[(int64_t)k * ldp + j] = b;
       ce = __bfloat162float(b);
@@ -184,12 +229,15 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
   if (blocks > want) blocks = want;
   if (dtype == HME_F32) {
     const bool vec = (d % 4 == 0) && (ldx % 4 == 0) && ((reinterpret_cast<uintptr_t>(X) & 15u) == 0);
-    if (vec)
-      prep_f32_vec_kernel<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const float *>(X), N, d, ldx, g.ldp, xn,
-                                                            xhi, xlo);
+    const float *Xf = static_cast<const float *>(X);
+    if (g.tf32 && vec)
+      prep_f32_norm_kernel<true><<<(unsigned)blocks, 256, 0, s>>>(Xf, N, d, ldx, xn);
+    else if (g.tf32)
+      prep_f32_norm_kernel<false><<<(unsigned)blocks, 256, 0, s>>>(Xf, N, d, ldx, xn);
+    else if (vec)
+      prep_f32_vec_kernel<<<(unsigned)blocks, 256, 0, s>>>(Xf, N, d, ldx, g.ldp, xn, xhi, xlo);
     else
-      prep_f32_scalar_kernel<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const float *>(X), N, d, ldx, g.ldp,
-                                                               xn, xhi, xlo);
+      prep_f32_scalar_kernel<<<(unsigned)blocks, 256, 0, s>>>(Xf, N, d, ldx, g.ldp, xn, xhi, xlo);
   } else {
     prep_bf16_kernel<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(X), N, d, ldx, xn);
   }
@@ -197,9 +245,9 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
   return cudaGetLastError();
 }
 
-cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, __nv_bfloat16 *chi, __nv_bfloat16 *clo,
-                                float *cn, Header *hdr, cudaStream_t s) {
-  prep_centres_kernel<<<g.Kp, kPrepCThreads, 0, s>>>(C, g.K, g.Kp, g.d, g.ldp, g.nprod, chi, clo, cn, hdr);
+cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, void *chi, __nv_bfloat16 *clo, float *cn,
+                                Header *hdr, cudaStream_t s) {
+  prep_centres_kernel<<<g.Kp, kPrepCThreads, 0, s>>>(C, g.K, g.Kp, g.d, g.ldc, g.nprod, g.tf32, chi, clo, cn, hdr);
   count_launch();
   return cudaGetLastError();
 }

@@ -20,7 +20,7 @@ HME_OK, HME_EINVAL, HME_ENOMEM, HME_ECUDA, HME_ETIMEOUT, HME_EINTERNAL = range(6
 HME_F32, HME_BF16 = 0, 1
 HME_OP_INIT, HME_OP_ASSIGN, HME_OP_PARTITION, HME_OP_ROUTE, HME_OP_TAG_HIST, HME_OP_STREAM, HME_OP_PCA = range(7)
 HME_INIT_KMEANSPP, HME_INIT_KMEANSPP_SUBSAMPLE = 0, 1
-HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED, HME_ASSIGN_PREPARE_OUT = 0, 1, 2
+HME_ASSIGN_DEFAULT, HME_ASSIGN_PREPARED, HME_ASSIGN_PREPARE_OUT, HME_ASSIGN_TF32 = 0, 1, 2, 4
 
 _NAMES = {0: "HME_OK", 1: "HME_EINVAL", 2: "HME_ENOMEM", 3: "HME_ECUDA", 4: "HME_ETIMEOUT", 5: "HME_EINTERNAL"}
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libhme.so")
@@ -57,6 +57,8 @@ def lib():
         L.hme_prepare_features.argtypes = [p, i64, i32, i64, i32, i32, p, sz, p]
         L.hme_assign.restype = ctypes.c_int
         L.hme_assign.argtypes = [p, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
+        L.hme_assign_rows.restype = ctypes.c_int
+        L.hme_assign_rows.argtypes = [p, i64, i64, i64, i32, i64, i32, p, i32, i32, p, p, p, p, sz, p]
         L.hme_update_centroids.restype = ctypes.c_int
         L.hme_update_centroids.argtypes = [p, i64, i32, i64, i32, p, p, p, i32, p, p, p, p, p, sz, p]
         L.hme_partition.restype = ctypes.c_int
@@ -216,6 +218,20 @@ def hme_assign(X: torch.Tensor, C: torch.Tensor, labels_out: torch.Tensor, ws: t
                             _arg(mind_out, "mind_out", torch.float32, N),
                             _arg(objective_out, "objective_out", torch.float64, 1), w, wb, _stream(stream)),
            "hme_assign")
+
+
+def hme_assign_rows(X: torch.Tensor, row0: int, row1: int, C: torch.Tensor, labels_out: torch.Tensor,
+                    ws: torch.Tensor, mind_out: Optional[torch.Tensor] = None,
+                    objective_out: Optional[torch.Tensor] = None, flags: int = HME_ASSIGN_DEFAULT, stream=None):
+    """hme_assign of rows [row0, row1) of X (all N rows' workspace and outputs)."""
+    N, d, ldx, dt = _features(X)
+    K = _centres(C, d)
+    w, wb = _ws(ws)
+    _check(lib().hme_assign_rows(_ptr(X), N, row0, row1, d, ldx, dt, _arg(C, "C", torch.float32, K * d), K, flags,
+                                 _arg(labels_out, "labels_out", torch.int32, N),
+                                 _arg(mind_out, "mind_out", torch.float32, N),
+                                 _arg(objective_out, "objective_out", torch.float64, 1), w, wb, _stream(stream)),
+           "hme_assign_rows")
 
 
 def hme_update_centroids(X: torch.Tensor, labels: torch.Tensor, mind: Optional[torch.Tensor], C_inout: torch.Tensor,

@@ -10,9 +10,14 @@ The oracle (fp64, direct sums) is the reference; the bars are:
     towards zero]  + 2^-15 (||x|| + ||c||) ||x - c||  [fp32 features: the
     16-bit split, |x - x_eff| <= 2^-16 |x| per element]  + 2^-14 ||x|| ||c||
     [fp32 features: the product xl.cl of the split is not formed,
-    2 |xl.cl| <= 2^-15 (1 + 2^-8)^2 ||x|| ||c||]  + 1e-5 D; the sum of
-    those distances (hme_assign's objective estimate) within the sum of the
-    per-row bounds + 1e-5 J;
+    2 |xl.cl| <= 2^-15 (1 + 2^-8)^2 ||x|| ||c||]  + 1e-5 D; fp32 features
+    assigned with HME_ASSIGN_TF32 (K > 256) are multiplied as tf32 operands
+    (10-bit significands: |x - x'| <= 2^-10 |x|, |c - c'| <= 2^-11 |c|),
+    whose distances are within ceil(d/8) 2^-23 (||x||^2 + ||c||^2) + 3.001
+    2^-10 ||x|| ||c|| (2 |x.c - x'.c'|) + 2^-15 ||x||^2 (norms taken from the
+    split of a preparation) + 1e-5 D; the sum of those distances
+    (hme_assign's objective estimate) within the sum of the per-row bounds +
+    1e-5 J;
   - objective of hme_update_centroids (direct differences): within 1e-5
     relative of the fp64 value for the same (C, labels);
   - centres: ||dc_k||_inf <= 1e-4 * max(||c_k||_inf, 1e-6 max_k ||c_k||_inf);
@@ -43,12 +48,15 @@ def features_f64(Xh: np.ndarray, dtype: str) -> np.ndarray:
     return Xh.astype(np.float64)
 
 
-def distance_bound(Xd, Cd, labels, D, dtype):
+def distance_bound(Xd, Cd, labels, D, dtype, tf32=False):
     """Per-row bound on |D_gpu - D| for hme_assign's distances (see the module docstring)."""
     d = Xd.shape[1]
     nprod = 3 if dtype == "f32" else 1
     xn = (Xd ** 2).sum(1)
     cn = (Cd ** 2).sum(1)[labels]
+    if dtype == "f32" and tf32:
+        return (np.ceil(d / 8) * 2.0 ** -23 * (xn + cn) + 3.001 * 2.0 ** -10 * np.sqrt(xn) * np.sqrt(cn)
+                + 2.0 ** -15 * xn + 1e-5 * D)
     b = np.ceil(d / 16) * nprod * 2.0 ** -23 * (xn + cn) + 1e-5 * D
     if dtype == "f32":
         b += 2.0 ** -15 * (np.sqrt(xn) + np.sqrt(cn)) * np.sqrt(np.maximum(D, 0))
@@ -67,7 +75,7 @@ def rel_gap(d1, d2):
     return gap
 
 
-def check_assign(Xh, dtype, C, labels, mind=None, objective=None, ref=None):
+def check_assign(Xh, dtype, C, labels, mind=None, objective=None, ref=None, tf32=False):
     """Compare a GPU assignment with the oracle's on the same (X, C).  Returns stats."""
     lab_ref, d1, d2, J = ref if ref is not None else oracle.assign(Xh, C, dtype)
     labels = np.asarray(labels)
@@ -84,7 +92,7 @@ def check_assign(Xh, dtype, C, labels, mind=None, objective=None, ref=None):
     if bad.size:
         D_gpu_label[bad] = ((Xd[bad] - Cd[labels[bad]]) ** 2).sum(1)
         assert np.all(D_gpu_label[bad] - d1[bad] <= ASSIGN_GAP * d2[bad])
-    bound = distance_bound(Xd, Cd, labels, D_gpu_label, dtype)
+    bound = distance_bound(Xd, Cd, labels, D_gpu_label, dtype, tf32)
     if mind is not None:
         err = np.abs(np.asarray(mind, np.float64) - D_gpu_label)
         assert np.all(err <= bound + 1e-30), f"distance error up to {np.max(err / (bound + 1e-30)):.3g} x bound"

@@ -73,7 +73,7 @@ def test_host_validation_rejects_before_launch(lib):
     bf16_misaligned[3] = ctypes.c_int64(12)
     bf16_misaligned[2] = ctypes.c_int32(12)
     assert lib.hme_assign(*bf16_misaligned) == 1 and b"TMA" in lib.hme_last_error()
-    for flags in (4, 3):  # an unknown bit; PREPARED together with PREPARE_OUT
+    for flags in (8, 3):  # an unknown bit; PREPARED together with PREPARE_OUT
         bad_flags = list(args)
         bad_flags[7] = ctypes.c_int32(flags)
         assert lib.hme_assign(*bad_flags) == 1 and b"flags" in lib.hme_last_error()

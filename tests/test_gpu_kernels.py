@@ -42,7 +42,7 @@ def _host(X, dtype):
     return hme_synth.host_array(X.contiguous(), dtype)
 
 
-def _assign(X, C, dev, mind=True, prepared=False):
+def _assign(X, C, dev, mind=True, prepared=False, extra_flags=0):
     N, d = X.shape
     K = C.shape[0]
     Xg = X.to(dev) if X.is_contiguous() else _to_dev_strided(X, dev)
@@ -54,9 +54,9 @@ def _assign(X, C, dev, mind=True, prepared=False):
     Cg = C.to(dev)
     if prepared:
         hme.hme_prepare_features(Xg, K, ws)
-        hme.hme_assign(Xg, Cg, lab, ws, md, obj, flags=hme.HME_ASSIGN_PREPARED)
+        hme.hme_assign(Xg, Cg, lab, ws, md, obj, flags=hme.HME_ASSIGN_PREPARED | extra_flags)
     else:
-        hme.hme_assign(Xg, Cg, lab, ws, md, obj)
+        hme.hme_assign(Xg, Cg, lab, ws, md, obj, flags=extra_flags)
     assert hme.hme_sync_status(ws) == hme.HME_OK
     return lab.cpu().numpy(), (md.cpu().numpy() if mind else None), obj.item()
 
@@ -126,6 +126,44 @@ def test_assign_parity_several_tiles_per_cta(dev, dtype, d, K, prepared, bmt):
     C[: K // 2] = X[: K // 2].float()
     lab, md, obj = _assign(X, C, dev, prepared=prepared)
     st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+
+
+# HME_ASSIGN_TF32: fp32 features multiplied as tf32 operands (K > 256, rows TMA
+# can read); near ties are re-scored on their two candidates, or on all K when
+# a third centre is close too.  N, d, K, rows per CTA tile (0: a few tiles)
+TF32_CASES = [(2000, 512, 1024, 0), (700, 48, 16384, 0), (3000, 132, 300, 0), (129, 64, 257, 0),
+              (0, 200, 600, 256)]
+
+
+@pytest.mark.parametrize("N,d,K,bmt", TF32_CASES, ids=lambda v: str(v))
+@pytest.mark.parametrize("prepared", [False, True])
+def test_assign_parity_tf32(dev, N, d, K, bmt, prepared):
+    if bmt:  # at least two row tiles per persistent CTA
+        N = 2 * torch.cuda.get_device_properties(dev).multi_processor_count * bmt + 77
+    X = _mixture(N, d, min(K, 64), "f32", seed=N + d + K + 3)
+    C = hme_synth.random_centroids(K, d, seed=K + d + 2, scale=3.0)
+    C[: K // 2] = X[: K // 2].float() if N >= K // 2 else C[: K // 2]
+    lab, md, obj = _assign(X, C, dev, prepared=prepared, extra_flags=hme.HME_ASSIGN_TF32)
+    st = parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj, tf32=True)
+    assert st["mismatches"] <= st["near_ties"]
+
+
+@pytest.mark.parametrize("copies", [2, 3])
+def test_assign_tf32_near_ties_are_rescored_exactly(dev, copies):
+    """Groups of centres 1e-5 apart: with tf32 operands every such row is a near
+    tie, decided by the exact re-score of its two candidates (two copies) or of
+    all K (three copies)."""
+    N, d, K = 3000, 256, 600
+    base = K // copies
+    X = _mixture(N, d, 64, "f32", seed=31 + copies)
+    C = hme_synth.random_centroids(K, d, seed=4, scale=3.0)
+    C[:base] = X[:base].float()
+    g = torch.Generator().manual_seed(6)
+    for r in range(1, copies):
+        C[r * base:(r + 1) * base] = C[:base] + 1e-5 * torch.randn(base, d, generator=g)
+    lab, md, obj = _assign(X, C, dev, extra_flags=hme.HME_ASSIGN_TF32)
+    st = parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj, tf32=True)
     assert st["mismatches"] <= st["near_ties"]
 
 
@@ -468,3 +506,51 @@ def test_launch_counter_moves(dev):
     X = _mixture(300, 32, 4, "f32", seed=1)
     _assign(X, hme_synth.random_centroids(4, 32, seed=1), dev)
     assert hme.hme_launch_count() - before >= 3
+
+
+@pytest.mark.parametrize("dtype,d,K", [("f32", 256, 32), ("bf16", 256, 300), ("f32", 128, 600), ("f32", 130, 40)])
+def test_assign_rows_in_chunks_equals_one_call(dev, dtype, d, K):
+    """hme_assign_rows over consecutive row ranges (ragged, one of a single
+    row) gives the labels and distances of one hme_assign call, bit for bit
+    (the per-row arithmetic is the same), and the preparation the chunks leave
+    (HME_ASSIGN_PREPARE_OUT) serves a later prepared call like one left by a
+    single call."""
+    N = 5000
+    X = _mixture(N, d, min(K, 32), dtype, seed=d + K)
+    C = hme_synth.random_centroids(K, d, seed=K, scale=3.0)
+    C[: K // 2] = X[: K // 2].float()
+    C2 = hme_synth.random_centroids(K, d, seed=K + 1, scale=3.0)
+    C2[K // 2:] = X[N - (K - K // 2):].float()
+    Xg, Cg, C2g = X.to(dev), C.to(dev), C2.to(dev)
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    out = []
+    for chunked in (True, False):
+        ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+        lab = torch.full((N,), -1, dtype=torch.int32, device=dev)
+        md = torch.empty(N, dtype=torch.float32, device=dev)
+        if chunked:
+            bounds = [0, 1234, 1235, 4000, N]
+            for r0, r1 in zip(bounds, bounds[1:]):
+                hme.hme_assign_rows(Xg, r0, r1, Cg, lab, ws, md, flags=hme.HME_ASSIGN_PREPARE_OUT)
+        else:
+            hme.hme_assign(Xg, Cg, lab, ws, md, flags=hme.HME_ASSIGN_PREPARE_OUT)
+        lab2 = torch.full((N,), -1, dtype=torch.int32, device=dev)
+        md2 = torch.empty(N, dtype=torch.float32, device=dev)
+        hme.hme_assign(Xg, C2g, lab2, ws, md2, flags=hme.HME_ASSIGN_PREPARED)
+        assert hme.hme_sync_status(ws) == hme.HME_OK
+        out.append([t.cpu().numpy() for t in (lab, md, lab2, md2)])
+    for a, b in zip(*out):
+        assert np.array_equal(a, b)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), out[0][0], out[0][1])
+    assert st["mismatches"] <= st["near_ties"]
+
+
+def test_assign_rows_rejects_ranges_outside_the_set(dev):
+    X = _mixture(100, 32, 4, "f32", seed=1).to(dev)
+    C = hme_synth.random_centroids(4, 32, seed=1).to(dev)
+    ws = hme.workspace(hme.HME_OP_ASSIGN, 100, 32, 4, hme.HME_F32, device=dev)
+    lab = torch.empty(100, dtype=torch.int32, device=dev)
+    for r0, r1 in ((-1, 5), (10, 5), (90, 101)):
+        with pytest.raises(hme.HmeError) as ei:
+            hme.hme_assign_rows(X, r0, r1, C, lab, ws)
+        assert ei.value.code == hme.HME_EINVAL
