@@ -64,7 +64,7 @@ AssignGeom assign_geom(int d, int K, int dtype, bool tf32 = false);
 struct PartLayout {
   int64_t tile;     // items per partition tile (one CTA each), a multiple of kPartChunk
   int64_t ntiles;
-  int b0, b1;       // digit bits of the chunk sort's passes (b1 = 0: one pass)
+  int b0, b1, b2;   // digit bits of the chunk sort's passes (0: no such pass)
   size_t tilecnt;   // int32[ntiles * K]
   size_t hist;      // int64[K]
   size_t offs;      // int64[K + 1]

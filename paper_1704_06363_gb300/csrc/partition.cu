@@ -12,12 +12,13 @@
 //   2. colscan  exclusive prefix of that matrix down each column (per bucket)
 //               and the bucket totals (hist).
 //   3. offsets  exclusive prefix of hist.
-//   4. scatter  each CTA walks its tile in index order, kPChunk items at a
-//               time.  A chunk is sorted by label inside shared memory with a
-//               stable least-significant-digit radix sort of one or two
-//               passes (digits of at most 8 bits; each warp ranks its items
-//               with one ballot per digit bit, then one block-wide scan over
-//               (digit, warp) gives every item its place), so that items of a
+//   4. scatter  each CTA walks its tile in index order, kPartChunk items at
+//               a time.  A chunk is sorted by label inside shared memory with
+//               a stable least-significant-digit radix sort of one or two
+//               passes (digits of at most 7 bits, 8 for the last pass of
+//               15-bit keys; every thread counts its 16 consecutive items per
+//               digit in private 16-bit counters and one block-wide scan of
+//               the counters gives every item its place), so that items of a
 //               bucket become one run, in index order.  The CTA keeps one
 //               output cursor per bucket, offsets[k] + (items of bucket k in
 //               earlier tiles) + (items already placed by this tile); the run
@@ -35,41 +36,66 @@
 // every valid label by the scatter, which stores none of them.
 #include "hme_common.cuh"
 
+#include <algorithm>
+
+#ifndef HME_PART_MAXB
+#define HME_PART_MAXB 5
+#endif
+
 namespace hme {
 
 namespace {
 
-constexpr int kPThreads = 512;                // threads of a count / scatter CTA
-constexpr int kPWarps = kPThreads / 32;
-constexpr int kPR = kPartChunk / kPThreads;   // items per thread per chunk
-constexpr int kMaxDigitBits = 8;
+constexpr int kPThreads = 512;                // threads of a count CTA
+constexpr int kSThreads = 512;                // threads of a scatter CTA
+constexpr int kSWarps = kSThreads / 32;
+constexpr int kSR = kPartChunk / kSThreads;   // items per scatter thread per chunk
+constexpr int kMaxDigitBits = HME_PART_MAXB;
 constexpr int kPartTilesPerSM = 2;
 constexpr int kPartSMs = 152;                 // GB300: the tile count fills two CTAs per SM
 constexpr size_t kMaxSmemScatter = 227 * 1024;
-static_assert(kPartChunk % kPThreads == 0 && kPartChunk <= 65536, "chunk positions fit 16 bits");
+static_assert(kPartChunk % kSThreads == 0 && kPartChunk <= 65536, "chunk positions fit 16 bits");
+static_assert(kSR <= 16 && kPartChunk < 65536, "per-thread digit counts and prefixes fit 16-bit halves");
 
 __host__ __device__ __forceinline__ int round4(int k) { return (k + 3) / 4 * 4; }
 
-// Shared-memory layout of the scatter CTA, in 32-bit words: cursors, two key
-// buffers, the per-warp digit counts (rows of 2^bmax + 1 words: the scan
-// walks them column-wise without bank conflicts), the scan's warp totals and
-// (tag lists) the 16 kPR segment sums of the tag-length scan (int64, at an
-// even word).
+// Counter words of a rank pass of B digit bits: two 16-bit counters per word,
+// 2^B / 2 words per thread, laid out word-lane-major (word lane l of thread t
+// at l * kSThreads + t) with one padding word after every raking segment of
+// 2^B / 2 words (the segments are then read without bank conflicts).
+__host__ __device__ constexpr int ctr_lanes(int B) { return B >= 1 ? (1 << B) / 2 : 1; }
+__host__ __device__ __forceinline__ size_t ctr_words(int bmax) {
+  return (size_t)ctr_lanes(bmax) * kSThreads + kSThreads;
+}
+
+// Shared-memory layout of the scatter CTA, in 32-bit words: cursors, the key
+// buffer, the rank counters, the scan's warp totals; with tag lists then the
+// slot of every sorted position, the (j, warp) segment sums of the tag-length
+// scan (int64), the chunk's staged tag offsets int64[kPartChunk + 1], the
+// list destinations by item int64[kPartChunk] and (when it fits) the tag
+// cursors int64[K], the int64 arrays from an even word.
+// Key buffer: position i at word i + i / 32, so that both a thread's 16
+// consecutive positions (blocked) and a warp's 32 consecutive positions
+// (strided) fall into distinct banks.
+__host__ __device__ __forceinline__ int kpad(int i) { return i + (i >> 5); }
+__host__ __device__ __forceinline__ size_t scatter_ctr_word(int K) {
+  return (size_t)round4(K) + (size_t)kPartChunk + kPartChunk / 32;
+}
 __host__ __device__ __forceinline__ size_t scatter_wsum_word(int K, int bmax) {
-  return (size_t)round4(K) + 2 * (size_t)kPartChunk + (size_t)kPWarps * ((1 << bmax) + 1);
+  return scatter_ctr_word(K) + ctr_words(bmax);
+}
+__host__ __device__ __forceinline__ size_t scatter_spare_word(int K, int bmax) {
+  return scatter_wsum_word(K, bmax) + 32;
 }
 __host__ __device__ __forceinline__ size_t scatter_segsum_word(int K, int bmax) {
-  return (scatter_wsum_word(K, bmax) + 32 + 1) & ~(size_t)1;
+  return (scatter_spare_word(K, bmax) + kPartChunk + 1) & ~(size_t)1;
 }
-// tag lists: the chunk's staged offsets int64[kPartChunk + 1], the list
-// destinations by item int64[kPartChunk], and (when it fits) the tag cursors
-// int64[K], from an even word
 __host__ __device__ __forceinline__ size_t scatter_toff_word(int K, int bmax) {
-  return scatter_segsum_word(K, bmax) + 2 * (size_t)kPR * kPWarps;
+  return scatter_segsum_word(K, bmax) + 2 * (size_t)kSR * kSWarps;
 }
 __host__ __device__ __forceinline__ size_t scatter_smem_words(int K, int bmax, bool tags = false,
                                                              bool tcur_smem = false) {
-  if (!tags) return scatter_toff_word(K, bmax);
+  if (!tags) return scatter_spare_word(K, bmax);
   return scatter_toff_word(K, bmax) + 2 * (size_t)(kPartChunk + 2) + 2 * (size_t)kPartChunk +
          (tcur_smem ? 2 * (size_t)K : 0);
 }
@@ -218,88 +244,83 @@ __global__ void __launch_bounds__(1024) part_offsets_kernel(const int64_t *__res
   if (t == 1023) offsets[K] = run;
 }
 
-// Lanes of the warp whose digit equals this lane's (digits in [0, 2^B)).
-template <int B>
-__device__ __forceinline__ unsigned same_digit_lanes(unsigned dig) {
-  unsigned peers = 0xffffffffu;
-#pragma unroll
-  for (int i = 0; i < B; ++i) {
-    const bool bit = (dig >> i) & 1u;
-    const unsigned m = __ballot_sync(0xffffffffu, bit);
-    peers &= bit ? m : ~m;
-  }
-  return peers;
-}
-
-// One stable counting pass of the block-local radix sort.  Item r of this
-// thread sits at position warp * 32 kPR + 32 r + lane of the current order
-// and has packed value v[r] = key << 16 | (position in the chunk's index
-// order); its digit is (key >> SHIFT) mod 2^B.  Every item is written to
-// out[its position in the order by (digit, current position)].
+// One stable counting pass of the block-local radix sort, without ballots:
+// every thread keeps private counters.  Thread t holds the kSR consecutive
+// items kSR t .. kSR t + kSR - 1 of the current order; item r has packed value
+// v[r] = key << 16 | (position in the chunk's index order) and digit
+// (key >> SHIFT) mod 2^B.  (1) Each thread counts its items per digit, an
+// item's rank among its thread's items of the same digit being the count
+// before it (16-bit counters, two per word: digits l and l + 2^B/2 in word
+// lane l).  (2) An exclusive scan of the words in (word lane, thread) order
+// -- each thread sums its raking segment, one block scan of the segment sums
+// -- gives, in each half, the items of smaller digit or of the same digit in
+// lower threads; the upper halves then add the count of all lower-half
+// digits.  (3) Every item is written to out[its digit-and-thread prefix +
+// its rank] (padded index, kpad), its place in the order by (digit, current
+// position).
 template <int B, int SHIFT>
-__device__ __forceinline__ void rank_pass(const uint32_t (&v)[kPR], uint32_t *out, int32_t *wcnt, int32_t *wsum) {
-  constexpr int ND = 1 << B, STRIDE = ND + 1;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int32_t *mine = wcnt + warp * STRIDE;
+__device__ __forceinline__ void rank_pass(const uint32_t (&v)[kSR], uint32_t *out, uint32_t *ctr, uint32_t *wsum) {
+  constexpr int CL = ctr_lanes(B);   // counter words per thread
+  constexpr int SEG = CL;            // raking segment of a thread (words)
+  constexpr unsigned DMASK = (1u << B) - 1u;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  uint32_t *seg = ctr + t * (SEG + 1);  // this thread's raking segment (padded layout)
 #pragma unroll
-  for (int g = lane; g < ND; g += 32) mine[g] = 0;
-  __syncwarp();
-  const unsigned lt = (1u << lane) - 1u;
-  unsigned dig[kPR];
-  int rk[kPR];
+  for (int u = 0; u < SEG; ++u) seg[u] = 0;
+  __syncthreads();
+  uint32_t at[kSR];  // padded word index << 5 | half shift
+  uint32_t rk[kSR];
 #pragma unroll
-  for (int r = 0; r < kPR; ++r) {
-    dig[r] = (v[r] >> (16 + SHIFT)) & (unsigned)(ND - 1);
-    const unsigned peers = same_digit_lanes<B>(dig[r]);
-    const int before = mine[dig[r]];
-    rk[r] = before + __popc(peers & lt);
-    __syncwarp();
-    if ((peers & lt) == 0) mine[dig[r]] = before + __popc(peers);  // the lowest lane of the group
-    __syncwarp();
+  for (int r = 0; r < kSR; ++r) {
+    const unsigned d = (v[r] >> (16 + SHIFT)) & DMASK;
+    const unsigned l = d % CL, sh = (d / CL) * 16;
+    const unsigned i = l * kSThreads + t;
+    const unsigned pi = i + i / SEG;
+    // a shared atomic, not a load and a store: the thread's 16 increments
+    // then issue back to back (only this thread touches these words)
+    const uint32_t w = atomicAdd(&ctr[pi], 1u << sh);
+    rk[r] = (w >> sh) & 0xFFFFu;
+    at[r] = (pi << 5) | sh;
   }
   __syncthreads();
-  // exclusive scan over the (digit, warp) counts, digit-major: entry e is
-  // (digit e / kPWarps, warp e % kPWarps)
-  constexpr int NE = ND * kPWarps;
-  constexpr int PER = (NE + kPThreads - 1) / kPThreads;
-  const int e0 = threadIdx.x * PER;
-  int cv[PER];
-  int local = 0;
+  // raking: segment sums, block exclusive scan (packed 16-bit halves)
+  uint32_t sum = 0;
 #pragma unroll
-  for (int u = 0; u < PER; ++u) {
-    const int e = e0 + u;
-    cv[u] = e < NE ? wcnt[(e % kPWarps) * STRIDE + e / kPWarps] : 0;
-    local += cv[u];
-  }
-  int incl = local;
+  for (int u = 0; u < SEG; ++u) sum += seg[u];
+  uint32_t incl = sum;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int t = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += t;
+    const uint32_t x = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += x;
   }
   if (lane == 31) wsum[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    const int w = lane < kPWarps ? wsum[lane] : 0;
-    int wi = w;
+    const uint32_t w = lane < kSWarps ? wsum[lane] : 0u;
+    uint32_t wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int t = __shfl_up_sync(0xffffffffu, wi, o);
-      if (lane >= o) wi += t;
+      const uint32_t x = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += x;
     }
-    if (lane < kPWarps) wsum[lane] = wi - w;
+    if (lane < kSWarps) wsum[lane] = wi - w;
+    if (lane == kSWarps - 1) wsum[kSWarps] = wi;  // the grand total
   }
   __syncthreads();
-  int run = wsum[warp] + incl - local;
+  // the upper halves follow every lower-half digit
+  uint32_t run = wsum[warp] + incl - sum + ((wsum[kSWarps] & 0xFFFFu) << 16);
 #pragma unroll
-  for (int u = 0; u < PER; ++u) {
-    const int e = e0 + u;
-    if (e < NE) wcnt[(e % kPWarps) * STRIDE + e / kPWarps] = run;
-    run += cv[u];
+  for (int u = 0; u < SEG; ++u) {
+    const uint32_t w = seg[u];
+    seg[u] = run;
+    run += w;
   }
   __syncthreads();
 #pragma unroll
-  for (int r = 0; r < kPR; ++r) out[mine[dig[r]] + rk[r]] = v[r];
+  for (int r = 0; r < kSR; ++r) {
+    const uint32_t w = ctr[at[r] >> 5];
+    out[kpad((int)(((w >> (at[r] & 31u)) & 0xFFFFu) + rk[r]))] = v[r];
+  }
   __syncthreads();
 }
 
@@ -326,102 +347,112 @@ struct TagArgs {
   int tcur_smem;            // the tag cursors fit in shared memory
 };
 
-// The stable scatter (see the file comment): chunks sorted by passes of B0
-// and then B1 (0: none) digit bits.  perm_out[slot] = item index.
-template <int B0, int B1, bool TAGS>
-__global__ void __launch_bounds__(kPThreads, TAGS ? 1 : kPartTilesPerSM)
+// The stable scatter (see the file comment): chunks sorted by passes of B0,
+// then B1 and B2 (0: none) digit bits.  perm_out[slot] = item index.
+template <int B0, int B1, int B2, bool TAGS>
+__global__ void __launch_bounds__(kSThreads, TAGS ? 1 : kPartTilesPerSM)
     part_scatter_kernel(const int32_t *__restrict__ labels, int64_t N, int K, int64_t tile,
                         const int32_t *__restrict__ tileoff, const int64_t *__restrict__ offsets,
                         int32_t *__restrict__ perm_out, TagArgs ta) {
-  constexpr int BMAX = B0 > B1 ? B0 : B1;
+  constexpr int BMAX = B0 > B1 ? (B0 > B2 ? B0 : B2) : (B1 > B2 ? B1 : B2);
   extern __shared__ uint32_t psm[];
   int32_t *cursor = reinterpret_cast<int32_t *>(psm);
-  uint32_t *ka = psm + round4(K);
-  uint32_t *kb = ka + kPartChunk;
-  int32_t *wcnt = reinterpret_cast<int32_t *>(kb + kPartChunk);
-  int32_t *wsum = reinterpret_cast<int32_t *>(psm + scatter_wsum_word(K, BMAX));
-  // TAGS: per-(j, warp) segment sums of the tag-length scan, staged offsets,
-  // destinations by item, tag cursors
+  uint32_t *keys = psm + round4(K);
+  uint32_t *ctr = psm + scatter_ctr_word(K);
+  uint32_t *wsum = psm + scatter_wsum_word(K, BMAX);
+  // TAGS: slot by sorted position, per-(j, warp) segment sums of the tag-length
+  // scan, staged offsets, destinations by item, tag cursors
+  uint32_t *spare = psm + scatter_spare_word(K, BMAX);
   int64_t *segsum = reinterpret_cast<int64_t *>(psm + scatter_segsum_word(K, BMAX));
   int64_t *toff = reinterpret_cast<int64_t *>(psm + scatter_toff_word(K, BMAX));
   int64_t *dsts = toff + kPartChunk + 2;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t t = blockIdx.x;
-  for (int k = threadIdx.x; k < K; k += kPThreads) cursor[k] = (int32_t)(offsets[k] + tileoff[t * K + k]);
+  for (int k = threadIdx.x; k < K; k += kSThreads) cursor[k] = (int32_t)(offsets[k] + tileoff[t * K + k]);
   int64_t *tcur = nullptr;
   if (TAGS) {
     tcur = ta.tcur_smem ? dsts + kPartChunk : ta.tagcur + t * K;
-    for (int k = threadIdx.x; k < K; k += kPThreads) tcur[k] = ta.tagcur[t * K + k] + ta.tag_base[k];
+    for (int k = threadIdx.x; k < K; k += kSThreads) tcur[k] = ta.tagcur[t * K + k] + ta.tag_base[k];
   }
   const int64_t start = t * tile;
   const int64_t end = min(N, start + tile);
-  // item r of a thread: chunk position warp * 32 kPR + 32 r + lane (32 consecutive labels per warp load)
-  const int pbase = warp * 32 * kPR + lane;
-  int32_t lab[kPR];
+  // thread t holds chunk positions kSR t .. kSR t + kSR - 1 (blocked); the
+  // base is 16-byte aligned when labels is (start is a multiple of the chunk)
+  const int pbase = threadIdx.x * kSR;
+  const bool vec = (reinterpret_cast<uintptr_t>(labels) & 15u) == 0;
+  int32_t lab[kSR];
+  auto load = [&](int64_t at) {
+    if (vec && at + pbase + kSR <= end) {
+      const int4 *src = reinterpret_cast<const int4 *>(labels + at + pbase);
 #pragma unroll
-  for (int r = 0; r < kPR; ++r) {
-    const int64_t i = start + pbase + 32 * r;
-    lab[r] = i < end ? __ldg(labels + i) : -1;
-  }
+      for (int u = 0; u < kSR / 4; ++u) {
+        const int4 x = __ldg(src + u);
+        lab[4 * u] = x.x;
+        lab[4 * u + 1] = x.y;
+        lab[4 * u + 2] = x.z;
+        lab[4 * u + 3] = x.w;
+      }
+    } else {
+#pragma unroll
+      for (int r = 0; r < kSR; ++r) {
+        const int64_t i = at + pbase + r;
+        lab[r] = i < end ? __ldg(labels + i) : -1;
+      }
+    }
+  };
+  load(start);
   for (int64_t pos = start; pos < end; pos += kPartChunk) {
     const int nvalid = (int)min((int64_t)kPartChunk, end - pos);
     if (TAGS) {
       // toff[p] = tag_off[pos + p], p <= nvalid (8-byte asynchronous copies)
-      for (int q = threadIdx.x; q <= nvalid; q += kPThreads)
+      for (int q = threadIdx.x; q <= nvalid; q += kSThreads)
         asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_u32(toff + q)), "l"(ta.tag_off + pos + q)
                      : "memory");
       asm volatile("cp.async.commit_group;" ::: "memory");
     }
-    uint32_t v[kPR];
-    unsigned okmask = 0;  // bit r: this thread's item r has a label in [0, K)
+    uint32_t v[kSR];
 #pragma unroll
-    for (int r = 0; r < kPR; ++r) {
-      const bool ok = lab[r] >= 0 && lab[r] < K;
-      const unsigned key = ok ? (unsigned)lab[r] : (unsigned)K;
-      v[r] = (key << 16) | (unsigned)(pbase + 32 * r);
-      if (ok) okmask |= 1u << r;
+    for (int r = 0; r < kSR; ++r) {
+      const unsigned key = (lab[r] >= 0 && lab[r] < K) ? (unsigned)lab[r] : (unsigned)K;
+      v[r] = (key << 16) | (unsigned)(pbase + r);
     }
     // the next chunk's labels are in flight during the sort of this one
-    const int64_t nxt = pos + kPartChunk;
+    load(pos + kPartChunk);
+    rank_pass<B0, 0>(v, keys, ctr, wsum);
+    if (B1 > 0) {  // the second pass reads its items before the first writes over them (rank_pass syncs)
 #pragma unroll
-    for (int r = 0; r < kPR; ++r) {
-      const int64_t i = nxt + pbase + 32 * r;
-      lab[r] = i < end ? __ldg(labels + i) : -1;
+      for (int r = 0; r < kSR; ++r) v[r] = keys[kpad(pbase + r)];
+      rank_pass<(B1 > 0 ? B1 : 1), B0>(v, keys, ctr, wsum);
     }
-    rank_pass<B0, 0>(v, kb, wcnt, wsum);
-    const uint32_t *sorted = kb;
-    uint32_t *spare = ka;
-    if (B1 > 0) {
-      uint32_t w[kPR];
+    if (B2 > 0) {
 #pragma unroll
-      for (int r = 0; r < kPR; ++r) w[r] = kb[pbase + 32 * r];
-      rank_pass<(B1 > 0 ? B1 : 1), B0>(w, ka, wcnt, wsum);
-      sorted = ka;
-      spare = kb;
+      for (int r = 0; r < kSR; ++r) v[r] = keys[kpad(pbase + r)];
+      rank_pass<(B2 > 0 ? B2 : 1), B0 + B1>(v, keys, ctr, wsum);
     }
+    const uint32_t *sorted = keys;
     // runs of equal keys: the first item of a run turns the bucket's cursor
     // into its base (cursor - position), every item stores at base + position,
     // the last item moves the cursor past the run.  Sorted position q of item
-    // j of this thread is tid + kPThreads j: consecutive lanes, consecutive q.
-    uint32_t sv[kPR];
+    // j of this thread is tid + kSThreads j: consecutive lanes, consecutive q.
+    uint32_t sv[kSR];
     unsigned last = 0;  // bit j: item j ends its run
 #pragma unroll
-    for (int j = 0; j < kPR; ++j) {
-      const int q = threadIdx.x + kPThreads * j;
-      sv[j] = sorted[q];
+    for (int j = 0; j < kSR; ++j) {
+      const int q = threadIdx.x + kSThreads * j;
+      sv[j] = sorted[kpad(q)];
       const unsigned key = sv[j] >> 16;
       unsigned prev = __shfl_up_sync(0xffffffffu, key, 1);
       unsigned next = __shfl_down_sync(0xffffffffu, key, 1);
-      if (lane == 0) prev = q > 0 ? (sorted[q - 1] >> 16) : 0xFFFFFFFFu;
-      if (lane == 31) next = q + 1 < kPartChunk ? (sorted[q + 1] >> 16) : 0xFFFFFFFFu;
+      if (lane == 0) prev = q > 0 ? (sorted[kpad(q - 1)] >> 16) : 0xFFFFFFFFu;
+      if (lane == 31) next = q + 1 < kPartChunk ? (sorted[kpad(q + 1)] >> 16) : 0xFFFFFFFFu;
       if (key != next) last |= 1u << j;
       if (key < (unsigned)K && key != prev) cursor[key] -= q;
     }
     __syncthreads();
-    int32_t slot[kPR];
+    int32_t slot[kSR];
 #pragma unroll
-    for (int j = 0; j < kPR; ++j) {
-      const int q = threadIdx.x + kPThreads * j;
+    for (int j = 0; j < kSR; ++j) {
+      const int q = threadIdx.x + kSThreads * j;
       const unsigned key = sv[j] >> 16;
       slot[j] = -1;
       if (key < (unsigned)K) {
@@ -432,19 +463,19 @@ __global__ void __launch_bounds__(kPThreads, TAGS ? 1 : kPartTilesPerSM)
     }
     __syncthreads();
 #pragma unroll
-    for (int j = 0; j < kPR; ++j)
+    for (int j = 0; j < kSR; ++j)
       if (slot[j] >= 0 && ((last >> j) & 1u)) cursor[sv[j] >> 16] = slot[j] + 1;
     if (TAGS) {
       asm volatile("cp.async.wait_all;" ::: "memory");
       __syncthreads();
       // lengths in sorted order and their block-wide exclusive prefix: a warp
-      // scan per j, then the 16 kPR (j, warp) segments in order
-      int64_t incl[kPR];
-      int32_t len[kPR];
+      // scan per j, then the kSR kSWarps (j, warp) segments in order
+      int64_t incl[kSR];
+      int32_t len[kSR];
       // 32-bit warp scans when the chunk's lists hold fewer than 2^31 tags
       const bool narrow = toff[nvalid] - toff[0] < ((int64_t)1 << 31);
 #pragma unroll
-      for (int j = 0; j < kPR; ++j) {
+      for (int j = 0; j < kSR; ++j) {
         const unsigned key = sv[j] >> 16;
         const int p = (int)(sv[j] & 0xFFFFu);
         len[j] = key < (unsigned)K ? (int32_t)(toff[p + 1] - toff[p]) : 0;
@@ -466,11 +497,11 @@ __global__ void __launch_bounds__(kPThreads, TAGS ? 1 : kPartTilesPerSM)
           }
         }
         incl[j] = x;
-        if (lane == 31) segsum[j * kPWarps + warp] = x;
+        if (lane == 31) segsum[j * kSWarps + warp] = x;
       }
       __syncthreads();
       if (warp == 0) {
-        constexpr int NS = kPR * kPWarps;  // segments in sorted order
+        constexpr int NS = kSR * kSWarps;  // segments in sorted order
         constexpr int PS = NS / 32;
         int64_t sv4[PS];
         int64_t loc = 0;
@@ -495,54 +526,57 @@ __global__ void __launch_bounds__(kPThreads, TAGS ? 1 : kPartTilesPerSM)
       __syncthreads();
       // run starts: tag cursor -> base (cursor - P of the run's first item)
 #pragma unroll
-      for (int j = 0; j < kPR; ++j) {
-        const int q = threadIdx.x + kPThreads * j;
-        incl[j] += segsum[j * kPWarps + warp] - len[j];  // P: exclusive prefix of this item
+      for (int j = 0; j < kSR; ++j) {
+        const int q = threadIdx.x + kSThreads * j;
+        incl[j] += segsum[j * kSWarps + warp] - len[j];  // P: exclusive prefix of this item
         const unsigned key = sv[j] >> 16;
         unsigned prev = __shfl_up_sync(0xffffffffu, key, 1);
-        if (lane == 0) prev = q > 0 ? (sorted[q - 1] >> 16) : 0xFFFFFFFFu;
+        if (lane == 0) prev = q > 0 ? (sorted[kpad(q - 1)] >> 16) : 0xFFFFFFFFu;
         if (key < (unsigned)K && key != prev) tcur[key] -= incl[j];
       }
       __syncthreads();
-      // destinations: by slot (tag_off_out) and by item (for the copy)
+      // destinations: by slot (tag_off_out) and by item (for the copy; -1:
+      // an invalid label or a position past the tile, whose list stays)
 #pragma unroll
-      for (int j = 0; j < kPR; ++j) {
-        const int q = threadIdx.x + kPThreads * j;
+      for (int j = 0; j < kSR; ++j) {
+        const int q = threadIdx.x + kSThreads * j;
         const unsigned key = sv[j] >> 16;
         if (key < (unsigned)K) {
           const int64_t dst = tcur[key] + incl[j];
           ta.tag_off_out[(int32_t)spare[q]] = dst;
           dsts[sv[j] & 0xFFFFu] = dst;
           incl[j] = dst + len[j];  // the end of this item's list
+        } else {
+          dsts[sv[j] & 0xFFFFu] = -1;
         }
       }
       __syncthreads();
 #pragma unroll
-      for (int j = 0; j < kPR; ++j)
+      for (int j = 0; j < kSR; ++j)
         if ((sv[j] >> 16) < (unsigned)K && ((last >> j) & 1u)) tcur[sv[j] >> 16] = incl[j];
-      // copy in source order: item r of this thread sits at pbase + 32 r, so
-      // a warp's loads of its lists' first tags read neighbouring memory; the
-      // first four tags of two items are loaded before any is stored (eight
-      // loads in flight), longer lists finish in a loop
+      // copy in source order: item p = tid + kSThreads j, so a warp's loads of
+      // its lists' first tags read neighbouring memory; the first four tags of
+      // two items are loaded before any is stored (eight loads in flight),
+      // longer lists finish in a loop
 #pragma unroll 1
-      for (int r = 0; r < kPR; r += 2) {
+      for (int j = 0; j < kSR; j += 2) {
         int64_t src[2], dst[2];
-        int32_t ln[2], v[2][4];
+        int32_t ln[2], w[2][4];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          const int pp = pbase + 32 * (r + h);
-          const bool ok = (okmask >> (r + h)) & 1u;
+          const int pp = threadIdx.x + kSThreads * (j + h);
+          dst[h] = dsts[pp];
+          const bool ok = dst[h] >= 0;
           src[h] = ok ? toff[pp] : 0;
           ln[h] = ok ? (int32_t)(toff[pp + 1] - src[h]) : 0;
-          dst[h] = ok ? dsts[pp] : 0;
 #pragma unroll
-          for (int u = 0; u < 4; ++u) v[h][u] = u < ln[h] ? __ldg(ta.tags + src[h] + u) : 0;
+          for (int u = 0; u < 4; ++u) w[h][u] = u < ln[h] ? __ldg(ta.tags + src[h] + u) : 0;
         }
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
 #pragma unroll
           for (int u = 0; u < 4; ++u)
-            if (u < ln[h]) ta.tags_out[dst[h] + u] = v[h][u];
+            if (u < ln[h]) ta.tags_out[dst[h] + u] = w[h][u];
           for (int32_t u = 4; u < ln[h]; ++u) ta.tags_out[dst[h] + u] = __ldg(ta.tags + src[h] + u);
         }
       }
@@ -601,26 +635,43 @@ __global__ void part_fill_labels_kernel(const int64_t *__restrict__ offsets, int
   }
 }
 
-// The scatter instance for digit bits (b0, b1): one pass of 1 .. 8 bits, or
-// two passes of 4 .. 8 bits (keys of 9 .. 15 bits).
+// The scatter instance for digit bits (b0, b1, b2) (0: no such pass).
 template <bool TAGS>
-ScatterFn scatter_fn(int b0, int b1) {
-  switch (b0 * 16 + b1) {
-    case 1 * 16: return part_scatter_kernel<1, 0, TAGS>;
-    case 2 * 16: return part_scatter_kernel<2, 0, TAGS>;
-    case 3 * 16: return part_scatter_kernel<3, 0, TAGS>;
-    case 4 * 16: return part_scatter_kernel<4, 0, TAGS>;
-    case 5 * 16: return part_scatter_kernel<5, 0, TAGS>;
-    case 6 * 16: return part_scatter_kernel<6, 0, TAGS>;
-    case 7 * 16: return part_scatter_kernel<7, 0, TAGS>;
-    case 8 * 16: return part_scatter_kernel<8, 0, TAGS>;
-    case 4 * 16 + 5: return part_scatter_kernel<4, 5, TAGS>;
-    case 5 * 16 + 5: return part_scatter_kernel<5, 5, TAGS>;
-    case 5 * 16 + 6: return part_scatter_kernel<5, 6, TAGS>;
-    case 6 * 16 + 6: return part_scatter_kernel<6, 6, TAGS>;
-    case 6 * 16 + 7: return part_scatter_kernel<6, 7, TAGS>;
-    case 7 * 16 + 7: return part_scatter_kernel<7, 7, TAGS>;
-    case 7 * 16 + 8: return part_scatter_kernel<7, 8, TAGS>;
+ScatterFn scatter_fn(int b0, int b1, int b2) {
+  switch (b0 * 256 + b1 * 16 + b2) {
+    case 1 * 256 + 0 * 16 + 0: return part_scatter_kernel<1, 0, 0, TAGS>;
+    case 2 * 256 + 0 * 16 + 0: return part_scatter_kernel<2, 0, 0, TAGS>;
+    case 3 * 256 + 0 * 16 + 0: return part_scatter_kernel<3, 0, 0, TAGS>;
+    case 4 * 256 + 0 * 16 + 0: return part_scatter_kernel<4, 0, 0, TAGS>;
+    case 5 * 256 + 0 * 16 + 0: return part_scatter_kernel<5, 0, 0, TAGS>;
+    case 6 * 256 + 0 * 16 + 0: return part_scatter_kernel<6, 0, 0, TAGS>;
+    case 7 * 256 + 0 * 16 + 0: return part_scatter_kernel<7, 0, 0, TAGS>;
+    case 1 * 256 + 1 * 16 + 0: return part_scatter_kernel<1, 1, 0, TAGS>;
+    case 2 * 256 + 1 * 16 + 0: return part_scatter_kernel<2, 1, 0, TAGS>;
+    case 2 * 256 + 2 * 16 + 0: return part_scatter_kernel<2, 2, 0, TAGS>;
+    case 3 * 256 + 2 * 16 + 0: return part_scatter_kernel<3, 2, 0, TAGS>;
+    case 3 * 256 + 3 * 16 + 0: return part_scatter_kernel<3, 3, 0, TAGS>;
+    case 4 * 256 + 3 * 16 + 0: return part_scatter_kernel<4, 3, 0, TAGS>;
+    case 4 * 256 + 4 * 16 + 0: return part_scatter_kernel<4, 4, 0, TAGS>;
+    case 5 * 256 + 4 * 16 + 0: return part_scatter_kernel<5, 4, 0, TAGS>;
+    case 5 * 256 + 5 * 16 + 0: return part_scatter_kernel<5, 5, 0, TAGS>;
+    case 6 * 256 + 5 * 16 + 0: return part_scatter_kernel<6, 5, 0, TAGS>;
+    case 6 * 256 + 6 * 16 + 0: return part_scatter_kernel<6, 6, 0, TAGS>;
+    case 7 * 256 + 6 * 16 + 0: return part_scatter_kernel<7, 6, 0, TAGS>;
+    case 7 * 256 + 7 * 16 + 0: return part_scatter_kernel<7, 7, 0, TAGS>;
+    case 1 * 256 + 1 * 16 + 1: return part_scatter_kernel<1, 1, 1, TAGS>;
+    case 2 * 256 + 1 * 16 + 1: return part_scatter_kernel<2, 1, 1, TAGS>;
+    case 2 * 256 + 2 * 16 + 1: return part_scatter_kernel<2, 2, 1, TAGS>;
+    case 2 * 256 + 2 * 16 + 2: return part_scatter_kernel<2, 2, 2, TAGS>;
+    case 3 * 256 + 2 * 16 + 2: return part_scatter_kernel<3, 2, 2, TAGS>;
+    case 3 * 256 + 3 * 16 + 2: return part_scatter_kernel<3, 3, 2, TAGS>;
+    case 3 * 256 + 3 * 16 + 3: return part_scatter_kernel<3, 3, 3, TAGS>;
+    case 4 * 256 + 3 * 16 + 3: return part_scatter_kernel<4, 3, 3, TAGS>;
+    case 4 * 256 + 4 * 16 + 3: return part_scatter_kernel<4, 4, 3, TAGS>;
+    case 4 * 256 + 4 * 16 + 4: return part_scatter_kernel<4, 4, 4, TAGS>;
+    case 5 * 256 + 4 * 16 + 4: return part_scatter_kernel<5, 4, 4, TAGS>;
+    case 5 * 256 + 5 * 16 + 4: return part_scatter_kernel<5, 5, 4, TAGS>;
+    case 5 * 256 + 5 * 16 + 5: return part_scatter_kernel<5, 5, 5, TAGS>;
     default: return nullptr;
   }
 }
@@ -631,8 +682,15 @@ PartLayout part_layout(size_t base, int64_t N, int K, bool tags) {
   PartLayout pl;
   int bits = 0;
   while ((1 << bits) < K + 1) ++bits;  // labels 0 .. K-1 and the key K of an invalid label
-  pl.b0 = bits <= kMaxDigitBits ? bits : bits / 2;
-  pl.b1 = bits - pl.b0;
+  // passes of at most kMaxDigitBits bits, as equal as possible (larger first):
+  // small digits keep the per-thread counters, which every pass clears and
+  // scans, small
+  const int npass = (bits + kMaxDigitBits - 1) / kMaxDigitBits;
+  int b[3] = {0, 0, 0};
+  for (int i = 0; i < npass; ++i) b[i] = bits / npass + (i < bits % npass ? 1 : 0);
+  pl.b0 = b[0];
+  pl.b1 = b[1];
+  pl.b2 = b[2];
   // two CTAs per SM; one with tag lists (whose scatter needs more registers)
   const int64_t target = (tags ? 1 : kPartTilesPerSM) * kPartSMs;
   int64_t tile = (N + target - 1) / target;
@@ -671,11 +729,11 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
   int64_t *tag_hist = tags ? reinterpret_cast<int64_t *>(ws + pl.tag_hist) : nullptr;
   int64_t *tag_base = tags ? reinterpret_cast<int64_t *>(ws + pl.tag_base) : nullptr;
   const size_t smc = (size_t)round4(K) * sizeof(int32_t) + (tags ? (size_t)K * sizeof(int64_t) : 0);
-  const int bmax = pl.b0 > pl.b1 ? pl.b0 : pl.b1;
+  const int bmax = std::max(pl.b0, std::max(pl.b1, pl.b2));
   const bool tcur_smem = tags && scatter_smem_words(K, bmax, true, true) * sizeof(uint32_t) <= kMaxSmemScatter;
   const size_t sms = scatter_smem_words(K, bmax, tags, tcur_smem) * sizeof(uint32_t);
   auto count = tags ? part_count_kernel<true> : part_count_kernel<false>;
-  ScatterFn scatter = tags ? scatter_fn<true>(pl.b0, pl.b1) : scatter_fn<false>(pl.b0, pl.b1);
+  ScatterFn scatter = tags ? scatter_fn<true>(pl.b0, pl.b1, pl.b2) : scatter_fn<false>(pl.b0, pl.b1, pl.b2);
   if (!scatter) return cudaErrorInvalidValue;
   cudaError_t e;
   if (smc > 48 * 1024) {
@@ -702,7 +760,7 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
   if (pl.ntiles > 0) {
     TagArgs ta{};
     if (tags) ta = TagArgs{tl->tag_off, tl->tags, tagcnt, tag_base, tl->tag_off_out, tl->tags_out, tcur_smem ? 1 : 0};
-    scatter<<<(unsigned)pl.ntiles, kPThreads, sms, s>>>(labels, N, K, pl.tile, tilecnt, offsets, perm, ta);
+    scatter<<<(unsigned)pl.ntiles, kSThreads, sms, s>>>(labels, N, K, pl.tile, tilecnt, offsets, perm, ta);
     count_launch();
     if (sorted_labels) {
       const int64_t threads = (N + kFillSlots - 1) / kFillSlots;
