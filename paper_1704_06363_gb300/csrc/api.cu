@@ -142,6 +142,7 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   L.full_rows = take((size_t)(N > 0 ? N : 1) * 4);
   L.perm = take((size_t)(N > 0 ? N : 1) * 4);
   L.slab = take((size_t)(N > 0 ? N : 1) * 4);
+  L.split = take((size_t)(N < kSplitRows ? (N > 0 ? N : 1) : kSplitRows) * kMaxSlices * 16);
   L.part = part_layout(align_up(off, 256), N, K);
   off = L.part.end;
   L.sums = take((size_t)K * d * 8);
@@ -272,7 +273,7 @@ int launch_assign_prepared(const void *X, int64_t N, int64_t ldx, int dtype, con
   const int64_t lda = split ? g.ldp : ldx;
   HME_TRY(launch_assign(Xa, Xb, N, lda, g, at<void>(ws, L.cb_hi), at<__nv_bfloat16>(ws, L.cb_lo),
                         at<float>(ws, L.cn), at<float>(ws, L.xn), labels, mind, hdr, at<int32_t>(ws, L.flagged),
-                        at<int32_t>(ws, L.full_rows), s));
+                        at<int32_t>(ws, L.full_rows), at<float4>(ws, L.split), s));
   return HME_OK;
 }
 

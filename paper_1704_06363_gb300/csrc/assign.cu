@@ -83,6 +83,11 @@ struct AssignParams {
   float err_acc;    // ceil(d/16) * nprod * 2^-22 + 2^-20: accumulation + epilogue rounding
   float err_split;  // 2^-14 for split fp32 operands, else 0
   float err_ll;     // 1.0625 * 2^-14 for split fp32 operands (the dropped xl.cl), else 0
+  // small batches (lean scan only): the N-chunks of a row tile are spread over
+  // `slices` CTAs of cps chunks each; each writes its row states to part and
+  // assign_merge_kernel finishes the rows
+  int slices, cps;
+  float4 *part;     // [N][slices]: best, runner-up, best's index (bits)
 };
 
 constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4, kWhereXchg = 6;
@@ -336,7 +341,9 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       const uint64_t pol_b = l2_policy_evict_last();
       uint32_t it = 0, tile_it = 0;
       bool ok = true, a_pending = false;
-      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+      for (int item = blockIdx.x; item < p.num_tiles * p.slices && ok; item += gridDim.x, ++tile_it) {
+        const int tile = item / p.slices;
+        const int ch0 = (item % p.slices) * p.cps, ch1 = min(p.nchunks, ch0 + p.cps);
         const int32_t row0 = tile * BMT;
         if (ARES) {
           // the previous tile's MMAs must be done with the resident A rows
@@ -353,7 +360,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             }
           a_pending = true;
         }
-        for (int ch = 0; ch < p.nchunks && ok; ++ch) {
+        for (int ch = ch0; ch < ch1 && ok; ++ch) {
           for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
             const int s = it % S;
             const uint32_t ph = (it / S) & 1u;
@@ -391,7 +398,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       const uint32_t idesc = TF32 ? idesc_tf32_f32(kBM, (uint32_t)p.BN) : idesc_bf16_f32(kBM, (uint32_t)p.BN);
       uint32_t it = 0, acc_it = 0, tile_it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+      for (int item = blockIdx.x; item < p.num_tiles * p.slices && ok; item += gridDim.x, ++tile_it) {
+        const int ch0 = (item % p.slices) * p.cps, ch1 = min(p.nchunks, ch0 + p.cps);
         if (ARES) {
           if (!mbar_wait_bounded(smem_u32(a_full), tile_it & 1u, p.limit_ns, p.hdr, kWhereMma)) {
             ok = false;
@@ -399,7 +407,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           }
           tc_fence_after();
         }
-        for (int ch = 0; ch < p.nchunks && ok; ++ch, ++acc_it) {
+        for (int ch = ch0; ch < ch1 && ok; ++ch, ++acc_it) {
           const uint32_t a = acc_it % (uint32_t)nbuf;
           const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
           if (!mbar_wait_bounded(smem_u32(&tempty[a]), aph ^ 1u, p.limit_ns, p.hdr, kWhereMmaAcc)) {
@@ -478,9 +486,13 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
         cn_next[r] = (t < c1) ? __ldg(p.cn + ch * p.BN + t) : 0.0f;
       }
     };
-    fetch_cn(0);
+    fetch_cn(((int)blockIdx.x % p.slices) * p.cps);  // the first item's first chunk
     bool cb_filled = false;
-    for (int tile = blockIdx.x; tile < p.num_tiles && ok; tile += gridDim.x, ++tile_it) {
+    for (int item = blockIdx.x; item < p.num_tiles * p.slices && ok; item += gridDim.x, ++tile_it) {
+      const int tile = item / p.slices, slice = item % p.slices;
+      const int ch0 = slice * p.cps, ch1 = min(p.nchunks, ch0 + p.cps);
+      // the first chunk of this CTA's next work item (its scan prefetches that chunk's norms)
+      const int next_ch0 = ((item + (int)gridDim.x) % p.slices) * p.cps;
       float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
       int idx1 = 0, idx2 = 0;
       float lb1 = INFINITY, lb2 = INFINITY;  // second independent state of the lean scan (odd groups)
@@ -489,7 +501,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       int li2 = 0;
       const int64_t row = (int64_t)tile * BMT + row_in_tile;
       const float xr = (half == 0 && row < p.N) ? __ldg(p.xn + row) : 0.0f;  // in flight during the scan
-      for (int ch = 0; ch < p.nchunks; ++ch, ++acc_it) {
+      for (int ch = ch0; ch < ch1; ++ch, ++acc_it) {
         if (p.nchunks > 1 || !cb_filled) {
           __syncwarp();
 #pragma unroll
@@ -497,7 +509,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             if (c0 + lane + 32 * r < c1) cb[lane + 32 * r] = cn_next[r];
           __syncwarp();
           cb_filled = true;
-          if (p.nchunks > 1) fetch_cn(ch + 1 < p.nchunks ? ch + 1 : 0);
+          if (p.nchunks > 1) fetch_cn(ch + 1 < ch1 ? ch + 1 : next_ch0);
         }
         const uint32_t a = acc_it % (uint32_t)nbuf;
         const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
@@ -613,7 +625,13 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           }
         }
       }
-      if (row < p.N) obj += finish_row<LEAN>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
+      if (p.slices > 1) {
+        // a slice of the centres: its row state goes to assign_merge_kernel
+        if (LEAN && row < p.N)
+          p.part[row * p.slices + slice] = make_float4(best1, best2, __int_as_float(idx1), 0.0f);
+      } else if (row < p.N) {
+        obj += finish_row<LEAN>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
@@ -626,6 +644,32 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
+}
+
+// Small batches: the row states of the centre slices (lean scan: best value,
+// runner-up value, best's index) merged per row, then the row finished as in
+// the assign kernel (label, distance, near-tie queue, objective).
+__global__ void __launch_bounds__(256) assign_merge_kernel(const AssignParams p) {
+  const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
+  const float sqrt_cn_max = sqrtf(cn_max);
+  double obj = 0.0;
+  for (int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; row < p.N;
+       row += (int64_t)gridDim.x * blockDim.x) {
+    float best1 = INFINITY, best2 = INFINITY;
+    int idx1 = 0;
+    for (int sl = 0; sl < p.slices; ++sl) {
+      const float4 v = p.part[row * p.slices + sl];
+      const int i = __float_as_int(v.z);
+      const bool take = v.x < best1 || (v.x == best1 && i < idx1);
+      best2 = fminf(fmaxf(best1, v.x), fminf(best2, v.y));
+      best1 = take ? v.x : best1;
+      idx1 = take ? i : idx1;
+    }
+    obj += finish_row<true>(p, row, __ldg(p.xn + row), best1, best2, INFINITY, idx1, 0, cn_max, sqrt_cn_max);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
+  if ((threadIdx.x & 31) == 0 && obj != 0.0) atomicAdd(&p.hdr->objective, obj);
 }
 
 // ---------------------------------------------------------------------------
@@ -1433,7 +1477,7 @@ constexpr int kAresCS = 2;
 
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g, const void *chi,
                   const __nv_bfloat16 *clo, const float *cn, const float *xn, int32_t *labels, float *mind,
-                  Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s) {
+                  Header *hdr, int32_t *flagged, int32_t *full_rows, float4 *part, cudaStream_t s) {
   if (N == 0) return HME_OK;
   CUtensorMap mA0, mA1, mB0, mB1;
   int rc;
@@ -1496,10 +1540,25 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   // split operands: the dropped xl.cl; tf32 operands: their rounding (6.002 * 2^-10)
   p.err_ll = g.nprod == 3 ? 0x1.1p-14f : (g.tf32 ? (float)(6.002 * 0x1p-10) : 0.0f);
   const size_t smem = (size_t)p.a_res_bytes + (size_t)stages * p.stage_bytes + 1024 + ctrl_bytes;
-  int grid = num_sms();
-  if (grid > p.num_tiles) grid = p.num_tiles;
-  cudaError_t e;
   const bool lean = g.nchunks > 1;
+  // Few row tiles (a small routed batch) would leave most SMs idle: spread
+  // each tile's N-chunks over up to kMaxSlices CTAs (lean scan only).
+  p.slices = 1;
+  p.cps = g.nchunks;
+  p.part = nullptr;
+  if (lean && !g.tf32 && part && N <= kSplitRows && 2 * p.num_tiles <= num_sms()) {
+    int sl = num_sms() / p.num_tiles;
+    if (sl > g.nchunks) sl = g.nchunks;
+    if (sl > kMaxSlices) sl = kMaxSlices;
+    if (sl >= 2) {
+      p.cps = (g.nchunks + sl - 1) / sl;
+      p.slices = (g.nchunks + p.cps - 1) / p.cps;  // no empty slice
+      p.part = part;
+    }
+  }
+  int grid = num_sms();
+  if (grid > p.num_tiles * p.slices) grid = p.num_tiles * p.slices;
+  cudaError_t e;
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
   if (g.tf32)
@@ -1514,6 +1573,10 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   if (e != cudaSuccess) return cuda_fail(e, "assign: set smem");
   kern<<<grid, 64 + 128 * g.mt * cs, smem, s>>>(mA0, mA1, mB0, mB1, p);
   count_launch();
+  if (p.slices > 1) {
+    assign_merge_kernel<<<(unsigned)((N + 255) / 256), 256, 0, s>>>(p);
+    count_launch();
+  }
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "assign kernel launch");
   return HME_OK;
@@ -1545,6 +1608,8 @@ int launch_assign_split(const float *X, int64_t N, int64_t ldx, const AssignGeom
   p.num_kb = (g.d + kBK - 1) / kBK;
   p.BN = g.BN;
   p.nchunks = 1;
+  p.slices = 1;
+  p.cps = 1;
   p.write_split = xhi_out ? 1 : 0;
   p.xn_out = xn_out;
   p.z_out = out.z;

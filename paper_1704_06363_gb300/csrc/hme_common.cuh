@@ -39,6 +39,10 @@ constexpr int kBM = 128;        // rows per assign tile (tcgen05 M)
 constexpr int kBK = 64;         // bf16 elements per stage k-block (one 128-byte swizzle row)
 constexpr int kMaxBN = 256;     // centres per tcgen05 N-chunk
 constexpr int kMaxK = 16384;
+// small batches: at most kSplitRows rows (the row tiles of one wave) spread
+// their N-chunks over at most kMaxSlices CTAs each
+constexpr int64_t kSplitRows = 152 * 128;
+constexpr int kMaxSlices = 16;
 constexpr int kMaxD = 16384;
 
 // ---------------------------------------------------------------------------
@@ -84,6 +88,7 @@ struct Layout {
   size_t flagged;   // int32[3N]: near-tie rows queued with their two candidates
   size_t full_rows; // int32[N]: near-tie rows queued for all K centres
   size_t perm, slab;  // int32[N] each: sorted order of the labels (update)
+  size_t split;     // float4[min(N, kSplitRows) * kMaxSlices]: row states of centre slices (small batches)
   PartLayout part;  // partition scratch (update / route)
   size_t sums;      // f64[K * d]: per-cluster sums (kept between centre updates)
   size_t counts;    // i64[K]: per-cluster counts (kept between centre updates)
@@ -118,9 +123,11 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
 // features, three products) or unused.
 cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, void *chi, __nv_bfloat16 *clo, float *cn,
                                 Header *hdr, cudaStream_t s);
+// part: scratch of small batches (the Layout's split region), or NULL.
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g,
                   const void *chi, const __nv_bfloat16 *clo, const float *cn, const float *xn,
-                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, cudaStream_t s);
+                  int32_t *labels, float *mind, Header *hdr, int32_t *flagged, int32_t *full_rows, float4 *part,
+                  cudaStream_t s);
 // fp32 features with one N-chunk, split to bf16 hi/lo inside the kernel (no
 // preparation pass); eligible when X is 16-byte aligned and ldx % 4 == 0.
 // Optional outputs: with xhi/xlo/xn set (all or none) the kernel also writes

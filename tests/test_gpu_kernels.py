@@ -129,6 +129,37 @@ def test_assign_parity_several_tiles_per_cta(dev, dtype, d, K, prepared, bmt):
     assert st["mismatches"] <= st["near_ties"]
 
 
+# Batches of at most one wave of row tiles spread each tile's centre chunks
+# over several CTAs, whose per-row states a second kernel merges.
+#   N, d, K, dtype: what the launch does (tiles of 128 rows; 256 for MT = 2)
+SLICE_CASES = [
+    (256, 256, 4096, "bf16"),   # 2 tiles x 16 slices of one 256-centre chunk
+    (256, 256, 4096, "f32"),    # three split products, 16 slices
+    (5000, 64, 1100, "bf16"),   # 40 tiles x 3 slices of 2, 2 and 1 chunks (ragged)
+    (3000, 512, 1024, "bf16"),  # rows streamed, two row tiles per centre stage: 12 tiles x 4 slices
+    (9728, 96, 600, "f32"),     # the most tiles that slice: 76 tiles x 2 slices
+    (1, 40, 16384, "bf16"),     # one row against the most centres: 16 slices of 8 chunks
+]
+
+
+@pytest.mark.parametrize("N,d,K,dtype", SLICE_CASES, ids=lambda v: str(v))
+def test_small_batch_slices_the_centres(dev, N, d, K, dtype):
+    """Near ties between centres of different slices (a copy of each data
+    centre 1e-5 away, K/2 columns further on) and exact duplicates (the lowest
+    index wins) come out of the slice merge as the oracle has them."""
+    X = _mixture(N, d, min(K, 64), dtype, seed=N + K)
+    C = hme_synth.random_centroids(K, d, seed=K + 5, scale=3.0)
+    m = min(N, K // 4)
+    C[:m] = X[:m].float()
+    g = torch.Generator().manual_seed(N)
+    C[K // 2:K // 2 + m] = C[:m] + 1e-5 * torch.randn(m, d, generator=g)
+    C[K - 1] = C[0]  # exact duplicate of centre 0 in the last slice
+    lab, md, obj = _assign(X, C, dev)
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab, md, obj)
+    assert st["mismatches"] <= st["near_ties"]
+    assert lab[0] == 0  # row 0 sits on centre 0 and on its duplicate K - 1
+
+
 # HME_ASSIGN_TF32: fp32 features multiplied as tf32 operands (K > 256, rows TMA
 # can read); near ties are re-scored on their two candidates, or on all K when
 # a third centre is close too.  N, d, K, rows per CTA tile (0: a few tiles)
