@@ -52,6 +52,7 @@ constexpr int kSWarps = kSThreads / 32;
 constexpr int kSR = kPartChunk / kSThreads;   // items per scatter thread per chunk
 constexpr int kMaxDigitBits = HME_PART_MAXB;
 constexpr int kPartTilesPerSM = 2;
+constexpr int kPartWideK = 2048;             // from this K on, one tile per SM
 constexpr int kPartSMs = 152;                 // GB300: the tile count fills two CTAs per SM
 constexpr size_t kMaxSmemScatter = 227 * 1024;
 static_assert(kPartChunk % kSThreads == 0 && kPartChunk <= 65536, "chunk positions fit 16 bits");
@@ -600,38 +601,49 @@ using ScatterFn = void (*)(const int32_t *, int64_t, int, int64_t, const int32_t
                            TagArgs);
 
 // sorted_labels[s] = the bucket of slot s (offsets[k] <= s < offsets[k+1]),
-// for s < offsets[K]: every thread fills 16 consecutive slots, finding the
-// bucket of its first slot by binary search and stepping over the buckets
-// that end inside its slots; 16-byte stores.
+// for s < offsets[K]: every thread finds the buckets of 16 consecutive slots
+// (a binary search for the first, then a walk over the buckets that end
+// inside them) and leaves them in shared memory; the block then stores its
+// 4096 slots with consecutive threads on consecutive 16-byte words.
 constexpr int kFillSlots = 16;
-__global__ void part_fill_labels_kernel(const int64_t *__restrict__ offsets, int K, int64_t N,
-                                        int32_t *__restrict__ sorted_labels) {
-  const int64_t s0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * kFillSlots;
-  const int64_t n = __ldg(offsets + K);
-  if (s0 >= n || s0 >= N) return;
-  int lo = 0, hi = K - 1;  // the largest k with offsets[k] <= s0
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (__ldg(offsets + mid) <= s0)
-      lo = mid;
-    else
-      hi = mid - 1;
-  }
-  int k = lo;
-  int64_t next = __ldg(offsets + k + 1);
-  int32_t v[kFillSlots];
+constexpr int kFillThreads = 256;
+__global__ void __launch_bounds__(kFillThreads) part_fill_labels_kernel(const int64_t *__restrict__ offsets, int K,
+                                                                        int64_t N, int32_t *__restrict__ sorted_labels) {
+  __shared__ int32_t buf[kFillThreads * kFillSlots + kFillThreads];  // thread t's slots at t * 17
+  const int64_t n = min(N, __ldg(offsets + K));
+  const int64_t b0 = (int64_t)blockIdx.x * kFillThreads * kFillSlots;
+  const int64_t s0 = b0 + (int64_t)threadIdx.x * kFillSlots;
+  if (s0 < n) {
+    int lo = 0, hi = K - 1;  // the largest k with offsets[k] <= s0
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (__ldg(offsets + mid) <= s0)
+        lo = mid;
+      else
+        hi = mid - 1;
+    }
+    int k = lo;
+    int64_t next = __ldg(offsets + k + 1);
 #pragma unroll
-  for (int u = 0; u < kFillSlots; ++u) {
-    while (s0 + u >= next && k + 1 < K) next = __ldg(offsets + (++k) + 1);
-    v[u] = k;
+    for (int u = 0; u < kFillSlots; ++u) {
+      while (s0 + u >= next && k + 1 < K) next = __ldg(offsets + (++k) + 1);
+      buf[threadIdx.x * (kFillSlots + 1) + u] = k;
+    }
   }
-  const int64_t m = min((int64_t)kFillSlots, n - s0);
-  if (m == kFillSlots && (reinterpret_cast<uintptr_t>(sorted_labels + s0) & 15u) == 0) {
-    int4 *d = reinterpret_cast<int4 *>(sorted_labels + s0);
+  __syncthreads();
+  const int64_t m = min((int64_t)kFillThreads * kFillSlots, n - b0);  // slots of this block
+  if (m <= 0) return;
+  if (m == (int64_t)kFillThreads * kFillSlots && (reinterpret_cast<uintptr_t>(sorted_labels + b0) & 15u) == 0) {
 #pragma unroll
-    for (int u = 0; u < kFillSlots / 4; ++u) d[u] = make_int4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+    for (int u = 0; u < kFillSlots / 4; ++u) {
+      const int w = (u * kFillThreads + threadIdx.x) * 4;  // first of four slots
+      const int32_t *src = buf + (w / kFillSlots) * (kFillSlots + 1) + (w % kFillSlots);
+      reinterpret_cast<int4 *>(sorted_labels + b0)[u * kFillThreads + threadIdx.x] =
+          make_int4(src[0], src[1], src[2], src[3]);
+    }
   } else {
-    for (int u = 0; u < m; ++u) sorted_labels[s0 + u] = v[u];
+    for (int w = threadIdx.x; w < m; w += kFillThreads)
+      sorted_labels[b0 + w] = buf[(w / kFillSlots) * (kFillSlots + 1) + (w % kFillSlots)];
   }
 }
 
@@ -692,7 +704,11 @@ PartLayout part_layout(size_t base, int64_t N, int K, bool tags) {
   pl.b1 = b[1];
   pl.b2 = b[2];
   // two CTAs per SM; one with tag lists (whose scatter needs more registers)
-  const int64_t target = (tags ? 1 : kPartTilesPerSM) * kPartSMs;
+  // or with K >= 2048, where the ntiles x K partly written output lines of
+  // two tiles per SM no longer fit L2 (with labels spread over the buckets,
+  // runs are about one item long and every store would reach DRAM as a
+  // partial sector)
+  const int64_t target = (tags || K >= kPartWideK ? 1 : kPartTilesPerSM) * kPartSMs;
   int64_t tile = (N + target - 1) / target;
   tile = (tile + kPartChunk - 1) / kPartChunk * kPartChunk;
   if (tile < kPartChunk) tile = kPartChunk;
@@ -763,8 +779,8 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
     scatter<<<(unsigned)pl.ntiles, kSThreads, sms, s>>>(labels, N, K, pl.tile, tilecnt, offsets, perm, ta);
     count_launch();
     if (sorted_labels) {
-      const int64_t threads = (N + kFillSlots - 1) / kFillSlots;
-      part_fill_labels_kernel<<<(unsigned)((threads + 255) / 256), 256, 0, s>>>(offsets, K, N, sorted_labels);
+      const int64_t per = (int64_t)kFillThreads * kFillSlots;
+      part_fill_labels_kernel<<<(unsigned)((N + per - 1) / per), kFillThreads, 0, s>>>(offsets, K, N, sorted_labels);
       count_launch();
     }
   }

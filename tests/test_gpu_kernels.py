@@ -455,6 +455,48 @@ def test_partition_bit_exact(dev, N, K):
                                 sorted_labels=sl.cpu().numpy()), labels.numpy(), K)
 
 
+# Labels spread evenly over K buckets (the shape of converged K-means labels,
+# unlike the Zipf draws above), several sort chunks per tile, one and two
+# tiles per SM (K from 2048 on: one), every digit-pass split up to K = 16384.
+UNIFORM_PART_CASES = [(2_000_000, 300), (1_000_001, 600), (1_500_000, 2048), (3_000_000, 4096), (1_500_000, 5000),
+                      (777_777, 8192), (1_300_000, 16384)]
+
+
+@pytest.mark.parametrize("N,K", UNIFORM_PART_CASES, ids=lambda v: str(v))
+def test_partition_uniform_labels(dev, N, K):
+    g = torch.Generator().manual_seed(N ^ K)
+    labels = torch.randint(0, K, (N,), generator=g, dtype=torch.int32)
+    ws = hme.workspace(hme.HME_OP_PARTITION, N, 1, K, hme.HME_F32, device=dev)
+    hist = torch.empty(K, dtype=torch.int64, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    perm = torch.empty(N, dtype=torch.int32, device=dev)
+    sl = torch.empty(N, dtype=torch.int32, device=dev)
+    hme.hme_partition(labels.to(dev), K, hist, offs, perm, ws, sl)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    parity.check_partition(dict(hist=hist.cpu().numpy(), offsets=offs.cpu().numpy(), perm=perm.cpu().numpy(),
+                                sorted_labels=sl.cpu().numpy()), labels.numpy(), K)
+
+
+def test_partition_many_buckets_drops_bad_labels(dev):
+    """Labels outside [0, K) are counted nowhere, reported, and left out of
+    the order; the valid ones keep their stable order."""
+    N, K = 600_000, 1000
+    g = torch.Generator().manual_seed(7)
+    labels = torch.randint(-3, K + 3, (N,), generator=g, dtype=torch.int32)
+    ws = hme.workspace(hme.HME_OP_PARTITION, N, 1, K, hme.HME_F32, device=dev)
+    hist = torch.empty(K, dtype=torch.int64, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    perm = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    hme.hme_partition(labels.to(dev), K, hist, offs, perm, ws)
+    assert hme.hme_sync_status(ws) == hme.HME_EINVAL
+    lab = labels.numpy()
+    ok = (lab >= 0) & (lab < K)
+    assert np.array_equal(hist.cpu().numpy(), np.bincount(lab[ok], minlength=K))
+    nv = int(ok.sum())
+    ref = np.nonzero(ok)[0][np.argsort(lab[ok], kind="stable")]
+    assert np.array_equal(perm.cpu().numpy()[:nv], ref)
+
+
 def test_partition_tags_and_misaligned_labels(dev):
     N, K = 20001, 33
     w = hme_synth.WORKLOADS[4].with_rows(N)
