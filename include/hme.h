@@ -275,6 +275,12 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
  * when ws already holds Q prepared by hme_prepare_features or a PREPARE_OUT
  * call (e.g. routing the training set with the workspace of the Lloyd loop:
  * HME_OP_ROUTE and HME_OP_ASSIGN sizes agree).
+ * Batches of at most 16384 rows: from the second call with the same
+ * arguments (every pointer, size and flag, and the stream) on, the call's
+ * launches are replayed as one CUDA graph captured at that second call (the
+ * data behind the pointers may change freely between calls; it is read when
+ * the graph runs).  Up to 8 argument sets are kept, the least recently used
+ * replaced.  The environment variable HME_NO_GRAPHS=1 turns this off.
  * Errors: HME_EINVAL for sizes outside the limits, a NULL or misaligned Q, a
  * NULL C or offsets_out, a NULL expert_out / order_out with B > 0, unknown or
  * conflicting flags; HME_ENOMEM for a workspace smaller than

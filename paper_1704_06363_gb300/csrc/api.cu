@@ -5,6 +5,7 @@
 #include "hme_common.cuh"
 
 #include <atomic>
+#include <mutex>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -367,6 +368,125 @@ int check_pca(const void *X, int64_t N, int d, int64_t ldx, int dtype, int r, in
 }
 
 }  // namespace
+// Small routed batches are launch-bound (a dozen kernels of a few
+// microseconds each).  A route of at most kGraphRows rows whose arguments --
+// every pointer, size, flag and the stream -- repeat those of an earlier call
+// is captured once as a CUDA graph (on a stream of the library's own, so that
+// any stream of the caller's, the legacy default one included, can replay it)
+// and from then on replayed with one launch.  The captured launches depend on
+// the arguments only, never on the data, which the kernels read when they
+// run.  The first call with a given set of arguments runs directly (a batch
+// routed once pays no capture); a capture that fails leaves that set direct.
+constexpr int64_t kGraphRows = 16384;
+constexpr int kGraphSlots = 8;
+struct RouteKey {
+  const void *Q;
+  int64_t B;
+  int32_t d;
+  int64_t ldq;
+  int32_t dtype;
+  const float *C;
+  int32_t K;
+  int32_t flags;
+  int32_t *expert;
+  int64_t *offsets;
+  int32_t *order;
+  void *ws;
+  size_t ws_bytes;
+  void *stream;
+  int device = 0;
+  bool operator==(const RouteKey &o) const {
+    return Q == o.Q && B == o.B && d == o.d && ldq == o.ldq && dtype == o.dtype && C == o.C && K == o.K &&
+           flags == o.flags && expert == o.expert && offsets == o.offsets && order == o.order && ws == o.ws &&
+           ws_bytes == o.ws_bytes && stream == o.stream && device == o.device;
+  }
+};
+struct RouteGraph {
+  RouteKey key{};
+  bool used = false;
+  bool direct = false;  // capture failed: stay direct
+  cudaGraphExec_t exec = nullptr;
+  int64_t launches = 0;
+  uint64_t stamp = 0;
+};
+std::mutex g_rg_mu;
+RouteGraph g_rg[kGraphSlots];
+uint64_t g_rg_clock = 0;
+cudaStream_t g_cap_stream[64] = {};
+
+template <typename Body>
+int graph_route(RouteKey key, Body &&body, cudaStream_t s) {
+  static const bool off = [] {
+    const char *e = getenv("HME_NO_GRAPHS");
+    return e && *e && *e != '0';
+  }();
+  if (off || cudaGetDevice(&key.device) != cudaSuccess || key.device < 0 || key.device >= 64) return body(s);
+  std::unique_lock<std::mutex> lk(g_rg_mu);
+  RouteGraph *slot = nullptr;
+  for (auto &g : g_rg)
+    if (g.used && g.key == key) slot = &g;
+  if (slot && slot->exec) {
+    slot->stamp = ++g_rg_clock;
+    const cudaGraphExec_t exec = slot->exec;
+    const int64_t n = slot->launches;
+    lk.unlock();
+    HME_CUDA(cudaGraphLaunch(exec, s), "route: graph launch");
+    count_launch((int)n);
+    return HME_OK;
+  }
+  if (!slot) {  // first sighting: remember the arguments, run directly
+    RouteGraph *victim = &g_rg[0];
+    for (auto &g : g_rg)
+      if (!g.used || g.stamp < victim->stamp) victim = &g;
+    if (victim->exec) cudaGraphExecDestroy(victim->exec);
+    *victim = RouteGraph{};
+    victim->key = key;
+    victim->used = true;
+    victim->stamp = ++g_rg_clock;
+    lk.unlock();
+    return body(s);
+  }
+  if (slot->direct) {
+    lk.unlock();
+    return body(s);
+  }
+  // second sighting: capture on the library's stream, then replay on s
+  cudaStream_t &cs = g_cap_stream[key.device];
+  if (!cs && cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+    cs = nullptr;
+    slot->direct = true;
+    lk.unlock();
+    return body(s);
+  }
+  const int64_t before = g_launches.load();
+  cudaGraph_t graph = nullptr;
+  int rc = HME_OK;
+  if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
+    rc = body(cs);
+    const cudaError_t e = cudaStreamEndCapture(cs, &graph);
+    if (e != cudaSuccess && graph) {
+      cudaGraphDestroy(graph);
+      graph = nullptr;
+    }
+  }
+  cudaGraphExec_t exec = nullptr;
+  if (rc == HME_OK && graph && cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) exec = nullptr;
+  if (graph) cudaGraphDestroy(graph);
+  cudaGetLastError();  // a failed capture leaves no sticky error behind
+  if (!exec) {
+    slot->direct = true;
+    g_launches.fetch_sub(g_launches.load() - before);  // nothing captured ran
+    lk.unlock();
+    return rc == HME_OK ? body(s) : rc;
+  }
+  slot->exec = exec;
+  slot->launches = g_launches.load() - before;
+  slot->stamp = ++g_rg_clock;
+  lk.unlock();
+  HME_CUDA(cudaGraphLaunch(exec, s), "route: graph launch");
+  return HME_OK;
+}
+
 }  // namespace hme
 
 using namespace hme;
@@ -579,12 +699,19 @@ int hme_route(const void *Q, int64_t B, int32_t d, int64_t ldq, int32_t dtype, c
   const Layout L = feature_layout(B, d, K, dtype, 0);
   HME_TRY(check_ws(ws, ws_bytes, L.total));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  HME_TRY(clear_header(ws, s));
-  HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, flags, s));
-  HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
-                            offsets_out, order_out, nullptr, at<Header>(ws, 0), s),
-           "route: partition");
-  return HME_OK;
+  auto body = [&](cudaStream_t cs) -> int {
+    HME_TRY(clear_header(ws, cs));
+    HME_TRY(do_assign(Q, B, d, ldq, dtype, C, K, expert_out, nullptr, L, ws, flags, cs));
+    HME_CUDA(launch_partition(expert_out, B, K, L.part, static_cast<char *>(ws), at<int64_t>(ws, L.part.hist),
+                              offsets_out, order_out, nullptr, at<Header>(ws, 0), cs),
+             "route: partition");
+    return HME_OK;
+  };
+  if (B > 0 && B <= kGraphRows) {
+    const RouteKey key{Q, B, d, ldq, dtype, C, K, flags, expert_out, offsets_out, order_out, ws, ws_bytes, stream};
+    return graph_route(key, body, s);
+  }
+  return body(s);
 }
 
 int hme_tag_cluster_hist(const int64_t *offsets, const int64_t *tag_off, const int32_t *tags, int64_t N, int32_t K,

@@ -647,26 +647,37 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
 }
 
 // Small batches: the row states of the centre slices (lean scan: best value,
-// runner-up value, best's index) merged per row, then the row finished as in
+// runner-up value, best's index) merged per row -- a group of kMaxSlices lanes
+// per row, one slice each, merged by shuffles -- then the row finished as in
 // the assign kernel (label, distance, near-tie queue, objective).
+constexpr int kMergeRows = 256 / kMaxSlices;  // rows per block
 __global__ void __launch_bounds__(256) assign_merge_kernel(const AssignParams p) {
+  static_assert(kMaxSlices <= 32 && (32 % kMaxSlices) == 0, "a row's slices fit one warp");
   const float cn_max = __uint_as_float(*((volatile uint32_t *)&p.hdr->cn_max_bits));
   const float sqrt_cn_max = sqrtf(cn_max);
-  double obj = 0.0;
-  for (int64_t row = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; row < p.N;
-       row += (int64_t)gridDim.x * blockDim.x) {
-    float best1 = INFINITY, best2 = INFINITY;
-    int idx1 = 0;
-    for (int sl = 0; sl < p.slices; ++sl) {
-      const float4 v = p.part[row * p.slices + sl];
-      const int i = __float_as_int(v.z);
-      const bool take = v.x < best1 || (v.x == best1 && i < idx1);
-      best2 = fminf(fmaxf(best1, v.x), fminf(best2, v.y));
-      best1 = take ? v.x : best1;
-      idx1 = take ? i : idx1;
-    }
-    obj += finish_row<true>(p, row, __ldg(p.xn + row), best1, best2, INFINITY, idx1, 0, cn_max, sqrt_cn_max);
+  const int g = threadIdx.x % kMaxSlices;  // slice of this lane
+  const int64_t row = (int64_t)blockIdx.x * kMergeRows + threadIdx.x / kMaxSlices;
+  float best1 = INFINITY, best2 = INFINITY;
+  int idx1 = 0x7fffffff;
+  if (row < p.N && g < p.slices) {
+    const float4 v = p.part[row * p.slices + g];
+    best1 = v.x;
+    best2 = v.y;
+    idx1 = __float_as_int(v.z);
   }
+#pragma unroll
+  for (int o = kMaxSlices / 2; o > 0; o >>= 1) {
+    const float o1 = __shfl_xor_sync(0xffffffffu, best1, o);
+    const float o2 = __shfl_xor_sync(0xffffffffu, best2, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, idx1, o);
+    const bool take = o1 < best1 || (o1 == best1 && oi < idx1);
+    best2 = fminf(fmaxf(best1, o1), fminf(best2, o2));
+    best1 = take ? o1 : best1;
+    idx1 = take ? oi : idx1;
+  }
+  double obj = 0.0;
+  if (g == 0 && row < p.N)
+    obj = finish_row<true>(p, row, __ldg(p.xn + row), best1, best2, INFINITY, idx1, 0, cn_max, sqrt_cn_max);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
   if ((threadIdx.x & 31) == 0 && obj != 0.0) atomicAdd(&p.hdr->objective, obj);
@@ -1574,7 +1585,7 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   kern<<<grid, 64 + 128 * g.mt * cs, smem, s>>>(mA0, mA1, mB0, mB1, p);
   count_launch();
   if (p.slices > 1) {
-    assign_merge_kernel<<<(unsigned)((N + 255) / 256), 256, 0, s>>>(p);
+    assign_merge_kernel<<<(unsigned)((N + kMergeRows - 1) / kMergeRows), 256, 0, s>>>(p);
     count_launch();
   }
   e = cudaGetLastError();
@@ -1676,6 +1687,9 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
                            const int32_t *full_rows, cudaStream_t s) {
   if (N == 0) return cudaSuccess;
   const int grid = num_sms() * 4;
+  // the queues hold at most N rows: a warp per queued pair, a thread per finished row
+  const int gpair = (int)std::min<int64_t>(grid, (N + 7) / 8);
+  const int gfin = (int)std::min<int64_t>(grid, (N + 255) / 256);
   const bool al = ((reinterpret_cast<uintptr_t>(X) | reinterpret_cast<uintptr_t>(C)) & 15u) == 0;
   // all-K rows: block per row for few centres (low latency), tiled otherwise
   const bool row_path = K <= 128;
@@ -1693,18 +1707,18 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
   }
   if (dtype == HME_BF16) {
     if (al && d % 8 == 0 && ldx % 8 == 0)
-      rescore_pair_kernel<HME_BF16, 8><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
+      rescore_pair_kernel<HME_BF16, 8><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     else
-      rescore_pair_kernel<HME_BF16, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
+      rescore_pair_kernel<HME_BF16, 1><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     if (row_path)
       rescore_row_kernel<HME_BF16, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else
       rescore_full_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   } else {
     if (al && d % 4 == 0 && ldx % 4 == 0)
-      rescore_pair_kernel<HME_F32, 4><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
+      rescore_pair_kernel<HME_F32, 4><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     else
-      rescore_pair_kernel<HME_F32, 1><<<grid, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
+      rescore_pair_kernel<HME_F32, 1><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     if (row_path && cvec)
       rescore_row_kernel<HME_F32, 4><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else if (row_path)
@@ -1712,7 +1726,7 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
     else
       rescore_full_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   }
-  if (!row_path) rescore_full_finish_kernel<<<grid, 256, 0, s>>>(labels, mind, hdr, full_rows, keys_end);
+  if (!row_path) rescore_full_finish_kernel<<<gfin, 256, 0, s>>>(labels, mind, hdr, full_rows, keys_end);
   count_launch(row_path ? 2 : 3);
   return cudaGetLastError();
 }

@@ -354,7 +354,8 @@ template <int B0, int B1, int B2, bool TAGS>
 __global__ void __launch_bounds__(kSThreads, TAGS ? 1 : kPartTilesPerSM)
     part_scatter_kernel(const int32_t *__restrict__ labels, int64_t N, int K, int64_t tile,
                         const int32_t *__restrict__ tileoff, const int64_t *__restrict__ offsets,
-                        int32_t *__restrict__ perm_out, TagArgs ta) {
+                        int32_t *__restrict__ perm_out, TagArgs ta, int64_t *__restrict__ fz_hist,
+                        int64_t *__restrict__ fz_offs, Header *hdr) {
   constexpr int BMAX = B0 > B1 ? (B0 > B2 ? B0 : B2) : (B1 > B2 ? B1 : B2);
   extern __shared__ uint32_t psm[];
   int32_t *cursor = reinterpret_cast<int32_t *>(psm);
@@ -369,7 +370,57 @@ __global__ void __launch_bounds__(kSThreads, TAGS ? 1 : kPartTilesPerSM)
   int64_t *dsts = toff + kPartChunk + 2;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t t = blockIdx.x;
-  for (int k = threadIdx.x; k < K; k += kSThreads) cursor[k] = (int32_t)(offsets[k] + tileoff[t * K + k]);
+  if (fz_offs) {
+    // one tile holds every item (no TAGS): count it here, and the exclusive
+    // prefix of the counts is both offsets and the cursors
+    for (int k = threadIdx.x; k < K; k += kSThreads) cursor[k] = 0;
+    __syncthreads();
+    bool bad = false;
+    for (int64_t i = threadIdx.x; i < N; i += kSThreads) {
+      const int v = __ldg(labels + i);
+      if (v >= 0 && v < K)
+        atomicAdd(&cursor[v], 1);
+      else
+        bad = true;
+    }
+    if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadLabel);
+    __syncthreads();
+    const int per = (K + kSThreads - 1) / kSThreads;
+    const int k0 = min(K, (int)threadIdx.x * per), k1 = min(K, k0 + per);
+    int32_t loc = 0;
+    for (int k = k0; k < k1; ++k) loc += cursor[k];
+    int32_t incl = loc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t x = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += x;
+    }
+    if (lane == 31) wsum[warp] = (uint32_t)incl;
+    __syncthreads();
+    if (warp == 0) {
+      const int32_t x0 = lane < kSWarps ? (int32_t)wsum[lane] : 0;
+      int32_t xi = x0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int32_t x = __shfl_up_sync(0xffffffffu, xi, o);
+        if (lane >= o) xi += x;
+      }
+      if (lane < kSWarps) wsum[lane] = (uint32_t)(xi - x0);
+    }
+    __syncthreads();
+    int32_t run = (int32_t)wsum[warp] + incl - loc;
+    for (int k = k0; k < k1; ++k) {
+      const int32_t c = cursor[k];
+      fz_hist[k] = c;
+      fz_offs[k] = run;
+      cursor[k] = run;
+      run += c;
+    }
+    if (threadIdx.x == kSThreads - 1) fz_offs[K] = run;
+    __syncthreads();
+  } else {
+    for (int k = threadIdx.x; k < K; k += kSThreads) cursor[k] = (int32_t)(offsets[k] + tileoff[t * K + k]);
+  }
   int64_t *tcur = nullptr;
   if (TAGS) {
     tcur = ta.tcur_smem ? dsts + kPartChunk : ta.tagcur + t * K;
@@ -598,7 +649,7 @@ __global__ void part_tag_tail_kernel(const int64_t *__restrict__ offsets, int K,
 }
 
 using ScatterFn = void (*)(const int32_t *, int64_t, int, int64_t, const int32_t *, const int64_t *, int32_t *,
-                           TagArgs);
+                           TagArgs, int64_t *, int64_t *, Header *);
 
 // sorted_labels[s] = the bucket of slot s (offsets[k] <= s < offsets[k+1]),
 // for s < offsets[K]: every thread finds the buckets of 16 consecutive slots
@@ -760,14 +811,18 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
     e = cudaFuncSetAttribute(scatter, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sms);
     if (e != cudaSuccess) return e;
   }
-  if (pl.ntiles > 0) {
+  // a single tile without tag lists: the scatter CTA counts and scans itself
+  const bool fused = !tags && pl.ntiles == 1;
+  if (pl.ntiles > 0 && !fused) {
     count<<<(unsigned)pl.ntiles, kPThreads, smc, s>>>(labels, N, K, pl.tile, tilecnt, tags ? tl->tag_off : nullptr,
                                                       tagcnt, hdr);
     count_launch();
   }
-  part_colscan_kernel<int32_t><<<(K + 31) / 32, 1024, 0, s>>>(tilecnt, pl.ntiles, K, hist);
-  part_offsets_kernel<<<1, 1024, 0, s>>>(hist, K, offsets);
-  count_launch(2);
+  if (!fused) {
+    part_colscan_kernel<int32_t><<<(K + 31) / 32, 1024, 0, s>>>(tilecnt, pl.ntiles, K, hist);
+    part_offsets_kernel<<<1, 1024, 0, s>>>(hist, K, offsets);
+    count_launch(2);
+  }
   if (tags) {
     part_colscan_kernel<int64_t><<<(K + 31) / 32, 1024, 0, s>>>(tagcnt, pl.ntiles, K, tag_hist);
     part_offsets_kernel<<<1, 1024, 0, s>>>(tag_hist, K, tag_base);
@@ -776,7 +831,8 @@ cudaError_t launch_partition(const int32_t *labels, int64_t N, int K, const Part
   if (pl.ntiles > 0) {
     TagArgs ta{};
     if (tags) ta = TagArgs{tl->tag_off, tl->tags, tagcnt, tag_base, tl->tag_off_out, tl->tags_out, tcur_smem ? 1 : 0};
-    scatter<<<(unsigned)pl.ntiles, kSThreads, sms, s>>>(labels, N, K, pl.tile, tilecnt, offsets, perm, ta);
+    scatter<<<(unsigned)pl.ntiles, kSThreads, sms, s>>>(labels, N, K, pl.tile, fused ? nullptr : tilecnt, offsets,
+                                                        perm, ta, fused ? hist : nullptr, fused ? offsets : nullptr, hdr);
     count_launch();
     if (sorted_labels) {
       const int64_t per = (int64_t)kFillThreads * kFillSlots;

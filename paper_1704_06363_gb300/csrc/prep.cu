@@ -179,42 +179,47 @@ __global__ void __launch_bounds__(kPrepCThreads) prep_centres_kernel(const float
                                                                      void *__restrict__ chi_raw,
                                                                      __nv_bfloat16 *__restrict__ clo,
                                                                      float *__restrict__ cn, Header *hdr) {
+  // one warp per centre; the block's largest norm goes to cn_max once
   __nv_bfloat16 *chi = static_cast<__nv_bfloat16 *>(chi_raw);
   float *ct = static_cast<float *>(chi_raw);
-  __shared__ float part[kPrepCThreads / 32];
-  const int k = blockIdx.x;
-  if (k >= K) {
-    if (threadIdx.x == 0) cn[k] = INFINITY;
-    return;
-  }
-  float s = 0.0f;
-#pragma unroll 4
-  for (int j = threadIdx.x; j < d; j += kPrepCThreads) {
-    const float c = __ldg(C + (int64_t)k * d + j);
-    float ce;
-    if (tf32) {
-      ct[(int64_t)k * ldp + j] = round_tf32(c);
-      ce = c;
-    } else if (nprod == 1) {
-      const __nv_bfloat16 b = __float2bfloat16_rn(c);
-      chi[(int64_t)k * ldp + j] = b;
-      ce = __bfloat162float(b);
-    } else {
-      __nv_bfloat16 h, l;
-      split_bf16(c, h, l);
-      chi[(int64_t)k * ldp + j] = h;
-      clo[(int64_t)k * ldp + j] = l;
-      ce = __bfloat162float(h) + __bfloat162float(l);  // exact in fp32
+  __shared__ float wmax[kPrepCThreads / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float bmax = 0.0f;
+  for (int k = blockIdx.x * (kPrepCThreads / 32) + warp; k < Kp; k += gridDim.x * (kPrepCThreads / 32)) {
+    if (k >= K) {
+      if (lane == 0) cn[k] = INFINITY;
+      continue;
     }
-    s = fmaf(ce, ce, s);
+    float s = 0.0f;
+#pragma unroll 4
+    for (int j = lane; j < d; j += 32) {
+      const float c = __ldg(C + (int64_t)k * d + j);
+      float ce;
+      if (tf32) {
+        ct[(int64_t)k * ldp + j] = round_tf32(c);
+        ce = c;
+      } else if (nprod == 1) {
+        const __nv_bfloat16 bv = __float2bfloat16_rn(c);
+        chi[(int64_t)k * ldp + j] = bv;
+        ce = __bfloat162float(bv);
+      } else {
+        __nv_bfloat16 h, l;
+        split_bf16(c, h, l);
+        chi[(int64_t)k * ldp + j] = h;
+        clo[(int64_t)k * ldp + j] = l;
+        ce = __bfloat162float(h) + __bfloat162float(l);  // exact in fp32
+      }
+      s = fmaf(ce, ce, s);
+    }
+    s = warp_sum(s);
+    if (lane == 0) cn[k] = s;
+    bmax = fmaxf(bmax, s);
   }
-  s = warp_sum(s);
-  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = s;
+  if (lane == 0) wmax[warp] = bmax;
   __syncthreads();
   if (threadIdx.x == 0) {
     float t = 0.0f;
-    for (int w = 0; w < kPrepCThreads / 32; ++w) t += part[w];
-    cn[k] = t;
+    for (int w = 0; w < kPrepCThreads / 32; ++w) t = fmaxf(t, wmax[w]);
     atomicMax(&hdr->cn_max_bits, __float_as_uint(t));  // t >= 0: integer order is float order
   }
 }
@@ -247,7 +252,9 @@ cudaError_t launch_prep_features(const void *X, int64_t N, int d, int64_t ldx, i
 
 cudaError_t launch_prep_centres(const float *C, const AssignGeom &g, void *chi, __nv_bfloat16 *clo, float *cn,
                                 Header *hdr, cudaStream_t s) {
-  prep_centres_kernel<<<g.Kp, kPrepCThreads, 0, s>>>(C, g.K, g.Kp, g.d, g.ldc, g.nprod, g.tf32, chi, clo, cn, hdr);
+  const int per = kPrepCThreads / 32;  // centres per block and pass
+  const int blocks = std::min((g.Kp + per - 1) / per, num_sms() * 4);
+  prep_centres_kernel<<<blocks, kPrepCThreads, 0, s>>>(C, g.K, g.Kp, g.d, g.ldc, g.nprod, g.tf32, chi, clo, cn, hdr);
   count_launch();
   return cudaGetLastError();
 }

@@ -548,6 +548,32 @@ def test_route_parity(dev, dtype):
     parity.check_partition(dict(offsets=offs.cpu().numpy(), perm=order.cpu().numpy()), e, K)
 
 
+def test_route_replayed_graph_reads_fresh_data(dev):
+    """Repeated small routes with the same arguments replay a captured graph:
+    the third and fourth calls, on new batch contents and new centres at the
+    same addresses, route them exactly as a first call does."""
+    B, d, K = 256, 256, 4096
+    ws = hme.workspace(hme.HME_OP_ROUTE, B, d, K, hme.HME_BF16, device=dev)
+    Q = torch.empty(B, d, dtype=torch.bfloat16, device=dev)
+    C = torch.empty(K, d, dtype=torch.float32, device=dev)
+    expert = torch.empty(B, dtype=torch.int32, device=dev)
+    offs = torch.empty(K + 1, dtype=torch.int64, device=dev)
+    order = torch.empty(B, dtype=torch.int32, device=dev)
+    for call in range(4):
+        Qh = _mixture(B, d, 16, "bf16", seed=100 + call)
+        Ch = hme_synth.random_centroids(K, d, seed=200 + call, scale=3.0)
+        Ch[:B // 2] = Qh[:B // 2].float()
+        Q.copy_(Qh)
+        C.copy_(Ch)
+        before = hme.hme_launch_count()
+        hme.hme_route(Q, C, expert, offs, order, ws)
+        assert hme.hme_sync_status(ws) == hme.HME_OK
+        assert hme.hme_launch_count() > before  # replays count their kernels too
+        e = expert.cpu().numpy()
+        parity.check_assign(_host(Qh, "bf16"), "bf16", Ch.numpy(), e)
+        parity.check_partition(dict(offsets=offs.cpu().numpy(), perm=order.cpu().numpy()), e, K)
+
+
 @pytest.mark.parametrize("N,d,K,dtype,method", [
     (10000, 128, 16, "f32", hme.HME_INIT_KMEANSPP),
     (3000, 64, 9, "bf16", hme.HME_INIT_KMEANSPP),
