@@ -251,8 +251,10 @@ __device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row,
 //          shared memory, behind two bounded mbarriers), which merges them and
 //          writes the row's result
 //   TF32   fp32 operands read as tf32 (kind::tf32; k-blocks of 32 elements)
+//   T3     (not LEAN) the top-three scan over several N-chunks: a near tie
+//          with exactly two candidates is re-scored on those two only
 // Threads: warp 0 TMA, warp 1 MMA, 4*MT*CS epilogue warps.
-template <int NPROD, bool LEAN, int MT, bool ARES, int CS, bool TF32 = false>
+template <int NPROD, bool LEAN, int MT, bool ARES, int CS, bool TF32 = false, bool T3 = TF32>
 __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
     assign_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
                   const __grid_constant__ CUtensorMap tmB0, const __grid_constant__ CUtensorMap tmB1,
@@ -534,7 +536,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           if (more1) tmem_ld16(taddr + (uint32_t)(c + 16), rb);
           if (LEAN)
             lean_group(ra, cbc, kbase + c, best1, best2, idx1);
-          else if (TF32)
+          else if (T3)
             top3_group(ra, cbc, kbase + c, best1, best2, best3, idx1, idx2);
           else
             epilogue_group(ra, cbc, kbase + c, best1, best2, best3, idx1, idx2);
@@ -543,7 +545,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             if (more2) tmem_ld16(taddr + (uint32_t)(c + 32), ra);
             if (LEAN)
               lean_group(rb, cbc + 16, kbase + c + 16, lb1, lb2, li1);
-            else if (TF32)
+            else if (T3)
               top3_group(rb, cbc + 16, kbase + c + 16, lb1, lb2, lb3, li1, li2);
             else
               epilogue_group(rb, cbc + 16, kbase + c + 16, best1, best2, best3, idx1, idx2);
@@ -560,7 +562,7 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
         best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
         best1 = take_b ? lb1 : best1;
         idx1 = take_b ? li1 : idx1;
-      } else if (TF32) {  // merge the two top-three states
+      } else if (T3) {  // merge the two top-three states
         insert_top3(lb1, li1, best1, best2, best3, idx1, idx2);
         insert_top3(lb2, li2, best1, best2, best3, idx1, idx2);
         best3 = fminf(best3, lb3);
@@ -1572,10 +1574,20 @@ int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const 
   cudaError_t e;
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const CUtensorMap, const AssignParams);
   Kern kern;
+  // Several N-chunks of the three-product split: the top-three scan, so that
+  // near ties with two candidates are re-scored on those two (the split is
+  // bound by its MMAs, and the wider scan cuts the all-K re-scores about a
+  // hundredfold: 1.6e7 x 512, K = 1024 features, 8.8 -> 7.6 ms for 4e6 rows).
+  // bf16 features keep the lean scan: their kernel is bound by the epilogue,
+  // where the top-three scan cost half as much again (5e7 x 256, K = 4096
+  // features: 14.2 -> 21.3 ms for 8e6 rows) as the all-K re-scores it saves.
+  // Centre slices always use the lean states the merge kernel combines.
+  const bool top3 = lean && p.slices == 1 && g.nprod == 3;
   if (g.tf32)
     kern = assign_kernel<1, false, 2, false, 2, true>;  // top-three scan: two-candidate near ties re-scored cheaply
   else if (g.nprod == 3)
-    kern = lean ? assign_kernel<3, true, 1, false, 1> : assign_kernel<3, false, 1, false, 1>;
+    kern = top3 ? assign_kernel<3, false, 1, false, 1, false, true>
+                : (lean ? assign_kernel<3, true, 1, false, 1> : assign_kernel<3, false, 1, false, 1>);
   else if (g.ares)
     kern = assign_kernel<1, true, 1, true, kAresCS>;
   else

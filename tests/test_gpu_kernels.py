@@ -110,7 +110,7 @@ def test_assign_parity(dev, N, d, K, dtype, ld):
 MULTI_TILE_CASES = [
     ("f32", 256, 64, True, 128),     # three split products, one N-chunk
     ("f32", 256, 64, False, 128),    # fp32 rows split inside the kernel
-    ("f32", 200, 600, True, 128),    # three split products, lean scan over three N-chunks
+    ("f32", 200, 600, True, 128),    # three split products, top-three scan over three N-chunks
     ("bf16", 256, 1024, True, 128),  # resident rows, four 256-centre N-chunks (the K = 4096, d = 256 kernel)
     ("bf16", 512, 520, True, 256),   # two row tiles per centre stage, lean scan
     ("bf16", 1024, 256, True, 256),  # two row tiles per centre stage, one 512-column accumulator (K = 256)
@@ -281,15 +281,18 @@ def test_assign_duplicate_centres_and_zero_rows(dev):
     parity.check_assign(_host(X, "f32"), "f32", C.numpy(), lab, md, obj)
 
 
-@pytest.mark.parametrize("dtype,K,copies", [("f32", 24, 2), ("bf16", 24, 2), ("f32", 24, 3), ("bf16", 600, 2),
-                                            ("f32", 600, 3)])
-def test_assign_near_ties_are_rescored_exactly(dev, dtype, K, copies):
+@pytest.mark.parametrize("dtype,K,copies,N", [("f32", 24, 2, 3000), ("bf16", 24, 2, 3000), ("f32", 24, 3, 3000),
+                                              ("bf16", 600, 2, 3000), ("f32", 600, 3, 3000), ("f32", 600, 2, 40000),
+                                              ("f32", 600, 3, 40000)])
+def test_assign_near_ties_are_rescored_exactly(dev, dtype, K, copies, N):
     """Groups of centres 1e-5 apart make most rows near ties: the exact re-score decides them.
 
-    Two copies exercise the two-candidate re-score, three the all-K one; K = 600
-    (three N-chunks) exercises the lean scan, whose near ties all go to all K.
+    Two copies exercise the two-candidate re-score, three the all-K one.  K = 600
+    (three N-chunks) on 3000 rows spreads the chunks over CTAs, whose lean scan
+    sends every near tie to all K; on 40000 fp32 rows the split kernel's
+    top-three scan sends two-candidate near ties to the pair re-score.
     """
-    N, d = 3000, 256
+    d = 256
     base = K // copies
     X = _mixture(N, d, min(base, 64), dtype, seed=21 + K)
     C = hme_synth.random_centroids(K, d, seed=4, scale=3.0)
