@@ -87,7 +87,7 @@ struct AssignParams {
   // `slices` CTAs of cps chunks each; each writes its row states to part and
   // assign_merge_kernel finishes the rows
   int slices, cps;
-  float4 *part;     // [N][slices]: best, runner-up, best's index (bits)
+  float4 *part;     // [N][slices]: best, runner-up, third bound, centres of best and runner-up (bits)
 };
 
 constexpr uint32_t kWhereProducer = 1, kWhereMma = 2, kWhereMmaAcc = 3, kWhereEpi = 4, kWhereXchg = 6;
@@ -212,6 +212,34 @@ __device__ __forceinline__ void insert_top3(float v, int i, float &b1, float &b2
 // within E (or, in the lean scan, whenever the runner-up is).  Returns the
 // row's share of the objective estimate (0 for queued rows: the re-score adds
 // theirs).
+// Merge of two lean row states, each (b1, i1): best value and its centre,
+// b2: the exact runner-up value, i2: its centre or -1 when unknown, b3: a
+// lower bound of the third smallest value.  The best is the lexicographic
+// minimum over (value, centre); the runner-up is the loser's best, whose
+// centre is known, when that is below the winner's runner-up -- and the third
+// is then min(winner's b2, loser's b2) exactly -- else the winner's runner-up
+// (its centre as the winner knew it) with third >= min(winner's b3, loser's b1).
+// A fresh lean scan state is (b1, i1, b2, -1, b2).
+__device__ __forceinline__ void lean_merge(float &b1, int &i1, float &b2, int &i2, float &b3, float c1, int j1,
+                                           float c2, int j2, float c3) {
+  const bool other = c1 < b1 || (c1 == b1 && j1 < i1);
+  const float w2 = other ? c2 : b2, w3 = other ? c3 : b3, l1 = other ? b1 : c1, l2 = other ? b2 : c2;
+  const int wk = other ? j2 : i2, li = other ? i1 : j1;
+  if (other) {
+    b1 = c1;
+    i1 = j1;
+  }
+  if (l1 < w2) {
+    b2 = l1;
+    i2 = li;
+    b3 = fminf(w2, l2);
+  } else {
+    b2 = w2;
+    i2 = wk;
+    b3 = fminf(w3, l1);
+  }
+}
+
 template <bool LEAN>
 __device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row, float xr, float best1, float best2,
                                              float best3, int idx1, int idx2, float cn_max, float sqrt_cn_max) {
@@ -226,7 +254,9 @@ __device__ __forceinline__ double finish_row(const AssignParams &p, int64_t row,
                   p.err_ll * sqrt_xr * sqrt_cn_max;
   const bool near2 = (best2 < INFINITY) && ((D2 - D1) <= E);
   if (!near2) return (double)md;
-  const bool near3 = LEAN || ((best3 < INFINITY) && ((D3 - D1) <= E));
+  // lean scan: two candidates only when the runner-up's centre is known and
+  // the third value's lower bound is beyond E
+  const bool near3 = (LEAN && idx2 < 0) || ((best3 < INFINITY) && ((D3 - D1) <= E));
   if (near3) {
     const uint32_t slot = atomicAdd(&p.hdr->rescore_full_count, 1u);
     p.full_rows[slot] = (int32_t)row;
@@ -557,11 +587,10 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
         if (lane == 0) mbar_arrive(smem_u32(&tempty[a]));
       }
       if (!ok) break;
-      if (LEAN) {  // merge the two lean states: lowest value, then lowest index
-        const bool take_b = lb1 < best1 || (lb1 == best1 && li1 < idx1);
-        best2 = fminf(fmaxf(best1, lb1), fminf(best2, lb2));
-        best1 = take_b ? lb1 : best1;
-        idx1 = take_b ? li1 : idx1;
+      if (LEAN) {  // merge the two lean states (even and odd 16-column groups)
+        idx2 = -1;
+        best3 = best2;
+        lean_merge(best1, idx1, best2, idx2, best3, lb1, li1, lb2, -1, lb2);
       } else if (T3) {  // merge the two top-three states
         insert_top3(lb1, li1, best1, best2, best3, idx1, idx2);
         insert_top3(lb2, li2, best1, best2, best3, idx1, idx2);
@@ -578,9 +607,10 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
             ok = false;
             break;
           }
-          // indices < 2^16 (K <= 16384): both fit one word
-          xs[(half - 1) * 32] =
-              make_float4(best1, best2, best3, __uint_as_float((uint32_t)idx1 | ((uint32_t)idx2 << 16)));
+          // indices < 2^16 (K <= 16384): both fit one word (an unknown lean
+          // runner-up centre, -1, as 0xffff)
+          xs[(half - 1) * 32] = make_float4(
+              best1, best2, best3, __uint_as_float((uint32_t)idx1 | (((uint32_t)idx2 & 0xffffu) << 16)));
           mbar_arrive(smem_u32(&xfull[b]));
           continue;
         }
@@ -592,18 +622,17 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
 #pragma unroll
         for (int h = 0; h < CS - 1; ++h) os[h] = xs[h * 32];
         mbar_arrive(smem_u32(&xempty[b]));
-        // The merged result is the lexicographic minimum over (value, index)
-        // and the smallest remaining values: independent of the merge order.
+        // The merged best is the lexicographic minimum over (value, index)
+        // and the runner-up the smallest remaining value: independent of the
+        // merge order.  (Whether the lean runner-up's centre is known depends
+        // on it; that only chooses between the pair and the all-K re-score.)
 #pragma unroll
         for (int h = 0; h < CS - 1; ++h) {
           const float4 o = os[h];
           const uint32_t oi = __float_as_uint(o.w);
           const int o1 = (int)(oi & 0xffffu), o2 = (int)(oi >> 16);
           if (LEAN) {
-            const bool take_o = o.x < best1 || (o.x == best1 && o1 < idx1);
-            best2 = fminf(fmaxf(best1, o.x), fminf(best2, o.y));
-            best1 = take_o ? o.x : best1;
-            idx1 = take_o ? o1 : idx1;
+            lean_merge(best1, idx1, best2, idx2, best3, o.x, o1, o.y, o2 == 0xffff ? -1 : o2, o.z);
           } else {
             // insert the other share's best two (value, then index) and its third value
             auto insert = [&](float v, int i) {
@@ -630,7 +659,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       if (p.slices > 1) {
         // a slice of the centres: its row state goes to assign_merge_kernel
         if (LEAN && row < p.N)
-          p.part[row * p.slices + slice] = make_float4(best1, best2, __int_as_float(idx1), 0.0f);
+          p.part[row * p.slices + slice] =
+              make_float4(best1, best2, best3, __uint_as_float((uint32_t)idx1 | (((uint32_t)idx2 & 0xffffu) << 16)));
       } else if (row < p.N) {
         obj += finish_row<LEAN>(p, row, xr, best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
       }
@@ -648,10 +678,12 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
   }
 }
 
-// Small batches: the row states of the centre slices (lean scan: best value,
-// runner-up value, best's index) merged per row -- a group of kMaxSlices lanes
-// per row, one slice each, merged by shuffles -- then the row finished as in
-// the assign kernel (label, distance, near-tie queue, objective).
+// Small batches: the lean row states of the centre slices (best value and
+// centre, runner-up value and centre if known, third-value bound) merged per
+// row -- a group of kMaxSlices lanes per row, one slice each, merged by
+// shuffles (lean_merge gives the same state whichever side it runs on) --
+// then the row finished as in the assign kernel (label, distance, near-tie
+// queues, objective).
 constexpr int kMergeRows = 256 / kMaxSlices;  // rows per block
 __global__ void __launch_bounds__(256) assign_merge_kernel(const AssignParams p) {
   static_assert(kMaxSlices <= 32 && (32 % kMaxSlices) == 0, "a row's slices fit one warp");
@@ -659,27 +691,29 @@ __global__ void __launch_bounds__(256) assign_merge_kernel(const AssignParams p)
   const float sqrt_cn_max = sqrtf(cn_max);
   const int g = threadIdx.x % kMaxSlices;  // slice of this lane
   const int64_t row = (int64_t)blockIdx.x * kMergeRows + threadIdx.x / kMaxSlices;
-  float best1 = INFINITY, best2 = INFINITY;
-  int idx1 = 0x7fffffff;
+  float best1 = INFINITY, best2 = INFINITY, best3 = INFINITY;
+  int idx1 = 0x7fffffff, idx2 = -1;
   if (row < p.N && g < p.slices) {
     const float4 v = p.part[row * p.slices + g];
+    const uint32_t ii = __float_as_uint(v.w);
     best1 = v.x;
     best2 = v.y;
-    idx1 = __float_as_int(v.z);
+    best3 = v.z;
+    idx1 = (int)(ii & 0xffffu);
+    idx2 = (ii >> 16) == 0xffffu ? -1 : (int)(ii >> 16);
   }
 #pragma unroll
   for (int o = kMaxSlices / 2; o > 0; o >>= 1) {
     const float o1 = __shfl_xor_sync(0xffffffffu, best1, o);
     const float o2 = __shfl_xor_sync(0xffffffffu, best2, o);
+    const float o3 = __shfl_xor_sync(0xffffffffu, best3, o);
     const int oi = __shfl_xor_sync(0xffffffffu, idx1, o);
-    const bool take = o1 < best1 || (o1 == best1 && oi < idx1);
-    best2 = fminf(fmaxf(best1, o1), fminf(best2, o2));
-    best1 = take ? o1 : best1;
-    idx1 = take ? oi : idx1;
+    const int ok = __shfl_xor_sync(0xffffffffu, idx2, o);
+    lean_merge(best1, idx1, best2, idx2, best3, o1, oi, o2, ok, o3);
   }
   double obj = 0.0;
   if (g == 0 && row < p.N)
-    obj = finish_row<true>(p, row, __ldg(p.xn + row), best1, best2, INFINITY, idx1, 0, cn_max, sqrt_cn_max);
+    obj = finish_row<true>(p, row, __ldg(p.xn + row), best1, best2, best3, idx1, idx2, cn_max, sqrt_cn_max);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) obj += __shfl_xor_sync(0xffffffffu, obj, o);
   if ((threadIdx.x & 31) == 0 && obj != 0.0) atomicAdd(&p.hdr->objective, obj);

@@ -283,14 +283,18 @@ def test_assign_duplicate_centres_and_zero_rows(dev):
 
 @pytest.mark.parametrize("dtype,K,copies,N", [("f32", 24, 2, 3000), ("bf16", 24, 2, 3000), ("f32", 24, 3, 3000),
                                               ("bf16", 600, 2, 3000), ("f32", 600, 3, 3000), ("f32", 600, 2, 40000),
-                                              ("f32", 600, 3, 40000)])
+                                              ("f32", 600, 3, 40000), ("bf16", 600, 2, 40000), ("bf16", 600, 3, 40000),
+                                              ("bf16", 1100, 2, 40000)])
 def test_assign_near_ties_are_rescored_exactly(dev, dtype, K, copies, N):
     """Groups of centres 1e-5 apart make most rows near ties: the exact re-score decides them.
 
     Two copies exercise the two-candidate re-score, three the all-K one.  K = 600
     (three N-chunks) on 3000 rows spreads the chunks over CTAs, whose lean scan
     sends every near tie to all K; on 40000 fp32 rows the split kernel's
-    top-three scan sends two-candidate near ties to the pair re-score.
+    top-three scan sends two-candidate near ties to the pair re-score; on 40000
+    bf16 rows the lean states name the runner-up's centre when it was another
+    state's best (columns in different 16-column groups or epilogue shares), and
+    those ties go to the pair re-score too.
     """
     d = 256
     base = K // copies
