@@ -150,6 +150,7 @@ Layout feature_layout(int64_t N, int d, int K, int dtype, int64_t kpp_m) {
   L.counts = take((size_t)K * 8);
   L.x2sum = take(8);
   L.delta_k = take((size_t)4 * K * 4 + 16);
+  L.delta_mat = take((size_t)delta_tiles(N) * 2 * K * 4);
   L.reseed = take((size_t)kMaxSms * 2 * 8 * 64 * 8);  // (2 blocks x 8 warps per SM) x 64 keys
   if (kpp_m > 0) {
     L.kpp_rows = take((size_t)kpp_m * 4);
@@ -657,7 +658,7 @@ int hme_update_centroids(const void *X, int64_t N, int32_t d, int64_t ldx, int32
   int32_t *dk = at<int32_t>(ws, L.delta_k);
   int32_t *fl = at<int32_t>(ws, L.flagged);  // int32[3N]; free while no assign is in flight on this ws
   DeltaScratch ds{dk, dk + K, dk + 2 * K, dk + 3 * K, reinterpret_cast<int64_t *>(dk + 4 * K),
-                  perm, slab, fl, fl + N, at<unsigned long long>(ws, L.reseed)};
+                  perm, slab, fl, fl + N, at<unsigned long long>(ws, L.reseed), at<int32_t>(ws, L.delta_mat)};
   HME_CUDA(launch_update(X, N, d, ldx, dtype, labels, prev_labels, perm, slab, hist, offs + K, mind, K, st, ds,
                          C_inout, counts_out, n_reseeded_out, hdr, s),
            "update: centres");
@@ -851,7 +852,7 @@ int hme_kmeans_stream(const void *X, int64_t N, int32_t d, int64_t ldx, int32_t 
   int32_t *dk = at<int32_t>(ws, L.delta_k);
   int32_t *fl = at<int32_t>(ws, L.flagged);
   DeltaScratch ds{dk, dk + K, dk + 2 * K, dk + 3 * K, reinterpret_cast<int64_t *>(dk + 4 * K),
-                  perm, slab, fl, fl + chunk, at<unsigned long long>(ws, L.reseed)};
+                  perm, slab, fl, fl + chunk, at<unsigned long long>(ws, L.reseed), at<int32_t>(ws, L.delta_mat)};
 
   // copies of chunk j + 1 run on their own stream while chunk j is clustered
   cudaStream_t cs = nullptr;

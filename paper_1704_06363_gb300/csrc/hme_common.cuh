@@ -94,6 +94,7 @@ struct Layout {
   size_t counts;    // i64[K]: per-cluster counts (kept between centre updates)
   size_t x2sum;     // f64: sum of ||x||^2 (kept between centre updates)
   size_t delta_k;   // int32[4K] + int64[2]: counts, cursors and totals of the incremental update
+  size_t delta_mat; // int32[delta_tiles(N) * 2K]: its per-tile counts
   size_t reseed;    // u64[64 * selecting warps]: re-seed candidate keys
   size_t kpp_rows;  // int32[m]
   size_t kpp_d2;    // f64[m]
@@ -179,7 +180,10 @@ struct DeltaScratch {
   int64_t *totals;               // int64[2]: rows to add, rows to subtract
   int32_t *add_rows, *add_lab, *sub_rows, *sub_lab;  // int32[N] each
   unsigned long long *cand;      // re-seed candidates: 64 keys per selecting warp
+  int32_t *mat;                  // int32[delta_tiles(N) * 2K]: changed rows per (tile, bucket)
 };
+// Row tiles of the incremental update's count and fill (at most 304).
+int64_t delta_tiles(int64_t N);
 // prev_labels == nullptr: full pass (perm / sorted_labels / hist / valid_total
 // from the partition of labels); otherwise an incremental update from the
 // state left by a call with prev_labels.

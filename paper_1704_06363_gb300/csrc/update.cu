@@ -212,33 +212,23 @@ __global__ void __launch_bounds__(kUpdThreads) update_sums_kernel(const void *__
 }
 
 // Incremental update, in three small kernels over the label vectors:
-//   delta_count  rows whose label changed, counted per new label (to add) and
-//                per old label (to subtract), warp-aggregated (warps with no
-//                change skip); labels outside [0, K) count as unassigned on
-//                either side;
-//   delta_scan   exclusive prefix of both counts -> fill cursors and totals;
-//                also moves n_k by (added - subtracted);
-//   delta_fill   the changed rows grouped by label (order inside a group is
-//                irrelevant for sums), as (row, label) lists;
+//   delta_count  the rows are cut into ntiles contiguous tiles, one block
+//                each; a block counts its rows whose label changed per new
+//                label (to add) and per old label (to subtract) in shared
+//                memory (labels outside [0, K) count as unassigned on either
+//                side) and writes its row of the ntiles x 2K count matrix;
+//   delta_colscan for each of the 2K counts, the exclusive prefix over the
+//                tiles and the total (hist_add, hist_sub);
+//   delta_scan   exclusive prefix of both totals -> the lists' bucket starts
+//                and the list lengths; also moves n_k by (added - subtracted);
+//   delta_fill   a block takes slots from shared cursors (bucket start +
+//                earlier tiles' rows of the bucket): the changed rows grouped
+//                by label (order inside a group is irrelevant for sums), as
+//                (row, label) lists;
 // then one sums launch runs over both lists (added, then subtracted).
-// Warp-aggregated increment: lanes with the same key (found with one ballot
-// per key bit, keys in [0, 2^nbits)) add once, by the lowest lane, and each
-// lane gets its own slot (base + rank among equal keys).  Aggregation keeps
-// the atomics on K hot counters from serialising when many rows move.
-__device__ __forceinline__ int32_t warp_add(int32_t *ctr, int key, bool active, int nbits) {
-  unsigned peers = __ballot_sync(0xffffffffu, active);
-  for (int b = 0; b < nbits; ++b) {
-    const bool bit = (key >> b) & 1;
-    const unsigned m = __ballot_sync(0xffffffffu, bit);
-    peers &= bit ? m : ~m;
-  }
-  const int lane = threadIdx.x & 31;
-  const int leader = active ? __ffs(peers) - 1 : lane;
-  int32_t base = 0;
-  if (active && lane == leader) base = atomicAdd(ctr + key, __popc(peers));
-  base = __shfl_sync(0xffffffffu, base, leader);
-  return base + __popc(peers & ((1u << lane) - 1u));
-}
+constexpr int kDeltaThreads = 512;
+constexpr int64_t kDeltaTile = 16384;  // rows per tile at least (tiles: at most kDeltaTiles)
+constexpr int kDeltaTiles = 304;
 
 // Labels i .. i+VEC-1 of both vectors (16-byte loads when VEC == 4); entries
 // past N read as -1 on both sides (unchanged).
@@ -260,34 +250,49 @@ __device__ __forceinline__ void load_pair(const int32_t *labels, const int32_t *
 }
 
 template <int VEC>
-__global__ void __launch_bounds__(256) delta_count_kernel(const int32_t *__restrict__ labels,
-                                                          const int32_t *__restrict__ prev, int64_t N, int K,
-                                                          int nbits, int32_t *hist_add, int32_t *hist_sub,
-                                                          Header *hdr) {
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
+__global__ void __launch_bounds__(kDeltaThreads) delta_count_kernel(const int32_t *__restrict__ labels,
+                                                                    const int32_t *__restrict__ prev, int64_t N,
+                                                                    int K, int64_t tile, int32_t *__restrict__ mat,
+                                                                    Header *hdr) {
+  extern __shared__ int32_t dh[];  // [0, K): to add; [K, 2K): to subtract
+  for (int k = threadIdx.x; k < 2 * K; k += kDeltaThreads) dh[k] = 0;
+  __syncthreads();
+  const int64_t t0 = (int64_t)blockIdx.x * tile, t1 = min(N, t0 + tile);
   bool bad = false;
-  // whole warps iterate together (the loop bound is rounded up to a warp)
-  const int64_t Nw = (N + 32 * VEC - 1) / (32 * VEC) * (32 * VEC);
-  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VEC; i < Nw; i += stride) {
+  for (int64_t i = t0 + (int64_t)threadIdx.x * VEC; i < t1; i += (int64_t)kDeltaThreads * VEC) {
     int a[VEC], b[VEC];
-    load_pair<VEC>(labels, prev, i, N, a, b);
-    bool any = false;
+    load_pair<VEC>(labels, prev, i, t1, a, b);
 #pragma unroll
     for (int e = 0; e < VEC; ++e) {
-      if (i + e < N && (a[e] < 0 || a[e] >= K)) bad = true;
-      if (a[e] < 0 || a[e] >= K) a[e] = -1;
-      if (b[e] < 0 || b[e] >= K) b[e] = -1;
-      any |= a[e] != b[e];
-    }
-    if (!__any_sync(0xffffffffu, any)) continue;  // nothing moved in this warp's span
-#pragma unroll
-    for (int e = 0; e < VEC; ++e) {
-      const bool moved = a[e] != b[e];
-      warp_add(hist_add, a[e], moved && a[e] >= 0, nbits);
-      warp_add(hist_sub, b[e], moved && b[e] >= 0, nbits);
+      if (i + e < t1 && (a[e] < 0 || a[e] >= K)) bad = true;
+      const int na = (a[e] >= 0 && a[e] < K) ? a[e] : -1;
+      const int nb = (b[e] >= 0 && b[e] < K) ? b[e] : -1;
+      if (na != nb) {
+        if (na >= 0) atomicAdd(&dh[na], 1);
+        if (nb >= 0) atomicAdd(&dh[K + nb], 1);
+      }
     }
   }
   if (bad) atomicOr(&hdr->status, (uint32_t)kStatusBadLabel);
+  __syncthreads();
+  int32_t *row = mat + (int64_t)blockIdx.x * 2 * K;
+  for (int k = threadIdx.x; k < 2 * K; k += kDeltaThreads) row[k] = dh[k];
+}
+
+// For every column c of the ntiles x 2K count matrix: the exclusive prefix
+// over the tiles in place, the column total to hist[c] (hist_add then
+// hist_sub, adjacent).
+__global__ void __launch_bounds__(256) delta_colscan_kernel(int32_t *__restrict__ mat, int64_t ntiles, int K,
+                                                            int32_t *__restrict__ hist) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= 2 * K) return;
+  int32_t run = 0;
+  for (int64_t t = 0; t < ntiles; ++t) {
+    const int32_t v = mat[t * 2 * K + c];
+    mat[t * 2 * K + c] = run;
+    run += v;
+  }
+  hist[c] = run;
 }
 
 // Exclusive prefix of hist_add and hist_sub (one block), the fill cursors,
@@ -340,37 +345,40 @@ __global__ void __launch_bounds__(1024) delta_scan_kernel(const int32_t *__restr
 }
 
 template <int VEC>
-__global__ void __launch_bounds__(256) delta_fill_kernel(const int32_t *__restrict__ labels,
-                                                         const int32_t *__restrict__ prev, int64_t N, int K,
-                                                         int nbits, int32_t *cur_add, int32_t *cur_sub,
-                                                         int32_t *add_rows,
-                                                         int32_t *add_lab, int32_t *sub_rows, int32_t *sub_lab) {
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x * VEC;
-  const int64_t Nw = (N + 32 * VEC - 1) / (32 * VEC) * (32 * VEC);
-  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VEC; i < Nw; i += stride) {
+__global__ void __launch_bounds__(kDeltaThreads) delta_fill_kernel(const int32_t *__restrict__ labels,
+                                                                   const int32_t *__restrict__ prev, int64_t N,
+                                                                   int K, int64_t tile,
+                                                                   const int32_t *__restrict__ mat,
+                                                                   const int32_t *__restrict__ cur_add,
+                                                                   const int32_t *__restrict__ cur_sub,
+                                                                   int32_t *add_rows, int32_t *add_lab,
+                                                                   int32_t *sub_rows, int32_t *sub_lab) {
+  extern __shared__ int32_t dc[];  // this tile's next slot of each list bucket: [0, K) add, [K, 2K) subtract
+  const int32_t *row = mat + (int64_t)blockIdx.x * 2 * K;
+  for (int k = threadIdx.x; k < K; k += kDeltaThreads) {
+    dc[k] = cur_add[k] + row[k];
+    dc[K + k] = cur_sub[k] + row[K + k];
+  }
+  __syncthreads();
+  const int64_t t0 = (int64_t)blockIdx.x * tile, t1 = min(N, t0 + tile);
+  for (int64_t i = t0 + (int64_t)threadIdx.x * VEC; i < t1; i += (int64_t)kDeltaThreads * VEC) {
     int a[VEC], b[VEC];
-    load_pair<VEC>(labels, prev, i, N, a, b);
-    bool any = false;
+    load_pair<VEC>(labels, prev, i, t1, a, b);
 #pragma unroll
     for (int e = 0; e < VEC; ++e) {
-      if (a[e] < 0 || a[e] >= K) a[e] = -1;
-      if (b[e] < 0 || b[e] >= K) b[e] = -1;
-      any |= a[e] != b[e];
-    }
-    if (!__any_sync(0xffffffffu, any)) continue;
-#pragma unroll
-    for (int e = 0; e < VEC; ++e) {
-      const bool moved = a[e] != b[e];
-      const bool add = moved && a[e] >= 0, sub = moved && b[e] >= 0;
-      const int32_t sa = warp_add(cur_add, a[e], add, nbits);  // order inside a group is irrelevant
-      const int32_t sb = warp_add(cur_sub, b[e], sub, nbits);
-      if (add) {
-        add_rows[sa] = (int32_t)(i + e);
-        add_lab[sa] = a[e];
-      }
-      if (sub) {
-        sub_rows[sb] = (int32_t)(i + e);
-        sub_lab[sb] = b[e];
+      const int na = (a[e] >= 0 && a[e] < K) ? a[e] : -1;
+      const int nb = (b[e] >= 0 && b[e] < K) ? b[e] : -1;
+      if (na != nb) {
+        if (na >= 0) {
+          const int32_t sa = atomicAdd(&dc[na], 1);
+          add_rows[sa] = (int32_t)(i + e);
+          add_lab[sa] = na;
+        }
+        if (nb >= 0) {
+          const int32_t sb = atomicAdd(&dc[K + nb], 1);
+          sub_rows[sb] = (int32_t)(i + e);
+          sub_lab[sb] = nb;
+        }
       }
     }
   }
@@ -754,6 +762,17 @@ cudaError_t launch_update_add(const void *X, int64_t n, int d, int64_t ldx, int 
   return cudaGetLastError();
 }
 
+// Rows per tile of the incremental update: at most kDeltaTiles tiles of at
+// least kDeltaTile rows, a multiple of 4 (tiles start on 16-byte boundaries of
+// aligned labels).
+int64_t delta_tile_len(int64_t N) {
+  int64_t tile = (N + kDeltaTiles - 1) / kDeltaTiles;
+  if (tile < kDeltaTile) tile = kDeltaTile;
+  return (tile + 3) / 4 * 4;
+}
+
+int64_t delta_tiles(int64_t N) { return N > 0 ? (N + delta_tile_len(N) - 1) / delta_tile_len(N) : 1; }
+
 cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtype, const int32_t *labels,
                           const int32_t *prev_labels, const int32_t *perm, const int32_t *sorted_labels,
                           const int64_t *hist, const int64_t *valid_total, const float *mind, int K,
@@ -773,33 +792,27 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
                     st.sums, st.x2sum, false, s);
   } else if (N > 0) {
     // incremental: only the rows whose label changed
-    e = cudaMemsetAsync(ds.hist_add, 0, (size_t)2 * K * sizeof(int32_t), s);  // hist_add, hist_sub adjacent
-    if (e != cudaSuccess) return e;
+    const int64_t tile = delta_tile_len(N);
+    const int64_t ntiles = (N + tile - 1) / tile;
     const bool vec = (reinterpret_cast<uintptr_t>(labels) & 15u) == 0 &&
                      (reinterpret_cast<uintptr_t>(prev_labels) & 15u) == 0;
-    const int per = vec ? 4 : 1;
-    int64_t blocks = (int64_t)num_sms() * 8;
-    const int64_t want = (N + 256 * per - 1) / (256 * per);
-    if (blocks > want) blocks = want;
-    int nbits = 0;
-    while ((1 << nbits) < K) ++nbits;
-    if (vec)
-      delta_count_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.hist_add,
-                                                             ds.hist_sub, hdr);
-    else
-      delta_count_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.hist_add,
-                                                             ds.hist_sub, hdr);
+    const size_t smem = (size_t)2 * K * sizeof(int32_t);
+    auto count = vec ? delta_count_kernel<4> : delta_count_kernel<1>;
+    auto fill = vec ? delta_fill_kernel<4> : delta_fill_kernel<1>;
+    if (smem > 48 * 1024) {
+      e = cudaFuncSetAttribute(count, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+      e = cudaFuncSetAttribute(fill, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+    }
+    count<<<(unsigned)ntiles, kDeltaThreads, smem, s>>>(labels, prev_labels, N, K, tile, ds.mat, hdr);
+    delta_colscan_kernel<<<(unsigned)((2 * K + 255) / 256), 256, 0, s>>>(ds.mat, ntiles, K, ds.hist_add);
     delta_scan_kernel<<<1, 1024, 0, s>>>(ds.hist_add, ds.hist_sub, K, ds.cur_add, ds.cur_sub, ds.totals, st.counts,
                                          hdr);
-    if (vec)
-      delta_fill_kernel<4><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.cur_add,
-                                                            ds.cur_sub, ds.add_rows, ds.add_lab, ds.sub_rows,
-                                                            ds.sub_lab);
-    else
-      delta_fill_kernel<1><<<(unsigned)blocks, 256, 0, s>>>(labels, prev_labels, N, K, nbits, ds.cur_add,
-                                                            ds.cur_sub, ds.add_rows, ds.add_lab, ds.sub_rows,
-                                                            ds.sub_lab);
-    count_launch(3);
+    fill<<<(unsigned)ntiles, kDeltaThreads, smem, s>>>(labels, prev_labels, N, K, tile, ds.mat, ds.cur_add,
+                                                        ds.cur_sub, ds.add_rows, ds.add_lab, ds.sub_rows,
+                                                        ds.sub_lab);
+    count_launch(4);
     launch_sums_any(X, N, d, ldx, dtype,
                     SumsLists{ds.add_rows, ds.add_lab, ds.totals + 0, ds.sub_rows, ds.sub_lab, ds.totals + 1},
                     st.sums, st.x2sum, true, s);
