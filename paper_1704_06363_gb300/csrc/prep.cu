@@ -144,6 +144,37 @@ __global__ void __launch_bounds__(256) prep_bf16_kernel(const __nv_bfloat16 *__r
   const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const int d8 = d >> 3;  // ldx % 8 == 0 and a 16-byte aligned base are checked on the host
+  if (d8 <= 32 && 8 * d8 == d) {
+    // at most one 16-byte vector per lane and row: four rows in flight per
+    // warp (the same per-row arithmetic as the general loop below)
+    for (int64_t r0 = w0; r0 < N; r0 += 4 * nw) {
+      uint4 u[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t row = r0 + k * nw;
+        u[k] = make_uint4(0u, 0u, 0u, 0u);
+        if (row < N && lane < d8)
+          asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                       : "=r"(u[k].x), "=r"(u[k].y), "=r"(u[k].z), "=r"(u[k].w)
+                       : "l"(X + row * ldx + 8 * lane));
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int64_t row = r0 + k * nw;
+        const __nv_bfloat162 *h2 = reinterpret_cast<const __nv_bfloat162 *>(&u[k]);
+        float s = 0.0f;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float2 f = __bfloat1622float2(h2[t]);
+          s = fmaf(f.x, f.x, s);
+          s = fmaf(f.y, f.y, s);
+        }
+        s = warp_sum(s);
+        if (lane == 0 && row < N) xn[row] = s;
+      }
+    }
+    return;
+  }
   for (int64_t row = w0; row < N; row += nw) {
     const __nv_bfloat16 *xr = X + row * ldx;
     float s = 0.0f;
