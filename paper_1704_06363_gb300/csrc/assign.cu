@@ -428,7 +428,19 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
     // ---------------- MMA issuer ----------------
     if (lane == 0) {
       const uint32_t idesc = TF32 ? idesc_tf32_f32(kBM, (uint32_t)p.BN) : idesc_bf16_f32(kBM, (uint32_t)p.BN);
-      uint32_t it = 0, acc_it = 0, tile_it = 0;
+      uint32_t tile_it = 0;
+      // Stage, accumulator buffer and their phases advance by counting, and
+      // the operand descriptors by adding to their start-address field (in
+      // 16-byte units: +2 per 16-element k-step; every offset here is a
+      // multiple of 1024 bytes and shared addresses stay below 2^18), so the
+      // one issuing thread spends few instructions per MMA.
+      int s = 0;
+      uint32_t ph = 0, a = 0, aph = 0;
+      const uint64_t ring_desc = smem_desc_sw128(ring);
+      const uint64_t ares_desc = smem_desc_sw128(ares);
+      const uint64_t boff0 = (uint64_t)(((ARES ? 0u : (uint32_t)(NOPS * MT) * p.a_bytes)) >> 4);
+      const uint64_t boff1 = boff0 + (uint64_t)(p.b_bytes >> 4);
+      const uint64_t abytes16 = (uint64_t)(p.a_bytes >> 4);
       bool ok = true;
       for (int item = blockIdx.x; item < p.num_tiles * p.slices && ok; item += gridDim.x, ++tile_it) {
         const int ch0 = (item % p.slices) * p.cps, ch1 = min(p.nchunks, ch0 + p.cps);
@@ -439,46 +451,51 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
           }
           tc_fence_after();
         }
-        for (int ch = ch0; ch < ch1 && ok; ++ch, ++acc_it) {
-          const uint32_t a = acc_it % (uint32_t)nbuf;
-          const uint32_t aph = (acc_it / (uint32_t)nbuf) & 1u;
+        for (int ch = ch0; ch < ch1 && ok; ++ch) {
           if (!mbar_wait_bounded(smem_u32(&tempty[a]), aph ^ 1u, p.limit_ns, p.hdr, kWhereMmaAcc)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t dt = tmem_base + a * p.acc_stride;
-          for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
-            const int s = it % S;
-            const uint32_t ph = (it / S) & 1u;
+          for (int kb = 0; kb < p.num_kb; ++kb) {
             if (!mbar_wait_bounded(smem_u32(&full[s]), ph, p.limit_ns, p.hdr, kWhereMma)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t st = ring + (uint32_t)s * p.stage_bytes;
+            const uint64_t st_desc = ring_desc + (uint64_t)(((uint32_t)s * p.stage_bytes) >> 4);
+            const uint64_t bd0 = st_desc + boff0, bd1 = st_desc + boff1;
 #pragma unroll
-            for (int k = 0; k < kBK / 16; ++k) {
-              const uint64_t bd0 = smem_desc_sw128(b_addr(0, st) + k * 32);
-              const uint64_t bd1 = NPROD == 3 ? smem_desc_sw128(b_addr(1, st) + k * 32) : 0;
+            for (int mt = 0; mt < MT; ++mt) {
+              const uint32_t dtm = dt + (uint32_t)(mt * p.BN);
+              const uint64_t ad0 = ARES ? ares_desc + (uint64_t)((mt * p.num_kb + kb) * NOPS) * abytes16
+                                        : st_desc + (uint64_t)mt * abytes16;
+              const uint64_t ad1 = ARES ? ad0 + abytes16 : st_desc + (uint64_t)(MT + mt) * abytes16;
 #pragma unroll
-              for (int mt = 0; mt < MT; ++mt) {
-                const uint32_t dtm = dt + (uint32_t)(mt * p.BN);
-                const uint64_t ad0 = smem_desc_sw128(a_addr(0, mt, kb, st) + k * 32);
+              for (int k = 0; k < kBK / 16; ++k) {
+                const uint64_t dk = (uint64_t)(2 * k);
                 if (TF32)
-                  tc_mma_tf32(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                  tc_mma_tf32(dtm, ad0 + dk, bd0 + dk, idesc, (kb > 0 || k > 0) ? 1u : 0u);
                 else
-                  tc_mma_bf16(dtm, ad0, bd0, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+                  tc_mma_bf16(dtm, ad0 + dk, bd0 + dk, idesc, (kb > 0 || k > 0) ? 1u : 0u);
                 if (NPROD == 3) {
-                  const uint64_t ad1 = smem_desc_sw128(a_addr(1, mt, kb, st) + k * 32);
-                  tc_mma_bf16(dtm, ad0, bd1, idesc, 1u);  // xh . cl
-                  tc_mma_bf16(dtm, ad1, bd0, idesc, 1u);  // xl . ch
+                  tc_mma_bf16(dtm, ad0 + dk, bd1 + dk, idesc, 1u);  // xh . cl
+                  tc_mma_bf16(dtm, ad1 + dk, bd0 + dk, idesc, 1u);  // xl . ch
                 }
               }
             }
             tc_commit(smem_u32(&empty[s]));  // frees the stage once these MMAs finish
+            if (++s == S) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
           if (ok) tc_commit(smem_u32(&tfull[a]));  // accumulators of buffer a are complete
+          if (++a == (uint32_t)nbuf) {
+            a = 0;
+            aph ^= 1u;
+          }
         }
         if (ARES && ok) tc_commit(smem_u32(a_empty));  // the resident A rows may be replaced
       }
