@@ -132,15 +132,16 @@ __device__ __forceinline__ void epilogue_group(const uint32_t (&r)[16], const fl
 }
 
 // Lean variant for many centres (several N-chunks): per column
-// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)), best =
-// min(best, v), and the best's column -- six instructions, no branches.  jl is
-// the column of the best within this group; i1 moves only if the group
-// improved the best, so ties keep the lowest index.
+// v = ||c||^2 - 2 x.c, then runner-up = min(runner-up, max(best, v)) and
+// best = min(best, v) -- three ALU instructions.  The best's column is found
+// only in a group that improved the best (after the first groups, rarely: a
+// warp-uniform branch), as the first column of the group equal to the new
+// best, so ties keep the lowest index.
 __device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float *cn16, int k0, float &b1, float &b2,
                                            int &i1) {
   const float4 *c4 = reinterpret_cast<const float4 *>(cn16);
   const float before = b1;
-  int jl = 0;
+  float v[16];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const float4 cc = c4[q];
@@ -148,13 +149,17 @@ __device__ __forceinline__ void lean_group(const uint32_t (&r)[16], const float 
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const int j = 4 * q + e;
-      const float v = fmaf(-2.0f, __uint_as_float(r[j]), cq[e]);
-      b2 = fminf(b2, fmaxf(b1, v));
-      jl = (v < b1) ? j : jl;
-      b1 = fminf(b1, v);
+      v[j] = fmaf(-2.0f, __uint_as_float(r[j]), cq[e]);
+      b2 = fminf(b2, fmaxf(b1, v[j]));
+      b1 = fminf(b1, v[j]);
     }
   }
-  i1 = (b1 < before) ? k0 + jl : i1;
+  if (b1 < before) {  // the first column of the group that holds the new best
+    int jl = 15;
+#pragma unroll
+    for (int j = 14; j >= 0; --j) jl = (v[j] == b1) ? j : jl;
+    i1 = k0 + jl;
+  }
 }
 
 // Branch-free top three for many centres with tf32 operands (whose wider
