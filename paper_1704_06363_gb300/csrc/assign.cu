@@ -377,6 +377,8 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
       const uint64_t pol_a = l2_policy_evict_first();
       const uint64_t pol_b = l2_policy_evict_last();
       uint32_t it = 0, tile_it = 0;
+      int ps = 0;        // stage of iteration it
+      uint32_t pph = 0;  // and its phase
       bool ok = true, a_pending = false;
       for (int item = blockIdx.x; item < p.num_tiles * p.slices && ok; item += gridDim.x, ++tile_it) {
         const int tile = item / p.slices;
@@ -399,8 +401,13 @@ __global__ void __launch_bounds__(64 + 128 * MT * CS, 1)
         }
         for (int ch = ch0; ch < ch1 && ok; ++ch) {
           for (int kb = 0; kb < p.num_kb; ++kb, ++it) {
-            const int s = it % S;
-            const uint32_t ph = (it / S) & 1u;
+            // stage and phase of iteration it, by counting (no division)
+            const int s = ps;
+            const uint32_t ph = pph;
+            if (++ps == S) {
+              ps = 0;
+              pph ^= 1u;
+            }
             if (!mbar_wait_bounded(smem_u32(&empty[s]), ph ^ 1u, p.limit_ns, p.hdr, kWhereProducer)) {
               ok = false;
               break;
