@@ -1547,9 +1547,12 @@ int make_bf16_map(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols,
   return make_map(m, ptr, rows, cols, ld, box_rows);
 }
 
-// Epilogue warps per lane quarter of the resident-row kernel.  Two measured
-// 96 ms per assign at N = 5e7, d = 256, K = 4096; one 117 ms, four 104 ms.
-constexpr int kAresCS = 2;
+// Epilogue warps per lane quarter of the resident-row kernel.  On 8e6 rows of
+// the 5e7 x 256, K = 4096 set, with the lean MMA issue loop: four 12.58 ms,
+// two 12.84 ms (when the MMA thread still spent many instructions per MMA,
+// two had been the fastest: the epilogue warps sharing its sub-partition
+// took its issue slots).
+constexpr int kAresCS = 4;
 
 int launch_assign(const void *Xa, const void *Xb, int64_t N, int64_t lda, const AssignGeom &g, const void *chi,
                   const __nv_bfloat16 *clo, const float *cn, const float *xn, int32_t *labels, float *mind,
