@@ -280,9 +280,8 @@ HME_API int hme_partition(const int32_t *labels, int64_t N, int32_t K, int64_t *
  * launches are replayed as one CUDA graph captured at that second call (the
  * data behind the pointers may change freely between calls; it is read when
  * the graph runs).  Up to 8 argument sets are kept, the least recently used
- * replaced; a kept graph belongs to the CUDA context it was captured in (after
- * cudaDeviceReset, set HME_NO_GRAPHS or change an argument).  The environment
- * variable HME_NO_GRAPHS=1 turns this off.
+ * replaced; a kept graph is used only in the CUDA context it was captured in.
+ * The environment variable HME_NO_GRAPHS=1 turns this off.
  * Errors: HME_EINVAL for sizes outside the limits, a NULL or misaligned Q, a
  * NULL C or offsets_out, a NULL expert_out / order_out with B > 0, unknown or
  * conflicting flags; HME_ENOMEM for a workspace smaller than

@@ -378,6 +378,7 @@ int check_pca(const void *X, int64_t N, int d, int64_t ldx, int dtype, int r, in
 // the arguments only, never on the data, which the kernels read when they
 // run.  The first call with a given set of arguments runs directly (a batch
 // routed once pays no capture); a capture that fails leaves that set direct.
+// The CUDA context is part of the key (a graph cannot outlive its context).
 constexpr int64_t kGraphRows = 16384;
 constexpr int kGraphSlots = 8;
 struct RouteKey {
@@ -396,10 +397,11 @@ struct RouteKey {
   size_t ws_bytes;
   void *stream;
   int device = 0;
+  void *context = nullptr;  // a graph belongs to the context it was captured in
   bool operator==(const RouteKey &o) const {
     return Q == o.Q && B == o.B && d == o.d && ldq == o.ldq && dtype == o.dtype && C == o.C && K == o.K &&
            flags == o.flags && expert == o.expert && offsets == o.offsets && order == o.order && ws == o.ws &&
-           ws_bytes == o.ws_bytes && stream == o.stream && device == o.device;
+           ws_bytes == o.ws_bytes && stream == o.stream && device == o.device && context == o.context;
   }
 };
 struct RouteGraph {
@@ -422,6 +424,8 @@ int graph_route(RouteKey key, Body &&body, cudaStream_t s) {
     return e && *e && *e != '0';
   }();
   if (off || cudaGetDevice(&key.device) != cudaSuccess || key.device < 0 || key.device >= 64) return body(s);
+  key.context = current_context_handle();
+  if (!key.context) return body(s);
   std::unique_lock<std::mutex> lk(g_rg_mu);
   RouteGraph *slot = nullptr;
   for (auto &g : g_rg)

@@ -182,6 +182,8 @@ struct DeltaScratch {
   unsigned long long *cand;      // re-seed candidates: 64 keys per selecting warp
   int32_t *mat;                  // int32[delta_tiles(N) * 2K]: changed rows per (tile, bucket)
 };
+// The calling thread's current CUDA context (NULL if none or unavailable).
+void *current_context_handle();
 // Row tiles of the incremental update's count and fill (at most 304).
 int64_t delta_tiles(int64_t N);
 // prev_labels == nullptr: full pass (perm / sorted_labels / hist / valid_total

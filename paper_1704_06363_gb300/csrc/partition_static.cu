@@ -58,6 +58,18 @@ CtxGetCurrentFn ctx_get_current_fn() {
   return fn;
 }
 
+}  // namespace
+
+// The calling thread's current CUDA context (NULL if none or unavailable).
+void *current_context_handle() {
+  CtxGetCurrentFn get = ctx_get_current_fn();
+  CUcontext ctx = nullptr;
+  if (!get || get(&ctx) != CUDA_SUCCESS) return nullptr;
+  return ctx;
+}
+
+namespace {
+
 // Device address of g_partition_scratch in the current device's context (set
 // up on the first call in that context).
 int static_scratch(void **out) {
