@@ -1335,39 +1335,49 @@ __global__ void __launch_bounds__(256) rescore_row_kernel(const void *__restrict
 }
 
 // Exact re-score of near-tie rows against all K centres: a small tiled
-// "distance GEMM" on the CUDA cores.  A work item is 32 queued rows and one
-// slice of the centres, walked 64 centres and 32 dimensions at a time through
-// shared memory; thread (ty, tx) of a 16 x 16 grid owns rows {ty, ty+16} and
-// centres {tx, tx+16, tx+32, tx+48}.  sum_j (x_j - c_j)^2 is formed in fp32
-// per 32-wide chunk and the chunk sums are added in fp32 (relative error below
-// (32 + d/32) 2^-24, all terms non-negative).  With many queued rows a slice
-// is all K centres; with few (a small routed batch) the centres are split
-// over the blocks so that the work still spreads over the GPU.  A slice's best
-// (distance, centre) per row is merged with a 64-bit atomicMin on
-// (distance bits << 32 | centre): the distances are non-negative, so their
-// bit patterns order like the values, and equal distances keep the lower
-// centre.  rescore_full_finish_kernel then writes labels, distances and the
-// objective.
+// "distance GEMM" on the CUDA cores.  A work item is 16 x RPT queued rows and
+// one slice of the centres, walked 64 centres and 32 dimensions at a time
+// through shared memory (rows row-major; centres dimension-major, so that a
+// thread reads its four centres with one 16-byte load; with CV the centres
+// come from global memory in 16-byte loads with the lanes along the centres,
+// so that the transposing stores hit distinct banks).  Thread (ty, tx) of a
+// 16 x 16 grid owns rows ty + 16i (i < RPT) and centres 4tx .. 4tx+3: 4 RPT
+// distances for RPT + 1 shared loads per dimension.  RPT is 4 (64-row items)
+// or 2 (32-row items, twice as many), whichever is estimated to finish first:
+// a long queue runs faster in the larger tile, a short one (a small routed
+// batch) in more, smaller items.  sum_j (x_j - c_j)^2 is formed in fp32 per
+// 32-wide chunk (j ascending) and the chunk sums are added in fp32 in chunk
+// order, whatever RPT (relative error below (32 + d/32) 2^-24, all terms
+// non-negative).  With many queued rows a slice is all K centres; with few the
+// centres are split over the blocks so that the work still spreads over the
+// GPU.  A slice's best (distance, centre) per row is merged with a 64-bit
+// atomicMin on (distance bits << 32 | centre): the distances are non-negative,
+// so their bit patterns order like the values, and equal distances keep the
+// lower centre.  rescore_full_finish_kernel then writes labels, distances and
+// the objective.
 //
 // The keys of queued row f sit at full_keys_end[-1 - f]: the 8-byte aligned
 // tail of the pair queue (3 words per row of the call).  Rows queued for a
 // pair (3 words each) and for all K (2 words each) number at most N together,
 // so 3 pairs + 2 full <= 3N - full <= 3N - 1 words: the keys never reach a
 // queued pair.
-constexpr int kFR = 32, kFC = 64, kFD = 32;
+constexpr int kFRmax = 64, kFC = 64, kFD = 32;
 
-template <int DT>
-__global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
-                                                           const float *__restrict__ C, int K, const Header *hdr,
-                                                           const int32_t *__restrict__ full_rows,
-                                                           unsigned long long *full_keys_end) {
-  __shared__ float xs[kFR][kFD + 1];
-  __shared__ float cs[kFC][kFD + 1];
-  __shared__ float best_v[kFR];
-  __shared__ int best_k[kFR];
-  __shared__ int64_t rows[kFR];
+struct FullTiles {
+  float (*xs)[kFD + 1];   // [kFRmax][kFD + 1] rows
+  float (*cs)[kFC + 4];   // [kFD][kFC + 4] centres, dimension-major
+  float *best_v;          // [kFRmax]
+  int *best_k;            // [kFRmax]
+  int64_t *rows;          // [kFRmax]
+};
+
+template <int DT, bool CV, int RPT>
+__device__ __forceinline__ void rescore_full_body(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                  const float *__restrict__ C, int K, uint32_t count,
+                                                  const int32_t *__restrict__ full_rows,
+                                                  unsigned long long *full_keys_end, const FullTiles &sm) {
+  constexpr int kFR = 16 * RPT;
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-  const uint32_t count = *((volatile const uint32_t *)&hdr->rescore_full_count);
   const uint32_t ntiles = (count + kFR - 1) / kFR;
   const int kt = (K + kFC - 1) / kFC;  // tiles of kFC centres
   const int ks = (int)min((uint32_t)kt, max(1u, gridDim.x / max(ntiles, 1u)));  // slices per row tile
@@ -1378,17 +1388,21 @@ __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restric
     const int kbeg = (sl * kt / ks) * kFC, kend = min(K, ((sl + 1) * kt / ks) * kFC);
     const int nr = (int)min((uint32_t)kFR, count - b0);
     if (threadIdx.x < kFR) {
-      rows[threadIdx.x] = threadIdx.x < nr ? (int64_t)full_rows[b0 + threadIdx.x] : -1;
-      best_v[threadIdx.x] = INFINITY;
-      best_k[threadIdx.x] = 0;
+      sm.rows[threadIdx.x] = threadIdx.x < nr ? (int64_t)full_rows[b0 + threadIdx.x] : -1;
+      sm.best_v[threadIdx.x] = INFINITY;
+      sm.best_k[threadIdx.x] = 0;
     }
     __syncthreads();
     for (int k0 = kbeg; k0 < kend; k0 += kFC) {
-      float tot[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+      float tot[RPT][4];
+#pragma unroll
+      for (int i = 0; i < RPT; ++i)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tot[i][q] = 0.0f;
       for (int j0 = 0; j0 < d; j0 += kFD) {
         for (int e = threadIdx.x; e < kFR * kFD; e += 256) {
           const int r = e / kFD, j = e - r * kFD;
-          const int64_t row = rows[r];
+          const int64_t row = sm.rows[r];
           float x = 0.0f;
           if (row >= 0 && j0 + j < d) {
             if (DT == HME_BF16)
@@ -1396,46 +1410,75 @@ __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restric
             else
               x = reinterpret_cast<const float *>(Xv)[row * ldx + j0 + j];
           }
-          xs[r][j] = x;
+          sm.xs[r][j] = x;
         }
-        for (int e = threadIdx.x; e < kFC * kFD; e += 256) {
-          const int c = e / kFD, j = e - c * kFD;
-          const int k = k0 + c;
-          float v = 0.0f;
-          if (k < K && j0 + j < d) {
-            v = __ldg(C + (int64_t)k * d + j0 + j);
-            if (DT == HME_BF16) v = __bfloat162float(__float2bfloat16_rn(v));
+        if (CV) {  // 16-byte loads, lanes along the centres: conflict-free stores
+          for (int e = threadIdx.x; e < kFC * kFD / 4; e += 256) {
+            const int c = e % kFC, jq = 4 * (e / kFC);
+            const int k = k0 + c;
+            float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (k < K && j0 + jq < d) {  // d % 4 == 0: the whole vector is inside the row
+              v = __ldg(reinterpret_cast<const float4 *>(C + (int64_t)k * d + j0 + jq));
+              if (DT == HME_BF16) {
+                v.x = __bfloat162float(__float2bfloat16_rn(v.x));
+                v.y = __bfloat162float(__float2bfloat16_rn(v.y));
+                v.z = __bfloat162float(__float2bfloat16_rn(v.z));
+                v.w = __bfloat162float(__float2bfloat16_rn(v.w));
+              }
+            }
+            sm.cs[jq][c] = v.x;
+            sm.cs[jq + 1][c] = v.y;
+            sm.cs[jq + 2][c] = v.z;
+            sm.cs[jq + 3][c] = v.w;
           }
-          cs[c][j] = v;
+        } else {
+          for (int e = threadIdx.x; e < kFC * kFD; e += 256) {
+            const int c = e / kFD, j = e - c * kFD;
+            const int k = k0 + c;
+            float v = 0.0f;
+            if (k < K && j0 + j < d) {
+              v = __ldg(C + (int64_t)k * d + j0 + j);
+              if (DT == HME_BF16) v = __bfloat162float(__float2bfloat16_rn(v));
+            }
+            sm.cs[j][c] = v;
+          }
         }
         __syncthreads();
-        float part[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-#pragma unroll 8
-        for (int j = 0; j < kFD; ++j) {
-          const float x0 = xs[ty][j], x1 = xs[ty + 16][j];
+        float part[RPT][4];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float c = cs[tx + 16 * q][j];
-            const float t0 = x0 - c, t1 = x1 - c;
-            part[0][q] = fmaf(t0, t0, part[0][q]);
-            part[1][q] = fmaf(t1, t1, part[1][q]);
-          }
+        for (int i = 0; i < RPT; ++i)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) part[i][q] = 0.0f;
+#pragma unroll 4
+        for (int j = 0; j < kFD; ++j) {
+          float x[RPT];
+#pragma unroll
+          for (int i = 0; i < RPT; ++i) x[i] = sm.xs[ty + 16 * i][j];
+          const float4 c4 = *reinterpret_cast<const float4 *>(&sm.cs[j][4 * tx]);
+          const float c[4] = {c4.x, c4.y, c4.z, c4.w};
+#pragma unroll
+          for (int i = 0; i < RPT; ++i)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const float t = x[i] - c[q];
+              part[i][q] = fmaf(t, t, part[i][q]);
+            }
         }
 #pragma unroll
-        for (int r = 0; r < 2; ++r)
+        for (int i = 0; i < RPT; ++i)
 #pragma unroll
-          for (int q = 0; q < 4; ++q) tot[r][q] += part[r][q];
+          for (int q = 0; q < 4; ++q) tot[i][q] += part[i][q];
         __syncthreads();
       }
 #pragma unroll
-      for (int r = 0; r < 2; ++r) {
+      for (int i = 0; i < RPT; ++i) {
         float v = INFINITY;
         int kk = 0x7fffffff;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const int k = k0 + tx + 16 * q;
-          if (k < K && tot[r][q] < v) {
-            v = tot[r][q];
+          const int k = k0 + 4 * tx + q;
+          if (k < K && tot[i][q] < v) {
+            v = tot[i][q];
             kk = k;
           }
         }
@@ -1448,21 +1491,48 @@ __global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restric
             kk = ok;
           }
         }
-        const int rl = ty + 16 * r;
-        if (tx == 0 && (v < best_v[rl] || (v == best_v[rl] && kk < best_k[rl]))) {
-          best_v[rl] = v;
-          best_k[rl] = kk;
+        const int rl = ty + 16 * i;
+        if (tx == 0 && (v < sm.best_v[rl] || (v == sm.best_v[rl] && kk < sm.best_k[rl]))) {
+          sm.best_v[rl] = v;
+          sm.best_k[rl] = kk;
         }
       }
     }
     __syncthreads();
     if (threadIdx.x < nr) {
       const unsigned long long key =
-          ((unsigned long long)__float_as_uint(best_v[threadIdx.x]) << 32) | (uint32_t)best_k[threadIdx.x];
+          ((unsigned long long)__float_as_uint(sm.best_v[threadIdx.x]) << 32) | (uint32_t)sm.best_k[threadIdx.x];
       atomicMin(&full_keys_end[-1 - (int64_t)(b0 + threadIdx.x)], key);
     }
     __syncthreads();
   }
+}
+
+template <int DT, bool CV>
+__global__ void __launch_bounds__(256) rescore_full_kernel(const void *__restrict__ Xv, int d, int64_t ldx,
+                                                           const float *__restrict__ C, int K, const Header *hdr,
+                                                           const int32_t *__restrict__ full_rows,
+                                                           unsigned long long *full_keys_end) {
+  __shared__ float xs[kFRmax][kFD + 1];
+  __shared__ __align__(16) float cs[kFD][kFC + 4];
+  __shared__ float best_v[kFRmax];
+  __shared__ int best_k[kFRmax];
+  __shared__ int64_t rows[kFRmax];
+  const FullTiles sm{xs, cs, best_v, best_k, rows};
+  const uint32_t count = *((volatile const uint32_t *)&hdr->rescore_full_count);
+  // Estimated time (x gridDim) with each row tile: the larger of its longest
+  // work item and all its work spread over the blocks; a 64-row tile costs
+  // 1.6x a 32-row one (measured: 16 against 10).
+  const uint64_t kt = (uint64_t)((K + kFC - 1) / kFC), g = gridDim.x;
+  auto est = [&](uint64_t fr, uint64_t cost) -> uint64_t {
+    const uint64_t nt = (count + fr - 1) / fr;
+    const uint64_t ks = min(kt, max((uint64_t)1, g / max(nt, (uint64_t)1)));
+    return max((kt + ks - 1) / ks * cost * g, nt * kt * cost);
+  };
+  if (est(64, 16) < est(32, 10))
+    rescore_full_body<DT, CV, 4>(Xv, d, ldx, C, K, count, full_rows, full_keys_end, sm);
+  else
+    rescore_full_body<DT, CV, 2>(Xv, d, ldx, C, K, count, full_rows, full_keys_end, sm);
 }
 
 // The all-K re-score's result per queued row: label, distance, objective.
@@ -1790,8 +1860,10 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
       rescore_pair_kernel<HME_BF16, 1><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
     if (row_path)
       rescore_row_kernel<HME_BF16, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+    else if (cvec)
+      rescore_full_kernel<HME_BF16, true><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
     else
-      rescore_full_kernel<HME_BF16><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
+      rescore_full_kernel<HME_BF16, false><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   } else {
     if (al && d % 4 == 0 && ldx % 4 == 0)
       rescore_pair_kernel<HME_F32, 4><<<gpair, 256, 0, s>>>(X, d, ldx, C, labels, mind, hdr, flagged, keys_end);
@@ -1801,8 +1873,10 @@ cudaError_t launch_rescore(const void *X, int64_t N, int d, int64_t ldx, int dty
       rescore_row_kernel<HME_F32, 4><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
     else if (row_path)
       rescore_row_kernel<HME_F32, 1><<<grid, 256, row_smem, s>>>(X, d, ldx, C, K, labels, mind, hdr, full_rows);
+    else if (cvec)
+      rescore_full_kernel<HME_F32, true><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
     else
-      rescore_full_kernel<HME_F32><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
+      rescore_full_kernel<HME_F32, false><<<grid, 256, 0, s>>>(X, d, ldx, C, K, hdr, full_rows, keys_end);
   }
   if (!row_path) rescore_full_finish_kernel<<<gfin, 256, 0, s>>>(labels, mind, hdr, full_rows, keys_end);
   count_launch(row_path ? 2 : 3);

@@ -281,18 +281,40 @@ __global__ void __launch_bounds__(kDeltaThreads) delta_count_kernel(const int32_
 
 // For every column c of the ntiles x 2K count matrix: the exclusive prefix
 // over the tiles in place, the column total to hist[c] (hist_add then
-// hist_sub, adjacent).
-__global__ void __launch_bounds__(256) delta_colscan_kernel(int32_t *__restrict__ mat, int64_t ntiles, int K,
-                                                            int32_t *__restrict__ hist) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= 2 * K) return;
-  int32_t run = 0;
-  for (int64_t t = 0; t < ntiles; ++t) {
-    const int32_t v = mat[t * 2 * K + c];
-    mat[t * 2 * K + c] = run;
-    run += v;
+// hist_sub, adjacent).  A block takes 32 columns: warp w sums its strip of
+// about ntiles / 32 tiles (lane = column), one warp scans the 32 strip sums,
+// then every warp rewrites its strip from its strip's start.
+__global__ void __launch_bounds__(1024) delta_colscan_kernel(int32_t *__restrict__ mat, int64_t ntiles, int K,
+                                                             int32_t *__restrict__ hist) {
+  __shared__ int32_t part[32][33];
+  const int W = 2 * K;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int c = blockIdx.x * 32 + tx;
+  const int64_t R = (ntiles + 31) / 32;
+  const int64_t r0 = ty * R, r1 = min(ntiles, r0 + R);
+  int32_t sum = 0;
+  if (c < W)
+    for (int64_t t = r0; t < r1; ++t) sum += mat[t * W + c];
+  part[ty][tx] = sum;
+  __syncthreads();
+  if (ty == 0) {
+    int32_t run = 0;
+    for (int g = 0; g < 32; ++g) {
+      const int32_t v = part[g][tx];
+      part[g][tx] = run;
+      run += v;
+    }
+    if (c < W) hist[c] = run;
   }
-  hist[c] = run;
+  __syncthreads();
+  if (c < W) {
+    int32_t run = part[ty][tx];
+    for (int64_t t = r0; t < r1; ++t) {
+      const int32_t v = mat[t * W + c];
+      mat[t * W + c] = run;
+      run += v;
+    }
+  }
 }
 
 // Exclusive prefix of hist_add and hist_sub (one block), the fill cursors,
@@ -453,10 +475,17 @@ __device__ __forceinline__ unsigned long long reseed_key(const float *mind, int6
   return ((unsigned long long)__float_as_uint(v) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)i);
 }
 
-__device__ __forceinline__ int count_empty(const int64_t *counts, int K) {
+// Number of empty clusters, counted by the whole block (every thread must call
+// it; blockDim a multiple of 32); *acc is a shared-memory int it may overwrite.
+__device__ __forceinline__ int block_count_empty(const int64_t *counts, int K, int *acc) {
+  if (threadIdx.x == 0) *acc = 0;
+  __syncthreads();
   int e = 0;
-  for (int k = 0; k < K; ++k) e += counts[k] == 0;
-  return e;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) e += counts[k] == 0;
+  e = __reduce_add_sync(0xffffffffu, e);
+  if ((threadIdx.x & 31) == 0 && e != 0) atomicAdd(acc, e);
+  __syncthreads();
+  return *acc;
 }
 
 __global__ void __launch_bounds__(32 * kSelWarps) reseed_select_kernel(const float *__restrict__ mind, int64_t N,
@@ -464,9 +493,7 @@ __global__ void __launch_bounds__(32 * kSelWarps) reseed_select_kernel(const flo
                                                                        unsigned long long *cand) {
   __shared__ unsigned long long lists[kSelWarps][kReseedFast];
   __shared__ int E_s;
-  if (threadIdx.x == 0) E_s = count_empty(counts, K);
-  __syncthreads();
-  const int E = E_s;
+  const int E = block_count_empty(counts, K, &E_s);
   if (E == 0 || E > kReseedFast) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   unsigned long long *L = lists[warp];
@@ -509,9 +536,7 @@ __global__ void __launch_bounds__(1024) reseed_apply_kernel(const void *__restri
   __shared__ unsigned long long pick_key;
   __shared__ int pick_list;
   extern __shared__ int heads[];  // next position in each candidate list
-  if (threadIdx.x == 0) E_s = count_empty(counts, K);
-  __syncthreads();
-  const int E = E_s;
+  const int E = block_count_empty(counts, K, &E_s);
   if (E > kReseedFast) return;  // the general kernel handles it
   if (E == 0) {
     if (threadIdx.x == 0 && n_reseeded) *n_reseeded = 0;
@@ -806,7 +831,7 @@ cudaError_t launch_update(const void *X, int64_t N, int d, int64_t ldx, int dtyp
       if (e != cudaSuccess) return e;
     }
     count<<<(unsigned)ntiles, kDeltaThreads, smem, s>>>(labels, prev_labels, N, K, tile, ds.mat, hdr);
-    delta_colscan_kernel<<<(unsigned)((2 * K + 255) / 256), 256, 0, s>>>(ds.mat, ntiles, K, ds.hist_add);
+    delta_colscan_kernel<<<(unsigned)((2 * K + 31) / 32), 1024, 0, s>>>(ds.mat, ntiles, K, ds.hist_add);
     delta_scan_kernel<<<1, 1024, 0, s>>>(ds.hist_add, ds.hist_sub, K, ds.cur_add, ds.cur_sub, ds.totals, st.counts,
                                          hdr);
     fill<<<(unsigned)ntiles, kDeltaThreads, smem, s>>>(labels, prev_labels, N, K, tile, ds.mat, ds.cur_add,
