@@ -337,6 +337,57 @@ def test_small_batch_all_k_rescore_splits_the_centres(dev, dtype):
     parity.check_partition(dict(offsets=offs.cpu().numpy(), perm=order.cpu().numpy()), e, K)
 
 
+
+def _full_rescore_rows_per_item(count, K, grid):
+    """Rows per work item the all-K re-score picks for a queue of `count` rows:
+    the tile with the smaller estimate of max(longest item, all work / grid),
+    a 64-row tile costing 16 against 10 for a 32-row one."""
+    kt = -(-K // 64)
+
+    def est(fr, cost):
+        nt = -(-count // fr)
+        ks = min(kt, max(1, grid // max(nt, 1)))
+        return max(-(-kt // ks) * cost * grid, nt * kt * cost)
+
+    return 64 if est(64, 16) < est(32, 10) else 32
+
+
+@pytest.mark.parametrize("dtype,d,ld,K,N,rows_per_item", [("f32", 250, None, 4096, 8000, 64),
+                                                          ("bf16", 250, 256, 4096, 8000, 64),
+                                                          ("bf16", 256, None, 4096, 8000, 64),
+                                                          ("f32", 250, None, 600, 300, 32),
+                                                          ("bf16", 256, None, 4096, 200, 32)])
+def test_all_k_rescore_long_and_short_queues(dev, dtype, d, ld, K, N, rows_per_item):
+    """Three centres 1e-5 apart around every data row send nearly every row to
+    the all-K re-score.  A long queue runs in 64-row work items, a short one in
+    32-row items; d = 250 (centre rows not 16 bytes apart) stages the centres
+    one element at a time, d = 256 in 16-byte loads.  Labels, distances and the
+    objective match the oracle."""
+    copies = 3
+    base = K // copies
+    nb = min(base, N)  # data rows that become centres (with two copies each)
+    X = _mixture(N, d, min(base, 64), dtype, seed=91 + K + d, ld=ld)
+    C = hme_synth.random_centroids(K, d, seed=92, scale=3.0)
+    C[:nb] = X[:nb].float()
+    g = torch.Generator().manual_seed(93)
+    for r in range(1, copies):
+        C[r * base:r * base + nb] = C[:nb] + 1e-5 * torch.randn(nb, d, generator=g)
+    Xg = X.to(dev) if X.is_contiguous() else _to_dev_strided(X, dev)
+    dt = hme.HME_F32 if dtype == "f32" else hme.HME_BF16
+    ws = hme.workspace(hme.HME_OP_ASSIGN, N, d, K, dt, device=dev)
+    lab = torch.full((N,), -1, dtype=torch.int32, device=dev)
+    md = torch.empty(N, dtype=torch.float32, device=dev)
+    obj = torch.zeros(1, dtype=torch.float64, device=dev)
+    hme.hme_assign(Xg, C.to(dev), lab, ws, md, obj)
+    assert hme.hme_sync_status(ws) == hme.HME_OK
+    # workspace header, 32-bit words: [1] rows queued for a pair re-score, [3] for all K
+    all_k = int(ws[:16].view(torch.int32).cpu()[3])
+    assert all_k >= N // 2
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    assert _full_rescore_rows_per_item(all_k, K, 4 * sms) == rows_per_item  # the tile this case is for
+    st = parity.check_assign(_host(X, dtype), dtype, C.numpy(), lab.cpu().numpy(), md.cpu().numpy(), obj.item())
+    assert st["mismatches"] <= st["near_ties"]
+
 def test_route_reuses_prepared_features(dev):
     N, d, K = 4000, 128, 16
     X = _mixture(N, d, K, "f32", seed=8)
