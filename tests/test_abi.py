@@ -83,6 +83,37 @@ def test_host_validation_rejects_before_launch(lib):
                              None, None, p(256), ctypes.c_size_t(1 << 20), None) == 1
 
 
+
+def test_assign_rows_and_noalloc_partition_host_validation(lib):
+    """hme_assign_rows refuses row ranges outside [0, N), bad flags and missing
+    outputs, and hme_partition_noalloc refuses sizes outside its limits and
+    missing outputs, on the host before any CUDA call (no GPU here)."""
+    p, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    lib.hme_last_error.restype = ctypes.c_char_p
+    f = lib.hme_assign_rows
+    f.restype = ctypes.c_int
+    f.argtypes = [p, i64, i64, i64, i32, i64, i32, p, i32, i32, p, p, p, p, ctypes.c_size_t, p]
+    # X, N, row0, row1, d, ldx, dtype, C, K, flags, labels, mind, objective, ws, ws_bytes, stream
+    ok = [p(256), 100, 0, 100, 8, 8, 0, p(256), 4, 0, p(256), None, None, p(256), 1 << 30, None]
+    cases = [({2: -1}, 1, b"rows"), ({3: 101}, 1, b"rows"), ({2: 60, 3: 50}, 1, b"rows"),
+             ({9: 8}, 1, b"flags"), ({7: None}, 1, b"C"), ({10: None}, 1, b"labels_out"),
+             ({13: p(257)}, 1, b"aligned"), ({14: 16}, 2, b"")]
+    for change, code, word in cases:
+        args = list(ok)
+        for i, v in change.items():
+            args[i] = v
+        assert f(*args) == code, change
+        assert word in lib.hme_last_error(), change
+    g = lib.hme_partition_noalloc
+    g.restype = ctypes.c_int
+    g.argtypes = [p, i64, i32, p, p, p, p, p, p]
+    # labels, N, K, hist, offsets, perm, sorted labels, status, stream
+    ok = [p(256), 100, 4, p(256), p(256), p(256), None, None, None]
+    for i, bad in [(1, -1), (1, 2**31), (2, 0), (2, 16385), (3, None), (4, None), (0, None), (5, None)]:
+        args = list(ok)
+        args[i] = bad
+        assert g(*args) == 1, (i, bad)  # HME_EINVAL
+
 def test_product_path_has_no_oracle_import():
     """The product package never imports, links or runs the oracle."""
     pkg = os.path.join(ROOT, "paper_1704_06363_gb300")
